@@ -1,0 +1,343 @@
+#!/usr/bin/env python3
+"""Throughput of the SOMA SPSA training step on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+One step = one call of soma_spsa_step: for every expert and each of its n_pert
+probes, the antithetic forward passes of the whole byte-LSTM recurrence at
+theta +- eps z over the expert's batch, the per-pass mean cross entropy, the
+coefficients and the Philox-regenerating update.  The default workload is the
+SOMA N=2 configuration: 2 experts (E=64, H=960, 4,198,400 parameters each),
+64 probes, 32 sequences x 256 target bytes per expert, eps = lr = 1e-3.
+
+Prints ONE JSON line (rank 0).  `value` is perturbed LSTM tokens/s over all
+ranks (tokens/step = N_experts * 2 * n_pert * B * T per rank), inputs resident
+in HBM; `e2e` is the same metric through the public API with the step's bytes
+copied from pinned host memory and the losses read back inside the timed
+region.  With torchrun (N > 1) every rank steps its own independent set of
+experts (no collective on the data path: experts never exchange anything),
+so scaling is weak.  `--impl reference` times the fp64 CPU oracle on the
+host cores instead (rank 0 only), on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "perturbed LSTM tokens/s & SPSA steps/s per GB300; % of GEMM/HBM roofline"
+UNIT = "perturbed tokens/s"
+
+# DRAM traffic of one launch of the dominant kernel from an ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel
+# source it was taken on.
+TRAFFIC = {}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="soma_n2")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-seqs", type=int, default=32,
+                    help="sequences in the one-probe sample of the cpu_baseline timing")
+    ap.add_argument("--ref-sample-seqs", type=int, default=8,
+                    help="sequences per step of the --impl reference oracle run")
+    return ap.parse_args()
+
+
+def workload_desc(name, c):
+    from paper_2609_37899_gb300 import inputs
+    P = inputs.param_count(c["E"], c["H"])
+    return (f"{name}: {c['n_experts']} expert(s) x 1-layer byte LSTM (E={c['E']}, H={c['H']}, "
+            f"P={P:,}), n_pert={c['n_pert']}, eps={c['eps']}, lr={c['lr']}, "
+            f"B={c['batch']} x T={c['seq_len']} bytes per expert, order-{c['order']} "
+            f"Zipf(1.1) Markov clusters")
+
+
+def tokens_per_step(c):
+    return c["n_experts"] * 2 * c["n_pert"] * c["batch"] * c["seq_len"]
+
+
+def gate_flops_per_launch(c):
+    # one launch = one timestep of every (expert, probe, sign) lane:
+    # [B, E+H] x [E+H, 4H] per lane, 2 flops per multiply-add
+    return c["n_experts"] * c["n_pert"] * 2 * c["batch"] * 8 * c["H"] * (c["E"] + c["H"])
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons every 200 ms while running."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def cpu_baseline(cfg_name, c, n_seqs):
+    """The fp64 oracle, as it stands, on the host cores: one probe pair of
+    expert 0 over `n_seqs` of its sequences (both signs)."""
+    import oracle
+    from paper_2609_37899_gb300 import inputs
+    theta = inputs.config_params(cfg_name)[:1]
+    bx = inputs.config_batch(cfg_name)[:1, :n_seqs]
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    oracle.build()
+    t0 = time.perf_counter()
+    oracle.spsa_losses(theta, c["E"], c["H"], np.float32(c["eps"]), 0, 0, bx, probes=[0],
+                       n_threads=cores)
+    dt = time.perf_counter() - t0
+    toks = 2 * n_seqs * c["seq_len"]
+    return {"value": toks / dt, "unit": UNIT, "cores": min(cores, n_seqs), "kind": "oracle",
+            "sample": f"expert 0, probe 0, both signs, {n_seqs} of {c['batch']} sequences x "
+                      f"{c['seq_len']} bytes ({toks} perturbed tokens) in {dt:.2f} s; OpenMP "
+                      f"over sequences, so {min(cores, n_seqs)} of {cores} cores busy"}
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2609_37899_gb300 import inputs
+    c = inputs.CONFIGS[args.config]
+    n_seqs = min(args.ref_sample_seqs, c["batch"])
+    theta = inputs.config_params(args.config)
+    bx = inputs.config_batch(args.config)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    oracle.build()
+
+    def one(k):
+        e = k % c["n_experts"]
+        i = k % c["n_pert"]
+        oracle.spsa_losses(theta[e:e + 1], c["E"], c["H"], np.float32(c["eps"]), 0, 0,
+                           bx[e:e + 1, :n_seqs], probes=[i], n_threads=cores, first_expert=e)
+
+    for k in range(args.warmup):
+        one(k)
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        one(args.warmup + k)
+    dt = time.perf_counter() - t0
+    toks = 2 * n_seqs * c["seq_len"]
+    value = toks * args.steps / dt
+    sample = (f"per step one probe pair (both signs) of one expert over {n_seqs} of "
+              f"{c['batch']} sequences x {c['seq_len']} bytes = {toks} perturbed tokens")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_desc(args.config, c), "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": min(cores, n_seqs),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_37899_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def our_arm(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2609_37899_gb300 import api, build, inputs
+    if not os.path.exists(api.LIB_PATH):
+        build.build()
+    c = inputs.CONFIGS[args.config]
+    N, E, H, n, B, T = c["n_experts"], c["E"], c["H"], c["n_pert"], c["batch"], c["seq_len"]
+    K, W = args.steps, args.warmup
+    experts = api.SomaExperts(N, E, H, n, B, T, device=dev)
+    experts.init(seed=1000 + rank, std=c["init_std"] or 0.0)
+    # every step gets its own batch: W + K host batches, pinned, and their
+    # HBM-resident copies for the device-timed run
+    host = [torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=s)).pin_memory()
+            for s in range(W + K)]
+    resident = [h.to(dev) for h in host]
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for s in range(W):
+        experts.step(resident[s], c["eps"], c["lr"], 0, s)
+    barrier()
+    api.trace_enable(True)
+    api.trace_read(reset=True)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        start.record(stream)
+        for s in range(K):
+            experts.step(resident[W + s], c["eps"], c["lr"], 0, W + s)
+        stop.record(stream)
+        barrier()
+    api.trace_enable(False)
+    traced = api.trace_read(reset=True)
+    ms = start.elapsed_time(stop)
+    status = api.get_status()
+
+    # end to end through the public API: H2D of the step's bytes, the step,
+    # D2H of its losses, every step
+    losses_host = torch.empty(N, n, 2, dtype=torch.float32).pin_memory()
+    dev_bytes = torch.empty_like(resident[0])
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(K):
+        dev_bytes.copy_(host[W + s], non_blocking=True)
+        losses, _ = experts.step(dev_bytes, c["eps"], c["lr"], 0, W + K + s)
+        losses_host.copy_(losses, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    ms_e2e = e0.elapsed_time(e1)
+
+    if dist is not None:
+        t = torch.tensor([ms, ms_e2e], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, ms_e2e = float(t[0]), float(t[1])
+    if rank != 0:
+        dist.destroy_process_group()
+        return 0
+
+    tok = tokens_per_step(c) * world
+    value = tok * K / (ms / 1e3)
+    gate_ms, gate_n = traced["gate"]
+    peaks, peak_src = measured_peaks()
+    peak = peaks["bf16_tflops_sustained"]
+    achieved = gate_flops_per_launch(c) / (gate_ms / gate_n / 1e3) / 1e12 if gate_n else None
+    tr = TRAFFIC.get(args.config)
+    traffic = tr["bytes_per_launch"] if tr and tr.get("source_hash") == source_hash() else None
+    launches = sum(v[1] for v in traced.values())
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "steps_per_s": K / (ms / 1e3),
+        "config": {
+            "workload": workload_desc(args.config, c),
+            "tokens_per_step_per_gpu": tokens_per_step(c),
+            "l2": "inputs larger than L2: every step streams a "
+                  f"{experts.workspace.numel() / 2**30:.2f} GiB workspace through HBM",
+            "parallelism": f"experts batched in one launch per timestep; {world} independent "
+                           "replica(s), no collective",
+        },
+        "roofline": {
+            "bound": "tensor", "kernel": "gate_step_kernel (recurrent gate GEMM + cell)",
+            "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+            "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+            "peak_source": f"{peak_src} bf16 dense sustained (MEASURED_PEAKS.json)",
+            "flops_per_launch": gate_flops_per_launch(c), "launches": gate_n,
+            "kernel_ms_per_launch": gate_ms / gate_n if gate_n else None,
+            "share_of_step": gate_ms / ms if ms else None,
+        },
+        "kernel_ms": {k: v[0] / K for k, v in traced.items()},
+        "e2e": {"value": tok * K / (ms_e2e / 1e3), "unit": UNIT,
+                "h2d_bytes_per_step": int(resident[0].numel()),
+                "d2h_bytes_per_step": int(N * n * 2 * 4)},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+        "status": api.STATUS_NAMES.get(status, status),
+    }
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = cpu_baseline(args.config, c, min(args.cpu_sample_seqs, B))
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return reference_arm(args)
+    return our_arm(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,164 @@
+/*
+ * soma_api.h -- C ABI of libsoma.so: the SPSA training step of N independent
+ * byte-level LSTM experts on one GPU (SOMA, "Scaling Zero-Order Pretraining
+ * through Model Sharding").
+ *
+ * The library computes, for every expert e and probe i = 0..n_pert-1,
+ *   L+_{e,i} = L_e(theta_e + eps z_{e,i}),  L-_{e,i} = L_e(theta_e - eps z_{e,i})
+ * on one batch shared by every probe and both signs (Sec. 4, Eq. main-spsa),
+ * the coefficients c_{e,i} = (L+ - L-) / (2 eps), and the update
+ *   theta_e <- theta_e - lr * (1/n_pert) * sum_i c_{e,i} z_{e,i}
+ * (Eq. main-spsa inside the plain-SGD form of Eq. localspsa).  L is the mean
+ * next-byte cross entropy in nats/byte over all B*T targets (Table
+ * experimental-setup, "Evaluation protocol"), with the LSTM state reset to
+ * zero for every sequence.  Experts never interact: each has its own batch,
+ * probes and loss (Eq. separable-training-objective).
+ *
+ * Model of one expert (App. C, one LSTM layer instead of the paper's two
+ * residual blocks; every parameter is perturbed).  Flat fp32 parameter
+ * vector of P = V*E + 4H*E + 4H*H + 4H + V*H + V entries, in this order:
+ *   Emb[V][E], W_ih[4H][E], W_hh[4H][H], b[4H], W_out[V][H], b_out[V]
+ * row-major, gate blocks of W_ih, W_hh and b in the order i, f, g, o.
+ *   x_t = Emb[byte_t];  a = W_ih x_t + W_hh h_{t-1} + b
+ *   i,f,o = sigmoid(a_i,a_f,a_o); g = tanh(a_g); c_t = f c_{t-1} + i g;
+ *   h_t = o tanh(c_t);  logits = W_out h_t + b_out;
+ *   nll_t = logsumexp(logits) - logits[byte_{t+1}].
+ *
+ * Probes (dense Rademacher, Sec. 5 / App. F): z_{e,i}[p] in {-1,+1} for flat
+ * parameter index p, regenerated from Philox4x32-10 (Salmon et al., SC'11):
+ *   key = (seed & 0xffffffff, seed >> 32)
+ *   counter = (p >> 7, i, step & 0xffffffff, e)
+ *   bit = bit (p & 31) of output word ((p & 127) >> 5);  z = 1 - 2 bit.
+ * No probe is ever stored.
+ *
+ * Conventions for every entry point:
+ *  - Every buffer is owned by the caller.  Device pointers must point to
+ *    memory of the current device and be 16-byte aligned; the library never
+ *    allocates or frees.  Scratch memory is the caller's workspace, sized by
+ *    soma_workspace_bytes().
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Calls enqueue work on it and return without synchronising.
+ *  - Host-side argument errors return a soma_status code before anything is
+ *    enqueued.  Errors found on the device (a non-finite loss) are recorded
+ *    in a per-device status word read by soma_get_status().
+ *  - The library keeps no other state: no handle, no global RNG.  Calls on
+ *    different streams may run concurrently if their buffers are disjoint
+ *    (they share only the per-device status word).
+ */
+#ifndef SOMA_API_H
+#define SOMA_API_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Model sizes.  vocab must be 256 (one token per byte, App. C). */
+typedef struct soma_dims {
+  int32_t vocab;  /* V = 256 */
+  int32_t embed;  /* E, 1..1024 */
+  int32_t hidden; /* H, 1..4096 */
+} soma_dims;
+
+typedef enum soma_status {
+  SOMA_OK = 0,
+  SOMA_ERR_INVALID_ARG = 1, /* null or misaligned pointer, bad count/size/eps/lr */
+  SOMA_ERR_UNSUPPORTED = 2, /* dims outside the supported range */
+  SOMA_ERR_WORKSPACE = 3,   /* workspace NULL or smaller than soma_workspace_bytes() */
+  SOMA_ERR_CUDA = 4,        /* a CUDA launch or runtime call failed */
+  SOMA_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+  SOMA_ERR_NONFINITE = 6    /* a loss or coefficient was NaN or infinite */
+} soma_status;
+
+/* Number of parameters P of one expert (layout above); -1 if d is invalid. */
+int64_t soma_param_count(soma_dims d);
+
+/* Bytes of workspace that soma_spsa_step() and soma_eval_loss() need for
+ * these sizes (the larger of the two); 0 if the sizes are invalid. */
+size_t soma_workspace_bytes(soma_dims d, int n_experts, int n_pert, int batch, int seq_len);
+
+/* Deterministic initialisation of params [n_experts][P] (device, fp32) from
+ * Philox4x32-10 in a domain disjoint from the probes (counter word 3 has its
+ * top bit set).  std > 0: every parameter ~ N(0, std).  std == 0: Emb ~
+ * N(0, 0.1), W_ih and W_hh ~ N(0, 1/sqrt(E+H)), W_out ~ N(0, 1/sqrt(H)),
+ * biases 0.  Normals by the Box-Muller transform.  std < 0 is invalid. */
+int soma_init_experts(float* params, int n_experts, soma_dims d, uint64_t seed, float std,
+                      void* stream);
+
+/* One SPSA step for every expert (Eq. main-spsa).
+ *   params      device fp32 [n_experts][P]; updated in place.
+ *   n_pert      probes per expert, 1..12288.
+ *   eps, lr     probe radius (finite, >= 0) and learning rate (finite).
+ *               eps == 0 gives L+ = L- = L(theta), every coefficient 0 and
+ *               params unchanged; lr == 0 leaves params bit-unchanged.
+ *   seed, step  select the probes (see the header comment); the library
+ *               does not advance `step`.
+ *   byte_batch  device uint8 [n_experts][batch][seq_len + 1]: expert e's
+ *               sequences, shared by all its probes and both signs.
+ *   losses_out  device fp32 [n_experts][n_pert][2]: (L+, L-) in nats/byte.
+ *   coef_out    device fp32 [n_experts][n_pert] (L+ - L-)/(2 eps), or NULL.
+ *   workspace   device scratch of >= soma_workspace_bytes() bytes.
+ * Returns SOMA_OK once the work is enqueued. */
+int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float eps, float lr,
+                   uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
+                   int seq_len, float* losses_out, float* coef_out, void* workspace,
+                   size_t workspace_bytes, void* stream);
+
+/* Unperturbed mean loss L(theta_e) in nats/byte for every expert.
+ *   params [n_experts][P] and byte_batch [n_experts][batch][seq_len + 1] as
+ *   above; loss_out device fp32 [n_experts]. */
+int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_t* byte_batch,
+                   int batch, int seq_len, float* loss_out, void* workspace,
+                   size_t workspace_bytes, void* stream);
+
+/* The update alone, for given coefficients (the last part of Eq. main-spsa):
+ *   params[e] -= lr * (1/n_pert) * sum_i coef[e][i] z_{e,i}.
+ *   coef: device fp32 [n_experts][n_pert].  No workspace. */
+int soma_spsa_update(float* params, int n_experts, soma_dims d, int n_pert, float lr,
+                     uint64_t seed, uint64_t step, const float* coef, void* stream);
+
+/* Synchronises `stream`, then returns and clears the current device's status
+ * word (SOMA_OK if no device-side error was recorded since the last call).
+ * Returns SOMA_ERR_CUDA if the synchronisation itself failed. */
+int soma_get_status(void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* soma_status_string(int code);
+
+/* Tracing.  While enabled, every kernel that soma_spsa_step, soma_eval_loss
+ * and soma_spsa_update launch is bracketed by two CUDA events recorded on the
+ * caller's stream; soma_trace_read() waits for the recorded events and sums
+ * device time and launch counts per kernel class.  Tracing is process-wide
+ * and off by default; events are created on first use and reused. */
+enum {
+  SOMA_TRACE_GATE = 0,   /* recurrent gate GEMM + fused cell update, one launch per timestep */
+  SOMA_TRACE_HEAD = 1,   /* output head + log-softmax + NLL */
+  SOMA_TRACE_REDUCE = 2, /* loss and coefficient reduction */
+  SOMA_TRACE_UPDATE = 3, /* Philox-regenerating parameter update */
+  SOMA_TRACE_KINDS = 4
+};
+typedef struct soma_kernel_times {
+  double ms[SOMA_TRACE_KINDS];       /* summed device time per class */
+  int64_t launches[SOMA_TRACE_KINDS];
+} soma_kernel_times;
+int soma_trace_enable(int enable);
+/* reset != 0 also forgets the records that were read. */
+int soma_trace_read(soma_kernel_times* out, int reset);
+
+/* Test exports (bit-exactness of the generator the kernels use).
+ * soma_debug_philox: out4[j] = Philox4x32-10(ctr4[j], key = seed halves) for
+ *   j < count; ctr4 and out4 are device uint32 [count][4].
+ * soma_debug_rademacher: z_out[q] = z_{expert,pert}[p0 + q] for q < count,
+ *   device int8, using the same bit extraction the kernels use. */
+int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
+                      void* stream);
+int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
+                          int64_t count, int8_t* z_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SOMA_API_H */

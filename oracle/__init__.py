@@ -77,6 +77,7 @@ def _load():
                                     ctypes.c_int, c_dp, ctypes.c_int]
         lib.oracle_loss.restype = ctypes.c_double
         lib.oracle_spsa_losses.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_int,
                                            ctypes.c_double, ctypes.c_uint64, ctypes.c_uint64,
                                            c_u8p, ctypes.c_int, ctypes.c_int,
                                            ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
@@ -145,13 +146,15 @@ def loss(theta, E: int, H: int, bytes_, n_threads: int = 0, per_token: bool = Fa
 
 
 def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
-                probes=None, n_pert: int | None = None, n_threads: int = 0):
+                probes=None, n_pert: int | None = None, n_threads: int = 0,
+                first_expert: int = 0):
     """Antithetic losses and coefficients for the selected probes.
 
     theta [N, P] (fp32 or fp64), bytes_ [N, B, T+1] uint8.  ``probes`` lists
     the probe indices to evaluate (default: range(n_pert)).  ``eps`` is taken
     as given (pass np.float32 values to mirror the fp32 argument of the
-    product).  Returns (L [N, n_sel, 2] with L+ then L-, coef [N, n_sel])."""
+    product).  Row e of theta is expert ``first_expert + e`` (the expert index
+    keys its probes).  Returns (L [N, n_sel, 2] with L+ then L-, coef [N, n_sel])."""
     th = _f64(theta)
     N = th.shape[0]
     bx = _u8(bytes_)
@@ -162,7 +165,8 @@ def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
     sel = np.ascontiguousarray(list(probes), dtype=np.int32)
     L = np.zeros((N, sel.size, 2), dtype=np.float64)
     coef = np.zeros((N, sel.size), dtype=np.float64)
-    rc = _load().oracle_spsa_losses(_ptr(th, ctypes.c_double), N, E, H, float(eps), seed, step,
+    rc = _load().oracle_spsa_losses(_ptr(th, ctypes.c_double), N, first_expert, E, H, float(eps),
+                                    seed, step,
                                     _ptr(bx, ctypes.c_uint8), B, T,
                                     _ptr(sel, ctypes.c_int32), sel.size,
                                     _ptr(L, ctypes.c_double), _ptr(coef, ctypes.c_double),

@@ -217,10 +217,11 @@ double oracle_loss(const double* theta, int E, int H, const uint8_t* bytes,
 /* Antithetic losses of the selected probes.
  *   theta [N][P] (fp64), bytes [N][B][T+1] (one batch per expert, shared by
  *   every probe and both signs), sel[n_sel] probe indices in [0, n_pert).
+ *   Row e of theta is expert e0 + e (its index in the probe counter).
  *   out_L  [N][n_sel][2] = L(theta_e + eps z), L(theta_e - eps z)
  *   out_coef [N][n_sel]  = (L+ - L-) / (2 eps); 0 when eps == 0.
  * Returns 0 on success. */
-int oracle_spsa_losses(const double* theta, int N, int E, int H, double eps,
+int oracle_spsa_losses(const double* theta, int N, int e0, int E, int H, double eps,
                        uint64_t seed, uint64_t step, const uint8_t* bytes,
                        int B, int T, const int32_t* sel, int n_sel,
                        double* out_L, double* out_coef, int n_threads) {
@@ -234,7 +235,7 @@ int oracle_spsa_losses(const double* theta, int N, int E, int H, double eps,
     const uint8_t* bx = bytes + (int64_t)e * B * (T + 1);
     for (int q = 0; q < n_sel; ++q) {
       int i = sel[q];
-      oracle_rademacher(seed, step, (uint32_t)e, (uint32_t)i, 0, P, z);
+      oracle_rademacher(seed, step, (uint32_t)(e0 + e), (uint32_t)i, 0, P, z);
       double L[2];
       for (int s = 0; s < 2; ++s) {
         double sign = (s == 0) ? 1.0 : -1.0;

@@ -1,0 +1,227 @@
+"""ctypes binding of libsoma.so (the C ABI in include/soma_api.h).
+
+Argument marshalling only: every step of the SPSA path runs in the CUDA
+kernels behind the C ABI.  PyTorch supplies device memory and streams.  The
+library is loaded on first use; if it is missing this module raises -- there
+is no fallback of any kind.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libsoma.so")
+V = 256
+
+_lock = threading.Lock()
+_lib = None
+
+SOMA_OK = 0
+STATUS_NAMES = {0: "SOMA_OK", 1: "SOMA_ERR_INVALID_ARG", 2: "SOMA_ERR_UNSUPPORTED",
+                3: "SOMA_ERR_WORKSPACE", 4: "SOMA_ERR_CUDA", 5: "SOMA_ERR_TIMEOUT",
+                6: "SOMA_ERR_NONFINITE"}
+
+
+class SomaError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        self.code = code
+        super().__init__(f"{what}: {STATUS_NAMES.get(code, code)} ({status_string(code)})")
+
+
+class soma_dims(ctypes.Structure):
+    _fields_ = [("vocab", ctypes.c_int32), ("embed", ctypes.c_int32), ("hidden", ctypes.c_int32)]
+
+
+TRACE_KINDS = ("gate", "head", "reduce", "update")
+
+
+class soma_kernel_times(ctypes.Structure):
+    _fields_ = [("ms", ctypes.c_double * 4), ("launches", ctypes.c_int64 * 4)]
+
+
+def _sig(lib, name, res, args):
+    f = getattr(lib, name)
+    f.restype = res
+    f.argtypes = args
+
+
+def lib():
+    """The loaded libsoma.so; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libsoma.so not found at {LIB_PATH}: build it with "
+                               "`python -m paper_2609_37899_gb300.build`")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, sz, i32, i64, u64, f32 = (ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int,
+                                      ctypes.c_int64, ctypes.c_uint64, ctypes.c_float)
+        _sig(L, "soma_param_count", i64, [soma_dims])
+        _sig(L, "soma_workspace_bytes", sz, [soma_dims, i32, i32, i32, i32])
+        _sig(L, "soma_init_experts", i32, [vp, i32, soma_dims, u64, f32, vp])
+        _sig(L, "soma_spsa_step", i32, [vp, i32, soma_dims, i32, f32, f32, u64, u64, vp, i32,
+                                        i32, vp, vp, vp, sz, vp])
+        _sig(L, "soma_eval_loss", i32, [vp, i32, soma_dims, vp, i32, i32, vp, vp, sz, vp])
+        _sig(L, "soma_spsa_update", i32, [vp, i32, soma_dims, i32, f32, u64, u64, vp, vp])
+        _sig(L, "soma_get_status", i32, [vp])
+        _sig(L, "soma_status_string", ctypes.c_char_p, [i32])
+        _sig(L, "soma_trace_enable", i32, [i32])
+        _sig(L, "soma_trace_read", i32, [ctypes.POINTER(soma_kernel_times), i32])
+        _sig(L, "soma_debug_philox", i32, [u64, vp, vp, i32, vp])
+        _sig(L, "soma_debug_rademacher", i32, [u64, u64, i32, i32, i64, i64, vp, vp])
+        _lib = L
+        return L
+
+
+def status_string(code: int) -> str:
+    return lib().soma_status_string(code).decode()
+
+
+def dims(E: int, H: int) -> soma_dims:
+    return soma_dims(V, E, H)
+
+
+def _check(code: int, what: str):
+    if code != SOMA_OK:
+        raise SomaError(code, what)
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t: torch.Tensor, dtype, name: str, numel: int | None = None) -> ctypes.c_void_p:
+    if not t.is_cuda or t.dtype != dtype or not t.is_contiguous():
+        raise ValueError(f"{name}: expected a contiguous CUDA {dtype} tensor")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name}: expected {numel} elements, got {t.numel()}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def param_count(E: int, H: int) -> int:
+    return int(lib().soma_param_count(dims(E, H)))
+
+
+def workspace_bytes(E: int, H: int, n_experts: int, n_pert: int, batch: int, seq_len: int) -> int:
+    return int(lib().soma_workspace_bytes(dims(E, H), n_experts, n_pert, batch, seq_len))
+
+
+def alloc_workspace(E, H, n_experts, n_pert, batch, seq_len, device="cuda") -> torch.Tensor:
+    n = workspace_bytes(E, H, n_experts, n_pert, batch, seq_len)
+    if n == 0:
+        raise ValueError("invalid sizes for the workspace")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def init_experts(params: torch.Tensor, E: int, H: int, seed: int, std: float = 0.0, stream=None):
+    n_experts = params.shape[0]
+    _check(lib().soma_init_experts(_dev(params, torch.float32, "params",
+                                        n_experts * param_count(E, H)),
+                                   n_experts, dims(E, H), seed, std, _stream(stream)),
+           "soma_init_experts")
+
+
+def spsa_step(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int, n_pert: int,
+              eps: float, lr: float, seed: int, step: int, losses: torch.Tensor,
+              coef: torch.Tensor | None, workspace: torch.Tensor, stream=None):
+    """One SPSA step; params [N, P] fp32 updated in place, losses [N, n_pert, 2],
+    coef [N, n_pert] or None, byte_batch [N, B, T+1] uint8 (all on the device)."""
+    N, B, T1 = byte_batch.shape
+    P = param_count(E, H)
+    _check(lib().soma_spsa_step(
+        _dev(params, torch.float32, "params", N * P), N, dims(E, H), n_pert, eps, lr, seed, step,
+        _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
+        _dev(losses, torch.float32, "losses", N * n_pert * 2),
+        _dev(coef, torch.float32, "coef", N * n_pert) if coef is not None else None,
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_spsa_step")
+
+
+def eval_loss(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int,
+              loss_out: torch.Tensor, workspace: torch.Tensor, stream=None):
+    N, B, T1 = byte_batch.shape
+    _check(lib().soma_eval_loss(
+        _dev(params, torch.float32, "params", N * param_count(E, H)), N, dims(E, H),
+        _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
+        _dev(loss_out, torch.float32, "loss_out", N),
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_eval_loss")
+
+
+def spsa_update(params: torch.Tensor, E: int, H: int, lr: float, seed: int, step: int,
+                coef: torch.Tensor, stream=None):
+    N, n_pert = coef.shape
+    _check(lib().soma_spsa_update(
+        _dev(params, torch.float32, "params", N * param_count(E, H)), N, dims(E, H), n_pert,
+        lr, seed, step, _dev(coef, torch.float32, "coef", N * n_pert), _stream(stream)),
+        "soma_spsa_update")
+
+
+def trace_enable(on: bool = True):
+    _check(lib().soma_trace_enable(1 if on else 0), "soma_trace_enable")
+
+
+def trace_read(reset: bool = True) -> dict:
+    """{kind: (total_ms, launches)} of the traced launches (waits for them)."""
+    t = soma_kernel_times()
+    _check(lib().soma_trace_read(ctypes.byref(t), 1 if reset else 0), "soma_trace_read")
+    return {k: (t.ms[j], int(t.launches[j])) for j, k in enumerate(TRACE_KINDS)}
+
+
+def get_status(stream=None) -> int:
+    return int(lib().soma_get_status(_stream(stream)))
+
+
+def debug_philox(seed: int, counters: torch.Tensor, stream=None) -> torch.Tensor:
+    """Philox4x32-10 words [n, 4] (int32 bit patterns) for counters [n, 4] int32."""
+    n = counters.shape[0]
+    out = torch.empty_like(counters)
+    _check(lib().soma_debug_philox(seed, _dev(counters, torch.int32, "counters"),
+                                   _dev(out, torch.int32, "out"), n, _stream(stream)),
+           "soma_debug_philox")
+    return out
+
+
+def debug_rademacher(seed: int, step: int, expert: int, probe: int, p0: int, count: int,
+                     device="cuda", stream=None) -> torch.Tensor:
+    z = torch.empty(count, dtype=torch.int8, device=device)
+    _check(lib().soma_debug_rademacher(seed, step, expert, probe, p0, count,
+                                       _dev(z, torch.int8, "z"), _stream(stream)),
+           "soma_debug_rademacher")
+    return z
+
+
+class SomaExperts:
+    """N experts' parameters and scratch on the current GPU, stepped by the
+    C ABI.  Holds device tensors only; each call is one library call."""
+
+    def __init__(self, n_experts: int, E: int, H: int, n_pert: int, batch: int, seq_len: int,
+                 device="cuda"):
+        self.N, self.E, self.H = n_experts, E, H
+        self.n_pert, self.batch, self.seq_len = n_pert, batch, seq_len
+        self.P = param_count(E, H)
+        self.params = torch.zeros(n_experts, self.P, dtype=torch.float32, device=device)
+        self.workspace = alloc_workspace(E, H, n_experts, n_pert, batch, seq_len, device)
+        self.losses = torch.zeros(n_experts, n_pert, 2, dtype=torch.float32, device=device)
+        self.coef = torch.zeros(n_experts, n_pert, dtype=torch.float32, device=device)
+        self.loss = torch.zeros(n_experts, dtype=torch.float32, device=device)
+
+    def init(self, seed: int, std: float = 0.0, stream=None):
+        init_experts(self.params, self.E, self.H, seed, std, stream)
+
+    def step(self, byte_batch: torch.Tensor, eps: float, lr: float, seed: int, step: int,
+             stream=None):
+        spsa_step(self.params, byte_batch, self.E, self.H, self.n_pert, eps, lr, seed, step,
+                  self.losses, self.coef, self.workspace, stream)
+        return self.losses, self.coef
+
+    def eval(self, byte_batch: torch.Tensor, stream=None):
+        eval_loss(self.params, byte_batch, self.E, self.H, self.loss, self.workspace, stream)
+        return self.loss

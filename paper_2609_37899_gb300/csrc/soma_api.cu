@@ -1,0 +1,247 @@
+// soma_api.cu -- the C ABI of libsoma.so (declared in include/soma_api.h):
+// argument validation, workspace carving and the launch sequence of one SPSA
+// step (Eq. main-spsa): forward sweep over all (expert, probe, sign) lanes,
+// loss reduction into L+, L- and coefficients, Philox-regenerating update.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "soma_api.h"
+#include "soma_launch.h"
+
+using namespace soma;
+
+// Per-device status word (see soma_get_status).  Kernels get its address as
+// an argument; it is read and cleared only by soma_get_status.
+__device__ int g_soma_status = 0;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr int kMaxPert = 12 * 1024;  // coefficients of one expert staged in shared memory
+int* g_status_ptr[kMaxDevices] = {nullptr};
+
+int* status_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_soma_status) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = static_cast<int*>(p);
+  }
+  return g_status_ptr[dev];
+}
+
+bool dims_ok(const soma_dims& d) {
+  return d.vocab == kVocab && d.embed >= 1 && d.embed <= 1024 && d.hidden >= 1 &&
+         d.hidden <= 4096;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr size_t kAlign = 256;
+size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Workspace of one sweep with `n_pert` probes and `n_sign` signs.
+struct WsPlan {
+  int Tc;
+  size_t hist, cst, nll, coef, total;
+};
+
+WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T) {
+  Sweep s;
+  std::memset(&s, 0, sizeof(s));
+  s.lay = make_layout(d.embed, d.hidden);
+  s.n_experts = n_experts;
+  s.n_pert = n_pert;
+  s.n_sign = n_sign;
+  s.B = B;
+  s.T = T;
+  WsPlan w;
+  w.Tc = forward_hist_slots(s);
+  const size_t lanes = (size_t)s.lanes();
+  w.hist = round_up(lanes * w.Tc * B * (size_t)d.hidden * sizeof(float));
+  w.cst = round_up(lanes * B * (size_t)d.hidden * sizeof(float));
+  w.nll = round_up(lanes * B * (size_t)T * sizeof(float));
+  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
+  w.total = w.hist + w.cst + w.nll + w.coef;
+  return w;
+}
+
+ForwardBuffers carve(const WsPlan& w, void* ws) {
+  char* base = static_cast<char*>(ws);
+  ForwardBuffers fb;
+  fb.Tc = w.Tc;
+  fb.hist = reinterpret_cast<float*>(base);
+  fb.cst = reinterpret_cast<float*>(base + w.hist);
+  fb.nll = reinterpret_cast<float*>(base + w.hist + w.cst);
+  return fb;
+}
+
+float* coef_scratch(const WsPlan& w, void* ws) {
+  return reinterpret_cast<float*>(static_cast<char*>(ws) + w.hist + w.cst + w.nll);
+}
+
+bool sizes_ok(int n_experts, int n_pert, int batch, int seq_len) {
+  // lanes index the grid's x dimension and probe/expert indices fit Philox
+  // counter words (expert < 2^31 keeps the init domain disjoint)
+  if (n_experts < 1 || n_pert < 1 || batch < 1 || seq_len < 1) return false;
+  if (n_pert > kMaxPert) return false;
+  if ((int64_t)n_experts * n_pert * 2 > (int64_t)INT32_MAX) return false;
+  if ((int64_t)batch * (seq_len + 1) > (int64_t)INT32_MAX) return false;
+  return true;
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? SOMA_OK : SOMA_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int64_t soma_param_count(soma_dims d) {
+  if (!dims_ok(d)) return -1;
+  return make_layout(d.embed, d.hidden).P;
+}
+
+size_t soma_workspace_bytes(soma_dims d, int n_experts, int n_pert, int batch, int seq_len) {
+  if (!dims_ok(d) || !sizes_ok(n_experts, n_pert, batch, seq_len)) return 0;
+  const WsPlan step = plan_sweep(d, n_experts, n_pert, 2, batch, seq_len);
+  const WsPlan eval = plan_sweep(d, n_experts, 1, 1, batch, seq_len);
+  return step.total > eval.total ? step.total : eval.total;
+}
+
+int soma_init_experts(float* params, int n_experts, soma_dims d, uint64_t seed, float std,
+                      void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !aligned16(params) || n_experts < 1 || !(std >= 0.f) || !std::isfinite(std))
+    return SOMA_ERR_INVALID_ARG;
+  const Layout lay = make_layout(d.embed, d.hidden);
+  return cuda_status(launch_init(params, lay, n_experts, seed, std, (cudaStream_t)stream));
+}
+
+int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float eps, float lr,
+                   uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
+                   int seq_len, float* losses_out, float* coef_out, void* workspace,
+                   size_t workspace_bytes, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !byte_batch || !losses_out || !aligned16(params) ||
+      !sizes_ok(n_experts, n_pert, batch, seq_len) || !(eps >= 0.f) || !std::isfinite(eps) ||
+      !std::isfinite(lr))
+    return SOMA_ERR_INVALID_ARG;
+  const WsPlan w = plan_sweep(d, n_experts, n_pert, 2, batch, seq_len);
+  if (!workspace || !aligned16(workspace) || workspace_bytes < w.total) return SOMA_ERR_WORKSPACE;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+
+  Sweep s;
+  s.params = params;
+  s.bytes = byte_batch;
+  s.lay = make_layout(d.embed, d.hidden);
+  s.n_experts = n_experts;
+  s.n_pert = n_pert;
+  s.n_sign = 2;
+  s.B = batch;
+  s.T = seq_len;
+  s.eps = eps;
+  s.seed = seed;
+  s.step = step;
+  const ForwardBuffers fb = carve(w, workspace);
+  float* coef_ws = coef_scratch(w, workspace);
+
+  cudaError_t e = launch_forward_simt(s, fb, st);
+  if (e == cudaSuccess)
+    e = launch_reduce_losses(fb.nll, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
+                             coef_out, coef_ws, status, st);
+  // eps == 0 makes every coefficient 0 and lr == 0 every step 0: theta stays
+  // bit-identical, so the update is not launched at all.
+  if (e == cudaSuccess && eps != 0.f && lr != 0.f)
+    e = launch_spsa_update(params, s.lay, n_experts, n_pert, lr, seed, step, coef_ws, st);
+  return cuda_status(e);
+}
+
+int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_t* byte_batch,
+                   int batch, int seq_len, float* loss_out, void* workspace,
+                   size_t workspace_bytes, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !byte_batch || !loss_out || !aligned16(params) ||
+      !sizes_ok(n_experts, 1, batch, seq_len))
+    return SOMA_ERR_INVALID_ARG;
+  const WsPlan w = plan_sweep(d, n_experts, 1, 1, batch, seq_len);
+  if (!workspace || !aligned16(workspace) || workspace_bytes < w.total) return SOMA_ERR_WORKSPACE;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+  Sweep s;
+  s.params = params;
+  s.bytes = byte_batch;
+  s.lay = make_layout(d.embed, d.hidden);
+  s.n_experts = n_experts;
+  s.n_pert = 1;
+  s.n_sign = 1;
+  s.B = batch;
+  s.T = seq_len;
+  s.eps = 0.f;
+  s.seed = 0;
+  s.step = 0;
+  const ForwardBuffers fb = carve(w, workspace);
+  cudaError_t e = launch_forward_simt(s, fb, st);
+  if (e == cudaSuccess)
+    e = launch_reduce_losses(fb.nll, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
+                             nullptr, status, st);
+  return cuda_status(e);
+}
+
+int soma_spsa_update(float* params, int n_experts, soma_dims d, int n_pert, float lr,
+                     uint64_t seed, uint64_t step, const float* coef, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !coef || !aligned16(params) || n_experts < 1 || n_pert < 1 ||
+      n_pert > kMaxPert || !std::isfinite(lr))
+    return SOMA_ERR_INVALID_ARG;
+  if (lr == 0.f) return SOMA_OK;
+  const Layout lay = make_layout(d.embed, d.hidden);
+  return cuda_status(
+      launch_spsa_update(params, lay, n_experts, n_pert, lr, seed, step, coef, (cudaStream_t)stream));
+}
+
+int soma_get_status(void* stream) {
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return SOMA_ERR_CUDA;
+  int* p = status_ptr();
+  if (!p) return SOMA_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, p, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return SOMA_ERR_CUDA;
+  const int zero = 0;
+  if (cudaMemcpy(p, &zero, sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess)
+    return SOMA_ERR_CUDA;
+  return v;
+}
+
+const char* soma_status_string(int code) {
+  switch (code) {
+    case SOMA_OK: return "ok";
+    case SOMA_ERR_INVALID_ARG: return "invalid argument";
+    case SOMA_ERR_UNSUPPORTED: return "unsupported dimensions";
+    case SOMA_ERR_WORKSPACE: return "workspace missing or too small";
+    case SOMA_ERR_CUDA: return "CUDA error";
+    case SOMA_ERR_TIMEOUT: return "device-side wait timed out";
+    case SOMA_ERR_NONFINITE: return "non-finite loss or coefficient";
+    default: return "unknown status";
+  }
+}
+
+int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
+                      void* stream) {
+  if (!ctr4 || !out4 || count < 0) return SOMA_ERR_INVALID_ARG;
+  if (count == 0) return SOMA_OK;
+  return cuda_status(launch_debug_philox(seed, ctr4, out4, count, (cudaStream_t)stream));
+}
+
+int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
+                          int64_t count, int8_t* z_out, void* stream) {
+  if (!z_out || count < 0 || p0 < 0 || expert < 0 || pert < 0) return SOMA_ERR_INVALID_ARG;
+  if (count == 0) return SOMA_OK;
+  return cuda_status(
+      launch_debug_rademacher(seed, step, expert, pert, p0, count, z_out, (cudaStream_t)stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,146 @@
+// soma_device.cuh -- device helpers shared by the libsoma kernels: the
+// Philox4x32-10 probe generator, the parameter layout of one expert and the
+// argument blocks the host passes to the kernels.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace soma {
+
+constexpr int kVocab = 256;
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
+// 32x32 -> 64-bit products whose high halves are xor-ed into the other two
+// words with the round key; the key advances by the Weyl constants
+// (golden ratio, sqrt(3) - 1) after each round.
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ uint32_t mul_hi32(uint32_t a, uint32_t b) {
+#ifdef __CUDA_ARCH__
+  return __umulhi(a, b);
+#else
+  return (uint32_t)(((uint64_t)a * (uint64_t)b) >> 32);
+#endif
+}
+
+__host__ __device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo_a = 0xD2511F53u * ctr.x;
+    const uint32_t hi_a = mul_hi32(0xD2511F53u, ctr.x);
+    const uint32_t lo_b = 0xCD9E8D57u * ctr.z;
+    const uint32_t hi_b = mul_hi32(0xCD9E8D57u, ctr.z);
+    ctr = make_uint4(hi_b ^ ctr.y ^ k0, lo_b, hi_a ^ ctr.w ^ k1, lo_a);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return ctr;
+}
+
+__host__ __device__ __forceinline__ uint32_t word_of(const uint4& w, int j) {
+  return j == 0 ? w.x : (j == 1 ? w.y : (j == 2 ? w.z : w.w));
+}
+
+// Identity of one probe stream: z_{expert,probe} at update `step`.
+struct ProbeKey {
+  uint32_t k0, k1;   // seed halves
+  uint32_t step;     // low 32 bits of the update counter
+  uint32_t expert;   // counter word 3
+  uint32_t probe;    // counter word 1
+};
+
+__host__ __device__ __forceinline__ ProbeKey make_probe_key(uint64_t seed, uint64_t step,
+                                                             uint32_t expert, uint32_t probe) {
+  ProbeKey k;
+  k.k0 = (uint32_t)(seed & 0xffffffffu);
+  k.k1 = (uint32_t)(seed >> 32);
+  k.step = (uint32_t)(step & 0xffffffffu);
+  k.expert = expert;
+  k.probe = probe;
+  return k;
+}
+
+// The 128 probe bits of parameter block `blk` (parameters 128*blk .. +127).
+__host__ __device__ __forceinline__ uint4 probe_block(const ProbeKey& k, uint32_t blk) {
+  return philox4x32_10(make_uint4(blk, k.probe, k.step, k.expert), k.k0, k.k1);
+}
+
+// Bits of z for the 32 consecutive parameters p .. p+31: bit j set <=> z[p+j]
+// = -1.  One Philox call when the run stays inside one 128-parameter block,
+// two when it crosses into the next.
+__host__ __device__ __forceinline__ uint32_t probe_bits32(const ProbeKey& k, int64_t p) {
+  const uint32_t blk = (uint32_t)(p >> 7);
+  const int off = (int)(p & 127);
+  const int wi = off >> 5, sh = off & 31;
+  const uint4 a = probe_block(k, blk);
+  const uint32_t lo = word_of(a, wi);
+  if (sh == 0) return lo;
+  uint32_t hi;
+  if (wi < 3) {
+    hi = word_of(a, wi + 1);
+  } else {
+    hi = probe_block(k, blk + 1).x;
+  }
+  return (lo >> sh) | (hi << (32 - sh));
+}
+
+// w + s*eps*z for a z bit: the perturbed parameter in fp32.
+__host__ __device__ __forceinline__ float perturb(float w, uint32_t bit, float se) {
+  return w + (bit ? -se : se);
+}
+
+// ---------------------------------------------------------------------------
+// Parameter layout of one expert: Emb[V][E], W_ih[4H][E], W_hh[4H][H],
+// b[4H], W_out[V][H], b_out[V].
+// ---------------------------------------------------------------------------
+struct Layout {
+  int E, H;
+  int64_t emb, w_ih, w_hh, b, w_out, b_out, P;
+};
+
+__host__ __device__ inline Layout make_layout(int E, int H) {
+  Layout L;
+  L.E = E;
+  L.H = H;
+  L.emb = 0;
+  L.w_ih = L.emb + (int64_t)kVocab * E;
+  L.w_hh = L.w_ih + 4LL * H * E;
+  L.b = L.w_hh + 4LL * H * H;
+  L.w_out = L.b + 4LL * H;
+  L.b_out = L.w_out + (int64_t)kVocab * H;
+  L.P = L.b_out + kVocab;
+  return L;
+}
+
+// ---------------------------------------------------------------------------
+// One forward sweep over (expert, probe, sign) "lanes".  A lane is one
+// perturbed copy of one expert: lane = (e * n_pert + i) * n_sign + s, with
+// sign +1 for s = 0 and -1 for s = 1.  eval_loss is the sweep with
+// n_pert = n_sign = 1 and eps = 0.
+// ---------------------------------------------------------------------------
+struct Sweep {
+  const float* params;     // [N][P]
+  const uint8_t* bytes;    // [N][B][T+1]
+  Layout lay;
+  int n_experts, n_pert, n_sign;
+  int B, T;
+  float eps;
+  uint64_t seed, step;
+  __host__ __device__ int lanes() const { return n_experts * n_pert * n_sign; }
+};
+
+__host__ __device__ __forceinline__ void lane_parts(const Sweep& s, int lane, int& e, int& i,
+                                                    float& se) {
+  const int sgn = lane % s.n_sign;
+  const int ei = lane / s.n_sign;
+  i = ei % s.n_pert;
+  e = ei / s.n_pert;
+  se = sgn == 0 ? s.eps : -s.eps;
+}
+
+// Device status codes (mirror soma_status).
+constexpr int kStatusNonFinite = 6;
+constexpr int kStatusTimeout = 5;
+
+}  // namespace soma

@@ -1,0 +1,98 @@
+"""The C ABI library builds, loads and exports every declared symbol; host
+argument validation needs no GPU (no compute call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "soma_api.h")
+
+
+@pytest.fixture(scope="module")
+def soma():
+    from paper_2609_37899_gb300 import build
+    build.build()
+    from paper_2609_37899_gb300 import api
+    return api
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(soma_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for required in ["soma_init_experts", "soma_spsa_step", "soma_eval_loss",
+                     "soma_workspace_bytes", "soma_param_count", "soma_get_status",
+                     "soma_status_string", "soma_spsa_update", "soma_debug_philox",
+                     "soma_debug_rademacher"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(soma):
+    lib = ctypes.CDLL(soma.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_param_count_and_workspace(soma):
+    assert soma.param_count(32, 64) == 49_664
+    assert soma.param_count(64, 960) == 4_198_400
+    assert soma.param_count(32, 48) == 36_288
+    assert soma.lib().soma_param_count(soma.soma_dims(255, 32, 64)) == -1
+    assert soma.workspace_bytes(32, 64, 1, 8, 4, 64) > 0
+    assert soma.workspace_bytes(32, 64, 0, 8, 4, 64) == 0
+    assert soma.workspace_bytes(32, 64, 1, 0, 4, 64) == 0
+    # grows with every size it depends on
+    w = soma.workspace_bytes(64, 960, 2, 64, 32, 256)
+    assert soma.workspace_bytes(64, 960, 2, 64, 32, 512) > w
+    assert soma.workspace_bytes(64, 960, 2, 128, 32, 256) > w
+
+
+def test_status_strings(soma):
+    for code in range(7):
+        assert soma.status_string(code) != "unknown status"
+    assert soma.status_string(99) == "unknown status"
+
+
+def test_host_validation_rejects_before_launch(soma):
+    L = soma.lib()
+    d = soma.dims(32, 64)
+    fake = ctypes.c_void_p(0x10000)  # never dereferenced: validation fails first
+    ws = soma.workspace_bytes(32, 64, 1, 8, 4, 64)
+    # null params
+    assert L.soma_spsa_step(None, 1, d, 8, 1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, fake, ws,
+                            None) == 1
+    # misaligned params
+    assert L.soma_spsa_step(ctypes.c_void_p(0x10004), 1, d, 8, 1e-3, 1e-2, 0, 0, fake, 4, 64,
+                            fake, None, fake, ws, None) == 1
+    # negative / non-finite eps, non-finite lr
+    assert L.soma_spsa_step(fake, 1, d, 8, -1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, fake, ws,
+                            None) == 1
+    assert L.soma_spsa_step(fake, 1, d, 8, float("nan"), 1e-2, 0, 0, fake, 4, 64, fake, None,
+                            fake, ws, None) == 1
+    assert L.soma_spsa_step(fake, 1, d, 8, 1e-3, float("inf"), 0, 0, fake, 4, 64, fake, None,
+                            fake, ws, None) == 1
+    # bad dims
+    assert L.soma_spsa_step(fake, 1, soma.soma_dims(128, 32, 64), 8, 1e-3, 1e-2, 0, 0, fake, 4,
+                            64, fake, None, fake, ws, None) == 2
+    assert L.soma_spsa_step(fake, 1, soma.dims(32, 5000), 8, 1e-3, 1e-2, 0, 0, fake, 4, 64,
+                            fake, None, fake, ws, None) == 2
+    # zero sizes, too many probes
+    assert L.soma_spsa_step(fake, 0, d, 8, 1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, fake, ws,
+                            None) == 1
+    assert L.soma_spsa_step(fake, 1, d, 20000, 1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, fake,
+                            ws, None) == 1
+    # workspace too small or missing
+    assert L.soma_spsa_step(fake, 1, d, 8, 1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, fake,
+                            ws - 1, None) == 3
+    assert L.soma_spsa_step(fake, 1, d, 8, 1e-3, 1e-2, 0, 0, fake, 4, 64, fake, None, None, ws,
+                            None) == 3
+    assert L.soma_eval_loss(fake, 1, d, fake, 4, 64, fake, fake, 16, None) == 3
+    assert L.soma_init_experts(fake, 1, d, 0, -1.0, None) == 1
+    assert L.soma_spsa_update(fake, 1, d, 8, float("nan"), 0, 0, fake, None) == 1
+    assert L.soma_debug_rademacher(0, 0, 0, 0, -1, 4, fake, None) == 1
