@@ -162,7 +162,7 @@ def test_deterministic_and_resumable():
 def test_nonfinite_loss_is_reported_and_skips_the_update():
     E, H, N, n = 8, 16, 2, 3
     theta = inputs.init_params(N, E, H, seed=15, std=0.2)
-    theta[0, 10] = np.nan  # an embedding entry of expert 0
+    theta[0, 2] = np.nan  # Emb[0][2] of expert 0
     bx = inputs.expert_batch(N, 3, 8, 1, seed=16, step=0)
     bx[0, :, :] = 0  # every input byte reads the NaN row
     g = run_step(theta, bx, E, H, n, 1e-3, 1e-2, 1, 1)
