@@ -157,6 +157,30 @@ int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int c
 int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
                           int64_t count, int8_t* z_out, void* stream);
 
+/* SPSA step without a workspace argument, for callers that cannot allocate
+ * device memory (a host runtime that only passes on buffers it was given, or
+ * a loop that must not risk an allocation that blocks or fails).  The paper
+ * has no counterpart; this is an interface convenience of this library.
+ *
+ * Same arguments and results as soma_spsa_step() minus the workspace: the
+ * scratch is a fixed device array of SOMA_STATIC_WORKSPACE_BYTES inside the
+ * library, which every GPU that loads the library keeps until the process
+ * exits.  Sizes whose soma_workspace_bytes() exceed that return
+ * SOMA_ERR_WORKSPACE before anything is enqueued.  No cudaMalloc, cudaFree
+ * or other allocating routine is called (keep tracing off: it creates CUDA
+ * events on first use).
+ *  - The first call on each device looks up the array's device address with
+ *    that device current; make that first call before any stream capture.
+ *  - Every call shares the one array and the path writes each scratch word
+ *    before it reads it, so nothing needs clearing between calls; two calls
+ *    whose work overlaps on the GPU (different streams, or devices sharing
+ *    nothing but this rule) race on the array and give wrong results. */
+#define SOMA_STATIC_WORKSPACE_BYTES ((size_t)64 << 20)
+int soma_spsa_step_static(float* params, int n_experts, soma_dims d, int n_pert, float eps,
+                          float lr, uint64_t seed, uint64_t step, const uint8_t* byte_batch,
+                          int batch, int seq_len, float* losses_out, float* coef_out,
+                          void* stream);
+
 #ifdef __cplusplus
 }
 #endif
