@@ -41,7 +41,11 @@ UNIT = "perturbed tokens/s"
 # DRAM traffic of one launch of the dominant kernel from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel
 # source it was taken on.
-TRAFFIC = {}
+TRAFFIC = {
+    # profiles/gate_step_kernel_fp32_soma_n2.md
+    "soma_n2": {"bytes_per_launch": 145.918e6, "files": ["forward_simt.cu", "soma_device.cuh"],
+                "source_hash": "c530d39908133690"},
+}
 
 
 def parse():
@@ -202,13 +206,13 @@ def reference_arm(args):
     return 0
 
 
-def source_hash():
+def source_hash(files):
+    """Hash of the sources a traffic figure was measured on."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_37899_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, f), "rb") as fh:
-                h.update(fh.read())
+    for f in files:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()[:16]
 
 
@@ -292,7 +296,8 @@ def our_arm(args):
     peak = peaks["bf16_tflops_sustained"]
     achieved = gate_flops_per_launch(c) / (gate_ms / gate_n / 1e3) / 1e12 if gate_n else None
     tr = TRAFFIC.get(args.config)
-    traffic = tr["bytes_per_launch"] if tr and tr.get("source_hash") == source_hash() else None
+    traffic = (tr["bytes_per_launch"]
+               if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
     launches = sum(v[1] for v in traced.values())
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
