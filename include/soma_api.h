@@ -137,7 +137,8 @@ enum {
   SOMA_TRACE_HEAD = 1,   /* output head + log-softmax + NLL */
   SOMA_TRACE_REDUCE = 2, /* loss and coefficient reduction */
   SOMA_TRACE_UPDATE = 3, /* Philox-regenerating parameter update */
-  SOMA_TRACE_KINDS = 4
+  SOMA_TRACE_PREP = 4,   /* fp16 weight tiles and embedding operands */
+  SOMA_TRACE_KINDS = 5
 };
 typedef struct soma_kernel_times {
   double ms[SOMA_TRACE_KINDS];       /* summed device time per class */
@@ -156,6 +157,12 @@ int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int c
                       void* stream);
 int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
                           int64_t count, int8_t* z_out, void* stream);
+/* soma_debug_tc_gemm: d[128][n] = a[128][k] * b[n][k]^T (fp16 inputs as
+ *   uint16 bit patterns, row-major; fp32 output) through the same shared-
+ *   memory descriptors, tcgen05.mma and tensor-memory read-back as the
+ *   forward kernels.  16 <= n, k <= 256, both multiples of 16. */
+int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                       void* stream);
 
 /* SPSA step without a workspace argument, for callers that cannot allocate
  * device memory (a host runtime that only passes on buffers it was given, or

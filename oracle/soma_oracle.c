@@ -35,7 +35,11 @@
  *   key     = (seed & 0xffffffff, seed >> 32)
  *   counter = (p >> 7, i, step & 0xffffffff, e)
  *   w[0..3] = Philox4x32-10(counter, key)
- *   bit     = (w[(p & 127) >> 5] >> (p & 31)) & 1,   z = 1 - 2 * bit.
+ *   o       = p & 31  (position inside the 32-parameter run of one word)
+ *   bit     = (w[(p & 127) >> 5] >> ((o >> 1) + 16 * (o & 1))) & 1
+ *   z       = 1 - 2 * bit.
+ * Within each word, parameters 2j and 2j+1 of the run read bits j and
+ * j + 16: an even/odd interleave of the two 16-bit halves.
  */
 #include <math.h>
 #include <stdint.h>
@@ -94,7 +98,8 @@ void oracle_rademacher(uint64_t seed, uint64_t step, uint32_t expert,
     uint32_t w[4];
     oracle_philox4x32_10(ctr, key, w);
     int k = (int)(p & 127);
-    uint32_t bit = (w[k >> 5] >> (k & 31)) & 1u;
+    int o = k & 31;
+    uint32_t bit = (w[k >> 5] >> ((o >> 1) + 16 * (o & 1))) & 1u;
     z[q] = (int8_t)(1 - 2 * (int)bit);
   }
 }

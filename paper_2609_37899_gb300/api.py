@@ -36,11 +36,11 @@ class soma_dims(ctypes.Structure):
     _fields_ = [("vocab", ctypes.c_int32), ("embed", ctypes.c_int32), ("hidden", ctypes.c_int32)]
 
 
-TRACE_KINDS = ("gate", "head", "reduce", "update")
+TRACE_KINDS = ("gate", "head", "reduce", "update", "prep")
 
 
 class soma_kernel_times(ctypes.Structure):
-    _fields_ = [("ms", ctypes.c_double * 4), ("launches", ctypes.c_int64 * 4)]
+    _fields_ = [("ms", ctypes.c_double * 5), ("launches", ctypes.c_int64 * 5)]
 
 
 def _sig(lib, name, res, args):
@@ -74,6 +74,7 @@ def lib():
         _sig(L, "soma_trace_read", i32, [ctypes.POINTER(soma_kernel_times), i32])
         _sig(L, "soma_debug_philox", i32, [u64, vp, vp, i32, vp])
         _sig(L, "soma_debug_rademacher", i32, [u64, u64, i32, i32, i64, i64, vp, vp])
+        _sig(L, "soma_debug_tc_gemm", i32, [vp, vp, vp, i32, i32, vp])
         _lib = L
         return L
 
@@ -196,6 +197,17 @@ def debug_rademacher(seed: int, step: int, expert: int, probe: int, p0: int, cou
                                        _dev(z, torch.int8, "z"), _stream(stream)),
            "soma_debug_rademacher")
     return z
+
+
+def debug_tc_gemm(a: torch.Tensor, b: torch.Tensor, stream=None) -> torch.Tensor:
+    """a [128, K] fp16, b [N, K] fp16 (CUDA) -> a @ b.T [128, N] fp32 on the tensor cores."""
+    n, k = b.shape
+    d = torch.empty(128, n, dtype=torch.float32, device=a.device)
+    _check(lib().soma_debug_tc_gemm(_dev(a, torch.float16, "a", 128 * k),
+                                    _dev(b, torch.float16, "b", n * k),
+                                    _dev(d, torch.float32, "d"), n, k, _stream(stream)),
+           "soma_debug_tc_gemm")
+    return d
 
 
 class SomaExperts:

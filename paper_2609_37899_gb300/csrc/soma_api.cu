@@ -42,28 +42,43 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 constexpr size_t kAlign = 256;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Workspace of one sweep with `n_pert` probes and `n_sign` signs.
+// Workspace of one sweep with `n_pert` probes and `n_sign` signs.  Batches of
+// up to 128 sequences run on the tensor cores (both signs always); larger
+// batches on the fp32 CUDA-core kernels.
 struct WsPlan {
+  bool tc;
+  TcGeom g;
+  TcSizes z;
   int Tc;
   size_t hist, cst, nll, coef, total;
 };
 
 WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T) {
+  WsPlan w;
+  std::memset(&w, 0, sizeof(w));
+  const Layout lay = make_layout(d.embed, d.hidden);
+  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
+  if (tc_supported(B)) {
+    w.tc = true;
+    w.g = make_tc_geom(lay, n_experts, n_pert, B, T);
+    w.z = tc_sizes(w.g);
+    w.total = round_up(w.z.w16) + round_up(w.z.wo16) + 2 * round_up(w.z.op) + round_up(w.z.cst) +
+              2 * round_up(w.z.pm) + round_up(w.z.ply) + w.coef;
+    return w;
+  }
   Sweep s;
   std::memset(&s, 0, sizeof(s));
-  s.lay = make_layout(d.embed, d.hidden);
+  s.lay = lay;
   s.n_experts = n_experts;
   s.n_pert = n_pert;
   s.n_sign = n_sign;
   s.B = B;
   s.T = T;
-  WsPlan w;
   w.Tc = forward_hist_slots(s);
   const size_t lanes = (size_t)s.lanes();
   w.hist = round_up(lanes * w.Tc * B * (size_t)d.hidden * sizeof(float));
   w.cst = round_up(lanes * B * (size_t)d.hidden * sizeof(float));
   w.nll = round_up(lanes * B * (size_t)T * sizeof(float));
-  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
   w.total = w.hist + w.cst + w.nll + w.coef;
   return w;
 }
@@ -78,8 +93,30 @@ ForwardBuffers carve(const WsPlan& w, void* ws) {
   return fb;
 }
 
+TcBuffers carve_tc(const WsPlan& w, void* ws) {
+  uint8_t* p = static_cast<uint8_t*>(ws);
+  TcBuffers tb;
+  tb.w16 = p;
+  p += round_up(w.z.w16);
+  tb.wo16 = p;
+  p += round_up(w.z.wo16);
+  tb.op[0] = p;
+  p += round_up(w.z.op);
+  tb.op[1] = p;
+  p += round_up(w.z.op);
+  tb.cst = reinterpret_cast<float*>(p);
+  p += round_up(w.z.cst);
+  tb.pm = reinterpret_cast<float*>(p);
+  p += round_up(w.z.pm);
+  tb.ps = reinterpret_cast<float*>(p);
+  p += round_up(w.z.pm);
+  tb.ply = reinterpret_cast<float*>(p);
+  return tb;
+}
+
+// the coefficient scratch is the last region of both layouts
 float* coef_scratch(const WsPlan& w, void* ws) {
-  return reinterpret_cast<float*>(static_cast<char*>(ws) + w.hist + w.cst + w.nll);
+  return reinterpret_cast<float*>(static_cast<char*>(ws) + (w.total - w.coef));
 }
 
 bool sizes_ok(int n_experts, int n_pert, int batch, int seq_len) {
@@ -146,13 +183,21 @@ int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float 
   s.eps = eps;
   s.seed = seed;
   s.step = step;
-  const ForwardBuffers fb = carve(w, workspace);
   float* coef_ws = coef_scratch(w, workspace);
-
-  cudaError_t e = launch_forward_simt(s, fb, st);
-  if (e == cudaSuccess)
-    e = launch_reduce_losses(fb.nll, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
-                             coef_out, coef_ws, status, st);
+  cudaError_t e;
+  if (w.tc) {
+    const TcBuffers tb = carve_tc(w, workspace);
+    e = launch_forward_tc(s, w.g, tb, status, st);
+    if (e == cudaSuccess)
+      e = launch_reduce_tc(tb, n_experts * n_pert, 2, batch, seq_len, eps, losses_out, coef_out,
+                           coef_ws, status, st);
+  } else {
+    const ForwardBuffers fb = carve(w, workspace);
+    e = launch_forward_simt(s, fb, st);
+    if (e == cudaSuccess)
+      e = launch_reduce_losses(fb.nll, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
+                               coef_out, coef_ws, status, st);
+  }
   // eps == 0 makes every coefficient 0 and lr == 0 every step 0: theta stays
   // bit-identical, so the update is not launched at all.
   if (e == cudaSuccess && eps != 0.f && lr != 0.f)
@@ -184,11 +229,20 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
   s.eps = 0.f;
   s.seed = 0;
   s.step = 0;
-  const ForwardBuffers fb = carve(w, workspace);
-  cudaError_t e = launch_forward_simt(s, fb, st);
-  if (e == cudaSuccess)
-    e = launch_reduce_losses(fb.nll, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
-                             nullptr, status, st);
+  cudaError_t e;
+  if (w.tc) {
+    const TcBuffers tb = carve_tc(w, workspace);
+    e = launch_forward_tc(s, w.g, tb, status, st);
+    if (e == cudaSuccess)
+      e = launch_reduce_tc(tb, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr, nullptr,
+                           status, st);
+  } else {
+    const ForwardBuffers fb = carve(w, workspace);
+    e = launch_forward_simt(s, fb, st);
+    if (e == cudaSuccess)
+      e = launch_reduce_losses(fb.nll, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
+                               nullptr, status, st);
+  }
   return cuda_status(e);
 }
 
@@ -234,6 +288,16 @@ int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int c
   if (!ctr4 || !out4 || count < 0) return SOMA_ERR_INVALID_ARG;
   if (count == 0) return SOMA_OK;
   return cuda_status(launch_debug_philox(seed, ctr4, out4, count, (cudaStream_t)stream));
+}
+
+int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                       void* stream) {
+  if (!a || !b || !d || !aligned16(a) || !aligned16(b) || n < 16 || n > 256 || n % 16 ||
+      k < 16 || k > 256 || k % 16)
+    return SOMA_ERR_INVALID_ARG;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  return cuda_status(launch_debug_tc_gemm(a, b, d, n, k, status, (cudaStream_t)stream));
 }
 
 int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,

@@ -66,24 +66,42 @@ __host__ __device__ __forceinline__ uint4 probe_block(const ProbeKey& k, uint32_
   return philox4x32_10(make_uint4(blk, k.probe, k.step, k.expert), k.k0, k.k1);
 }
 
-// Bits of z for the 32 consecutive parameters p .. p+31: bit j set <=> z[p+j]
-// = -1.  One Philox call when the run stays inside one 128-parameter block,
-// two when it crosses into the next.
+// Raw probe word of the 32-parameter run w (parameters 32w .. 32w+31): word
+// (w & 3) of the Philox block w >> 2.  Inside a run, parameter 32w + o reads
+// raw bit (o >> 1) + 16 (o & 1): even offsets take the low half in order, odd
+// offsets the high half.
+__host__ __device__ __forceinline__ uint32_t probe_raw_word(const ProbeKey& k, uint32_t w) {
+  return word_of(probe_block(k, w >> 2), (int)(w & 3));
+}
+
+__host__ __device__ __forceinline__ uint32_t spread16(uint32_t x) {
+  x &= 0xFFFFu;
+  x = (x | (x << 8)) & 0x00FF00FFu;
+  x = (x | (x << 4)) & 0x0F0F0F0Fu;
+  x = (x | (x << 2)) & 0x33333333u;
+  x = (x | (x << 1)) & 0x55555555u;
+  return x;
+}
+
+// Raw word -> natural order (bit o <=> parameter 32w + o).
+__host__ __device__ __forceinline__ uint32_t raw_to_natural(uint32_t raw) {
+  return spread16(raw) | (spread16(raw >> 16) << 1);
+}
+
+// Bits of z for the 32 consecutive parameters p .. p+31 in natural order:
+// bit j set <=> z[p+j] = -1.  One Philox call when p is 32-aligned, at most
+// two otherwise.
 __host__ __device__ __forceinline__ uint32_t probe_bits32(const ProbeKey& k, int64_t p) {
-  const uint32_t blk = (uint32_t)(p >> 7);
-  const int off = (int)(p & 127);
-  const int wi = off >> 5, sh = off & 31;
-  const uint4 a = probe_block(k, blk);
-  const uint32_t lo = word_of(a, wi);
+  const uint32_t w = (uint32_t)(p >> 5);
+  const int sh = (int)(p & 31);
+  const uint32_t lo = raw_to_natural(probe_raw_word(k, w));
   if (sh == 0) return lo;
-  uint32_t hi;
-  if (wi < 3) {
-    hi = word_of(a, wi + 1);
-  } else {
-    hi = probe_block(k, blk + 1).x;
-  }
+  const uint32_t hi = raw_to_natural(probe_raw_word(k, w + 1));
   return (lo >> sh) | (hi << (32 - sh));
 }
+
+// Raw bit position of offset o (0..31) inside a run.
+__host__ __device__ constexpr int raw_bit(int o) { return (o >> 1) + 16 * (o & 1); }
 
 // w + s*eps*z for a z bit: the perturbed parameter in fp32.
 __host__ __device__ __forceinline__ float perturb(float w, uint32_t bit, float se) {

@@ -25,6 +25,42 @@ void trace_end(int kind, cudaStream_t stream);
 int forward_hist_slots(const Sweep& s);
 cudaError_t launch_forward_simt(const Sweep& s, const ForwardBuffers& fb, cudaStream_t stream);
 
+// ---- tensor-core path ------------------------------------------------------
+// Geometry of one sweep on the tensor cores.  K of the gate GEMM is
+// [x part padded to Ep | h part padded to Hp], in stages of 32; rows are
+// 32-unit tiles of 4 gates; sequences are padded to Bp and P probes share one
+// operand group tile of rowsB = 2 Bp P rows ([hbar | dh] per probe).
+struct TcGeom {
+  int E, H, Ep, Hp, S, Sx, Sh, MT, Bp, P, G, rowsB;
+  uint32_t tileB;  // bytes of one operand group tile of one stage
+  int n_experts, n_pert, B, T;
+};
+
+struct TcSizes {
+  size_t w16, wo16, op, cst, pm, ply;
+};
+
+struct TcBuffers {
+  uint8_t* w16;    // gate weight tiles, fp16
+  uint8_t* wo16;   // head weight tiles, fp16
+  uint8_t* op[2];  // operands of timesteps t and t + 1
+  float* cst;      // cell state, fp32 per sign
+  float* pm;       // head partial max
+  float* ps;       // head partial sum-exp
+  float* ply;      // target logits
+};
+
+TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T);
+bool tc_supported(int B);
+TcSizes tc_sizes(const TcGeom& g);
+cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
+                              cudaStream_t stream);
+cudaError_t launch_reduce_tc(const TcBuffers& tb, int pairs, int n_sign, int B, int T, float eps,
+                             float* losses_out, float* coef_out, float* coef_ws, int* status,
+                             cudaStream_t stream);
+cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K, int* status,
+                                 cudaStream_t stream);
+
 // losses_out [pairs][n_sign]; coef_out / coef_ws [pairs] (either may be null).
 cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B, int T, float eps,
                                  float* losses_out, float* coef_out, float* coef_ws, int* status,

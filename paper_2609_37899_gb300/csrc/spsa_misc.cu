@@ -62,7 +62,8 @@ constexpr int kUpdThreads = 128;
 
 // theta[e][p] -= lr * (1/n) * sum_i coef[e][i] z_{e,i}[p].  Thread q of
 // expert e owns the 32 parameters 32q .. 32q + 31, whose probe bits are one
-// 32-bit Philox output word for every probe.  An expert whose coefficients
+// raw 32-bit Philox output word for every probe (read in the run's bit
+// order, which the unrolled loop resolves at compile time).  An expert whose coefficients
 // are not all finite is left unchanged.
 __global__ void __launch_bounds__(kUpdThreads)
 spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr, uint64_t seed,
@@ -87,10 +88,10 @@ spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr,
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   for (int i = 0; i < n_pert; ++i) {
     const ProbeKey pk = make_probe_key(seed, step, (uint32_t)e, (uint32_t)i);
-    const uint32_t bits = probe_bits32(pk, p0);  // 32-aligned: one Philox call
+    const uint32_t raw = probe_raw_word(pk, (uint32_t)(p0 >> 5));  // p0 is 32-aligned
     const float c = cf[i];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) acc[j] += ((bits >> j) & 1u) ? -c : c;
+    for (int j = 0; j < 32; ++j) acc[j] += ((raw >> raw_bit(j)) & 1u) ? -c : c;
   }
   const float scale = lr / (float)n_pert;
   float* th = params + (int64_t)e * lay.P + p0;

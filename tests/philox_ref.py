@@ -67,12 +67,14 @@ def blocks(seed: int, counters) -> np.ndarray:
 
 
 def rademacher(seed: int, step: int, expert: int, probe: int, p0: int, count: int) -> np.ndarray:
-    """z[p] = 1 - 2 * bit (p & 127) of block (p >> 7, probe, step, expert)."""
+    """z[p] = 1 - 2 * bit of block (p >> 7, probe, step, expert): word
+    (p & 127) >> 5, bit (o >> 1) + 16 (o & 1) with o = p & 31."""
     p = np.arange(p0, p0 + count, dtype=np.int64)
     blk = np.unique(p >> 7)
     words = blocks(seed, [(int(b), probe, step & 0xFFFFFFFF, expert) for b in blk])
     row = {int(b): k for k, b in enumerate(blk)}
     k = p & 127
     w = np.array([words[row[int(b)], int(kk) >> 5] for b, kk in zip(p >> 7, k)], dtype=np.uint64)
-    bit = (w >> (k & 31).astype(np.uint64)) & np.uint64(1)
+    o = k & 31
+    bit = (w >> ((o >> 1) + 16 * (o & 1)).astype(np.uint64)) & np.uint64(1)
     return (1 - 2 * bit.astype(np.int64)).astype(np.int8)

@@ -190,3 +190,11 @@ def test_init_experts():
     assert abs(x[:, o["w_hh"]:o["b"]].mean()) < 1e-3
     a.init_experts(q, E, H, seed=3, std=0.5)
     assert q.std().item() == pytest.approx(0.5, rel=0.02)
+
+
+def test_large_batch_uses_the_cuda_core_path(oracle_mod):
+    # more than 128 sequences per expert: the fp32 CUDA-core kernels
+    N, E, H, B, T, n = 1, 3, 5, 130, 4, 2
+    theta = inputs.init_params(N, E, H, seed=21, std=0.3)
+    bx = inputs.expert_batch(N, B, T, 1, seed=22, step=0)
+    _full_parity(oracle_mod, theta, bx, E, H, n, 1e-3, 1e-2, 3, 1)
