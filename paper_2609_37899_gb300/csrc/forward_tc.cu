@@ -16,18 +16,18 @@
 // logits+- = [W_out hbar + eps Z_out dh + b_out] +- [W_out dh + eps Z_out hbar
 // + eps z_bo].
 //
-// Per timestep t:
-//   gate_tc_kernel  one CTA per (expert, 32-unit row tile, group of P probes):
-//                   D_W[128 x 2BpP] = W_tile x [vbar|dv]^T (one MMA chain,
-//                   shared by the P probes) and D_Z,p[128 x 2Bp] = Z_p x
-//                   [vbar_p|dv_p]^T, Z_p generated from Philox into shared
-//                   memory stage by stage; epilogue: gates, cell update,
-//                   next timestep's operand [hbar|dh] (fp16).
-//   head_tc_kernel  one CTA per (expert, 128-row vocabulary half, probe
-//                   group): the same MMAs over the h part of the operand,
-//                   then per (sequence, sign) max and sum-exp partials of
-//                   the half and the target logit.
-//   xpart_kernel    the embedding part of the next operand.
+// Per timestep t, two launches of one persistent kernel:
+//   gate tasks  (expert, 32-unit row tile, group of P probes):
+//               D_W[128 x 2BpP] = W_tile x [vbar|dv]^T (shared by the P
+//               probes) and D_Z,p[128 x 2Bp] = Z_p x [vbar_p|dv_p]^T, Z_p
+//               generated from Philox into shared memory stage by stage;
+//               epilogue: gates, cell update, next timestep's operand
+//               [hbar|dh] (fp16).
+//   head tasks  (expert, 128-row vocabulary half, probe group): the same
+//               MMAs over the h part of the operand, then per (sequence,
+//               sign) max and sum-exp partials of the half and the target
+//               logit; extra blocks of the same launch write the embedding
+//               part of the next operand.
 // A final reduction merges the two halves into per-target NLL and the
 // per-(expert, probe) losses and coefficients.
 #include <cuda_fp16.h>
@@ -43,14 +43,16 @@ using namespace tc;
 
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kStages = 3;
+constexpr int kZWarps = 8;
+constexpr int kLoaders = 4;  // one bulk copy stream per issuing thread: several issuers
+constexpr int kThreads = (kLoaders + 1 + kZWarps + 8) * 32;  // loaders, MMA, Z, epilogue
+constexpr int kStages = 6;
 constexpr int kKt = 32;                 // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
 constexpr uint32_t kSbo = kKt * 16;     // bytes between 8-row groups
 constexpr uint32_t kLbo = 128;          // bytes between core matrices along K
-constexpr uint32_t kZCols = 256;        // TMEM column where the Z products start
-constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kZCols = 128;        // Z products start 128 columns into a buffer
+constexpr uint32_t kTmemCols = 512;     // two accumulator buffers of 256 columns
 
 __device__ __forceinline__ uint32_t compact16(uint32_t x) {
   x &= 0x55555555u;
@@ -104,7 +106,20 @@ __device__ __forceinline__ uint32_t z_run_raw(const ProbeKey& pk, int64_t p0, ZS
 }
 
 // Writes the 128 x 32 Z tile row r (one 32-parameter run) in the canonical
-// K-major layout.
+// K-major layout; `row` points at element (r, 0), the four 8-element chunks
+// of the row are 128 bytes apart.
+__device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw) {
+  uint4 c0, c1, c2, c3;
+  c0.x = pm1_pair<0>(raw);  c0.y = pm1_pair<1>(raw);  c0.z = pm1_pair<2>(raw);  c0.w = pm1_pair<3>(raw);
+  c1.x = pm1_pair<4>(raw);  c1.y = pm1_pair<5>(raw);  c1.z = pm1_pair<6>(raw);  c1.w = pm1_pair<7>(raw);
+  c2.x = pm1_pair<8>(raw);  c2.y = pm1_pair<9>(raw);  c2.z = pm1_pair<10>(raw); c2.w = pm1_pair<11>(raw);
+  c3.x = pm1_pair<12>(raw); c3.y = pm1_pair<13>(raw); c3.z = pm1_pair<14>(raw); c3.w = pm1_pair<15>(raw);
+  *reinterpret_cast<uint4*>(row) = c0;
+  *reinterpret_cast<uint4*>(row + 128) = c1;
+  *reinterpret_cast<uint4*>(row + 256) = c2;
+  *reinterpret_cast<uint4*>(row + 384) = c3;
+}
+
 __device__ __forceinline__ void store_z_row(uint8_t* ztile, int r, uint32_t raw) {
   uint4 c0, c1, c2, c3;
   c0.x = pm1_pair<0>(raw);  c0.y = pm1_pair<1>(raw);  c0.z = pm1_pair<2>(raw);  c0.w = pm1_pair<3>(raw);
@@ -117,21 +132,43 @@ __device__ __forceinline__ void store_z_row(uint8_t* ztile, int r, uint32_t raw)
   *reinterpret_cast<uint4*>(ztile + kmajor_offset(r, 24, kKt)) = c3;
 }
 
-// Everything the main loop needs for one task.
-struct TaskIO {
-  const uint8_t* a;      // A1 tile of stage 0
-  size_t a_stride;       // bytes between the A1 tiles of consecutive stages
-  const uint8_t* b;      // operand group tile of stage 0
-  size_t b_stride;
-  int nst;               // stages
-  int p_valid;           // probes of this group that exist
-  bool do_z;             // eps != 0: the Z products are needed
+// ---------------------------------------------------------------------------
+// Persistent warp-specialised kernel.  One CTA per SM walks a static list of
+// tasks (blockIdx.x, blockIdx.x + n_ctas, ...; the head launch appends
+// n_ctas-independent blocks for the embedding operand, so the stride is
+// n_ctas, not the grid size).  Roles:
+//   warps 0..3    loaders: warp j bulk-copies the A tile and the operand
+//                 group tile of every stage gs = j (mod 4) into a ring of
+//                 kStages shared-memory slots (the copies of one issuing
+//                 thread complete one after another, so four issue them);
+//   warp 4        MMA issuer: W x operand and Z_p x operand_p per stage into
+//                 one of two TMEM accumulator buffers (256 columns each);
+//   warps 5..12   Z generators: the +-1 tiles of the stage, from Philox;
+//   warps 13..20  epilogue: reads a finished accumulator buffer while the
+//                 MMAs of the next task fill the other one.
+// Barriers: load_full / z_full (slot filled), slot_free (the slot's MMAs are
+// done), acc_full (a buffer's task is accumulated), acc_empty (its epilogue
+// has read it).  Every wait is bounded (wait_or_abort).
+// ---------------------------------------------------------------------------
+constexpr int kMmaWarp = kLoaders;
+constexpr int kZWarp0 = kMmaWarp + 1;
+constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
+constexpr int kEpiWarps = 8;
+constexpr int kAccCols = 256;
+
+struct Ctl {
+  uint64_t load_full[kStages];
+  uint64_t z_full[kStages];
+  uint64_t slot_free[kStages];
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
+  uint32_t tmem_slot;
+  volatile int abort;
 };
 
-// Main loop shared by the gate and head kernels.  zparam(r, s) is the flat
-// parameter index of element (row r, k = 0) of the stage-s Z run.
 // A wait that times out records SOMA_ERR_TIMEOUT in the status word and sets
-// the CTA's abort flag; every later wait and MMA of the task is skipped.
+// the CTA's abort flag; later waits return at once and the CTA winds down
+// without issuing further copies or MMAs.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               int* status) {
   if (*abort) return false;
@@ -139,76 +176,6 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   *abort = 1;
   atomicCAS(status, 0, kStatusTimeout);
   return false;
-}
-
-template <class ZParam>
-__device__ bool tc_mainloop(const TcGeom& g, const TaskIO& io, uint8_t* smem, uint64_t* load_full,
-                            uint64_t* mma_done, uint32_t tmem, const ProbeKey* pks,
-                            ZParam zparam, volatile int* abort, int* status) {
-  const int tid = threadIdx.x;
-  const StageLayout SL = stage_layout(g);
-  const uint32_t idesc_w = idesc_f16_f32(128, g.rowsB);
-  const uint32_t idesc_z = idesc_f16_f32(128, 2 * g.Bp);
-  const uint32_t b_bytes = g.tileB;
-  const int nz = io.do_z ? io.p_valid * 128 : 0;  // (probe, row) pairs to generate
-  ZSlot cache[2];
-  cache[0].blk = 0xFFFFFFFFu;
-  cache[1].blk = 0xFFFFFFFFu;
-
-  for (int s = 0; s < io.nst; ++s) {
-    const int q = s % kStages;
-    const uint32_t use = (uint32_t)(s / kStages);
-    uint8_t* st = smem + q * SL.bytes;
-    if (s >= kStages) wait_or_abort(&mma_done[q], (use - 1) & 1u, abort, status);
-    if (tid == 0 && !*abort) {
-      mbar_arrive_expect_tx(&load_full[q], kTileA + b_bytes);
-      bulk_g2s(st + SL.a_off, io.a + (size_t)s * io.a_stride, kTileA, &load_full[q]);
-      bulk_g2s(st + SL.b_off, io.b + (size_t)s * io.b_stride, b_bytes, &load_full[q]);
-    }
-    // Z tiles of this stage: thread handles pairs tid and tid + 256
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int pr = tid + j * kThreads;
-      if (pr < nz) {
-        const int p = pr >> 7, r = pr & 127;
-        const uint32_t raw = z_run_raw(pks[p], zparam(r, s), cache[j]);
-        store_z_row(st + SL.z_off + p * kTileA, r, raw);
-      }
-    }
-    fence_async_smem();
-    __syncthreads();
-    if (tid == 0 && !*abort) {
-      const bool ok = wait_or_abort(&load_full[q], use & 1u, abort, status);
-      tc_fence_after();
-      if (ok) {
-        const uint32_t a_addr = smem_u32(st + SL.a_off);
-        const uint32_t b_addr = smem_u32(st + SL.b_off);
-        const uint32_t z_addr = smem_u32(st + SL.z_off);
-#pragma unroll
-        for (int k16 = 0; k16 < kKt / 16; ++k16) {
-          const uint32_t acc = (s > 0 || k16 > 0) ? 1u : 0u;
-          mma_f16_ss(tmem, smem_desc(a_addr + k16 * 32 * 8, kLbo, kSbo),
-                     smem_desc(b_addr + k16 * 32 * 8, kLbo, kSbo), idesc_w, acc);
-          if (io.do_z) {
-            for (int p = 0; p < io.p_valid; ++p) {
-              const uint32_t brow = (uint32_t)(2 * g.Bp * p);
-              mma_f16_ss(tmem + kZCols + brow,
-                         smem_desc(z_addr + p * kTileA + k16 * 32 * 8, kLbo, kSbo),
-                         smem_desc(b_addr + (brow / 8) * kSbo + k16 * 32 * 8, kLbo, kSbo),
-                         idesc_z, acc);
-            }
-          }
-        }
-      }
-      mma_commit(&mma_done[q]);
-    }
-  }
-  // all MMAs issued by this CTA are complete once the last commit lands
-  const int last = io.nst - 1;
-  wait_or_abort(&mma_done[last % kStages], (uint32_t)(last / kStages) & 1u, abort, status);
-  tc_fence_after();
-  __syncthreads();
-  return !*abort;
 }
 
 struct TcArgs {
@@ -219,228 +186,178 @@ struct TcArgs {
   const uint8_t* wo16;   // [N][2][Sh] A tiles
   const uint8_t* op_in;  // [N][S][G] operand group tiles of this timestep
   uint8_t* op_out;       // next timestep's operand
-  float* cst;            // [N*n*2][B][Hp] cell state
+  float* cst;            // [N*n*2][Hp][Bp] cell state
   float* pm;             // [N*n*2][B][T][2] head max partials
   float* ps;             // sum-exp partials
   float* ply;            // [N*n*2][B][T] target logits
   int* status;
 };
 
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
-
-struct KernelShared {
-  uint64_t load_full[kStages];
-  uint64_t mma_done[kStages];
-  uint32_t tmem_slot;
-  volatile int abort;
+// One task: (expert, row tile, probe group).  For the gate the row tile is
+// 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
+// half.
+struct Task {
+  int e, m, grp, p_valid;
+  const uint8_t* a;  // A tile of stage 0
+  const uint8_t* b;  // operand group tile of stage 0
 };
 
-__device__ __forceinline__ void kernel_setup(KernelShared* ks, uint32_t& tmem) {
-  if (threadIdx.x == 0) {
-    ks->abort = 0;
-    for (int q = 0; q < kStages; ++q) {
-      mbar_init(&ks->load_full[q], 1);
-      mbar_init(&ks->mma_done[q], 1);
-    }
-    mbar_fence_init();
+template <bool HEAD>
+__device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
+  const TcGeom& g = a.g;
+  Task T;
+  T.grp = task % g.G;
+  const int rows = HEAD ? 2 : g.MT;
+  T.m = (task / g.G) % rows;
+  T.e = task / (g.G * rows);
+  T.p_valid = min(g.P, a.sw.n_pert - T.grp * g.P);
+  if (HEAD) {
+    T.a = a.wo16 + (((size_t)T.e * 2 + T.m) * g.Sh) * kTileA;
+    T.b = a.op_in + (((size_t)T.e * g.S + g.Sx) * g.G + T.grp) * g.tileB;
+  } else {
+    T.a = a.w16 + (((size_t)T.e * g.MT + T.m) * g.S) * kTileA;
+    T.b = a.op_in + (((size_t)T.e * g.S) * g.G + T.grp) * g.tileB;
   }
-  if (threadIdx.x < 32) tmem_alloc(&ks->tmem_slot, kTmemCols);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  tmem = ks->tmem_slot;
+  return T;
 }
 
-__device__ __forceinline__ void kernel_teardown(uint32_t tmem) {
-  tc_fence_before();
-  __syncthreads();
-  if (threadIdx.x < 32) tmem_dealloc(tmem, kTmemCols);
+// Flat parameter index of element (row r, k = 0) of the stage-st Z run.
+template <bool HEAD>
+__device__ __forceinline__ int64_t z_param(const TcArgs& a, const Task& T, int r, int st) {
+  const Layout& L = a.sw.lay;
+  if (HEAD) return L.w_out + (int64_t)(128 * T.m + r) * a.g.H + (int64_t)kKt * st;
+  const int64_t R = (int64_t)(r & 3) * a.g.H + 32 * T.m + (r >> 2);  // W row of tile row r
+  return st < a.g.Sx ? L.w_ih + R * a.g.E + (int64_t)kKt * st
+                     : L.w_hh + R * a.g.H + (int64_t)kKt * (st - a.g.Sx);
 }
 
-// grid: N * MT * G blocks, 256 threads.
-__global__ void __launch_bounds__(kThreads, 1) gate_tc_kernel(const TcArgs a) {
-  extern __shared__ uint8_t dyn_smem[];
-  uint8_t* smem = align1024(dyn_smem);
+// The four products of 8 sequences of one probe: W vbar, W dv (columns cw,
+// cw + Bp) and Z vbar, Z dv (the same columns past kZCols); one wait.
+__device__ __forceinline__ void load_chunk(uint32_t tl, uint32_t cw, int Bp, bool do_z, float* wv,
+                                           float* wd, float* zv, float* zd) {
+  uint32_t r0[8], r1[8], r2[8], r3[8];
+  tmem_ld8_nowait(tl + cw, r0);
+  tmem_ld8_nowait(tl + cw + Bp, r1);
+  if (do_z) {
+    tmem_ld8_nowait(tl + kZCols + cw, r2);
+    tmem_ld8_nowait(tl + kZCols + cw + Bp, r3);
+  }
+  tmem_wait_ld();
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    wv[j] = __uint_as_float(r0[j]);
+    wd[j] = __uint_as_float(r1[j]);
+    zv[j] = do_z ? __uint_as_float(r2[j]) : 0.f;
+    zd[j] = do_z ? __uint_as_float(r3[j]) : 0.f;
+  }
+}
+
+// Gate epilogue of one task for one warp: probe p = half, TMEM lanes of the
+// warp's quarter: gates, cell update (fp32 per sign), next operand.
+__device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
+                              int q4, int p) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  KernelShared* ks = reinterpret_cast<KernelShared*>(smem + kStages * stage_layout(g).bytes);
-  const int task = blockIdx.x;
-  const int grp = task % g.G;
-  const int m = (task / g.G) % g.MT;
-  const int e = task / (g.G * g.MT);
-  const int H = g.H, E = g.E;
   const Layout& L = s.lay;
-  const float* th = s.params + (int64_t)e * L.P;
-
-  __shared__ ProbeKey pks[16];
-  if (threadIdx.x < g.P)
-    pks[threadIdx.x] = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)(grp * g.P + threadIdx.x));
-  uint32_t tmem;
-  kernel_setup(ks, tmem);
-
-  TaskIO io;
-  io.a = a.w16 + (((size_t)e * g.MT + m) * g.S) * kTileA;
-  io.a_stride = kTileA;
-  io.b = a.op_in + (((size_t)e * g.S) * g.G + grp) * g.tileB;
-  io.b_stride = (size_t)g.G * g.tileB;
-  io.nst = g.S;
-  io.p_valid = min(g.P, s.n_pert - grp * g.P);
-  io.do_z = s.eps != 0.f;
-  const int Sx = g.Sx;
-  auto zparam = [&](int r, int st) -> int64_t {
-    const int64_t R = (int64_t)(r & 3) * H + 32 * m + (r >> 2);  // W row of tile row r
-    return st < Sx ? L.w_ih + R * E + (int64_t)kKt * st
-                   : L.w_hh + R * H + (int64_t)kKt * (st - Sx);
-  };
-  if (!tc_mainloop(g, io, smem, ks->load_full, ks->mma_done, tmem, pks, zparam, &ks->abort,
-                   a.status)) {
-    kernel_teardown(tmem);
-    return;
-  }
-
-  // ---- epilogue: gates, cell update, next operand --------------------------
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int q4 = warp & 3, half = warp >> 2;
+  const int lane = threadIdx.x & 31;
+  const int H = g.H;
   const int r = 32 * q4 + lane;
   const int u_loc = r >> 2, gate = r & 3;
-  const int U = 32 * m + u_loc;
+  const int U = 32 * T.m + u_loc;
   const bool unit_ok = U < H;
-  const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16);
-  const float sc = (gate == 2) ? 2.f : 1.f;   // tanh(x) = 2 sigmoid(2x) - 1
+  const uint32_t tl = tacc + ((uint32_t)(32 * q4) << 16);
+  const float sc = (gate == 2) ? 2.f : 1.f;  // tanh(x) = 2 sigmoid(2x) - 1
   const float add = (gate == 2) ? -1.f : 0.f;
   const int base = lane & ~3;
-  const bool sign_lane = gate < 2;             // gate 0 lane: sign +, gate 1 lane: sign -
+  const bool sign_lane = gate < 2;  // gate 0 lane: sign +, gate 1 lane: sign -
   const float eps = s.eps;
-  uint8_t* out_tile = a.op_out + (((size_t)e * g.S + Sx + m) * g.G + grp) * g.tileB;
-
-  for (int p = half; p < io.p_valid; p += 2) {
-    const int i = grp * g.P + p;
-    float bias = 0.f, dbias = 0.f;
-    if (unit_ok) {
-      const int64_t pb = L.b + (int64_t)gate * H + U;
-      bias = th[pb];
-      if (io.do_z) dbias = (probe_bits32(pks[p], pb) & 1u) ? -eps : eps;
+  const bool do_z = eps != 0.f;
+  const float* th = s.params + (int64_t)T.e * L.P;
+  uint8_t* out_tile = a.op_out + (((size_t)T.e * g.S + g.Sx + T.m) * g.G + T.grp) * g.tileB;
+  const int i = T.grp * g.P + p;
+  float bias = 0.f, dbias = 0.f;
+  if (unit_ok) {
+    const int64_t pb = L.b + (int64_t)gate * H + U;
+    bias = th[pb];
+    if (do_z) dbias = (probe_bits32(pk, pb) & 1u) ? -eps : eps;
+  }
+  const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
+  const bool owns_cell = sign_lane && unit_ok;
+  float* cbase = a.cst + ((lane_plus + (gate & 1)) * g.Hp + U) * (int64_t)g.Bp;
+  for (int b0 = 0; b0 < g.Bp; b0 += 8) {
+    float cprev[8];
+    if (owns_cell && a.t > 0) {
+      const float4 x = *reinterpret_cast<const float4*>(cbase + b0);
+      const float4 y = *reinterpret_cast<const float4*>(cbase + b0 + 4);
+      cprev[0] = x.x; cprev[1] = x.y; cprev[2] = x.z; cprev[3] = x.w;
+      cprev[4] = y.x; cprev[5] = y.y; cprev[6] = y.z; cprev[7] = y.w;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) cprev[j] = 0.f;
     }
-    const int64_t lane_plus = ((int64_t)e * s.n_pert + i) * 2;
-    for (int b0 = 0; b0 < g.Bp; b0 += 8) {
-      float wv[8], wd[8], zv[8], zd[8];
-      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0);
-      tmem_ld8(tl + cw, wv);
-      tmem_ld8(tl + cw + g.Bp, wd);
-      if (io.do_z) {
-        tmem_ld8(tl + kZCols + cw, zv);
-        tmem_ld8(tl + kZCols + cw + g.Bp, zd);
-      } else {
+    float wv[8], wd[8], zv[8], zd[8], cnew[8];
+    load_chunk(tl, (uint32_t)(2 * g.Bp * p + b0), g.Bp, do_z, wv, wd, zv, zd);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) zv[j] = zd[j] = 0.f;
+    for (int j = 0; j < 8; ++j) {
+      const int b = b0 + j;
+      const float C = fmaf(eps, zd[j], wv[j]) + bias;
+      const float D = fmaf(eps, zv[j], wd[j]) + dbias;
+      const float actp = fmaf(sigm(sc * (C + D)), sc, add);
+      const float actm = fmaf(sigm(sc * (C - D)), sc, add);
+      const float ip = __shfl_sync(0xffffffffu, actp, base);
+      const float fp = __shfl_sync(0xffffffffu, actp, base + 1);
+      const float gp = __shfl_sync(0xffffffffu, actp, base + 2);
+      const float op = __shfl_sync(0xffffffffu, actp, base + 3);
+      const float im = __shfl_sync(0xffffffffu, actm, base);
+      const float fm = __shfl_sync(0xffffffffu, actm, base + 1);
+      const float gm = __shfl_sync(0xffffffffu, actm, base + 2);
+      const float om = __shfl_sync(0xffffffffu, actm, base + 3);
+      const bool plus = gate == 0;
+      // lanes of gates 0 and 1 run the cell of sign + and sign - (the other
+      // two lanes compute a copy that is never stored)
+      const float c = plus ? fmaf(fp, cprev[j], ip * gp) : fmaf(fm, cprev[j], im * gm);
+      cnew[j] = c;
+      const float h = (plus ? op : om) * fmaf(sigm(2.f * c), 2.f, -1.f);
+      const float hp = __shfl_sync(0xffffffffu, h, base);
+      const float hm = __shfl_sync(0xffffffffu, h, base + 1);
+      if (owns_cell && b < s.B) {
+        const float val = plus ? 0.5f * (hp + hm) : 0.5f * (hp - hm);
+        const int row = 2 * g.Bp * p + (plus ? b : g.Bp + b);
+        *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, u_loc, kKt)) =
+            __float2half_rn(val);
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int b = b0 + j;
-        const float C = fmaf(eps, zd[j], wv[j]) + bias;
-        const float D = fmaf(eps, zv[j], wd[j]) + dbias;
-        const float actp = fmaf(sigm(sc * (C + D)), sc, add);
-        const float actm = fmaf(sigm(sc * (C - D)), sc, add);
-        const float ip = __shfl_sync(0xffffffffu, actp, base);
-        const float fp = __shfl_sync(0xffffffffu, actp, base + 1);
-        const float gp = __shfl_sync(0xffffffffu, actp, base + 2);
-        const float op = __shfl_sync(0xffffffffu, actp, base + 3);
-        const float im = __shfl_sync(0xffffffffu, actm, base);
-        const float fm = __shfl_sync(0xffffffffu, actm, base + 1);
-        const float gm = __shfl_sync(0xffffffffu, actm, base + 2);
-        const float om = __shfl_sync(0xffffffffu, actm, base + 3);
-        const bool active = sign_lane && unit_ok && b < s.B;
-        float h = 0.f;
-        if (active) {
-          const bool plus = gate == 0;
-          float* cp = a.cst + ((lane_plus + gate) * s.B + b) * (int64_t)g.Hp + U;
-          const float cprev = (a.t == 0) ? 0.f : *cp;
-          const float c = plus ? fmaf(fp, cprev, ip * gp) : fmaf(fm, cprev, im * gm);
-          *cp = c;
-          h = (plus ? op : om) * fmaf(sigm(2.f * c), 2.f, -1.f);
-        }
-        const float hp = __shfl_sync(0xffffffffu, h, base);
-        const float hm = __shfl_sync(0xffffffffu, h, base + 1);
-        if (active) {
-          const bool plus = gate == 0;
-          const float val = plus ? 0.5f * (hp + hm) : 0.5f * (hp - hm);
-          const int row = 2 * g.Bp * p + (plus ? b : g.Bp + b);
-          *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, u_loc, kKt)) =
-              __float2half_rn(val);
-        }
-      }
+    }
+    if (owns_cell) {
+      *reinterpret_cast<float4*>(cbase + b0) = make_float4(cnew[0], cnew[1], cnew[2], cnew[3]);
+      *reinterpret_cast<float4*>(cbase + b0 + 4) = make_float4(cnew[4], cnew[5], cnew[6], cnew[7]);
     }
   }
-  kernel_teardown(tmem);
 }
 
-// grid: N * 2 * G blocks, 256 threads.  Head of timestep t: reads the h
-// part of the operand of timestep t + 1 (which holds hbar_t and dh_t).
-__global__ void __launch_bounds__(kThreads, 1) head_tc_kernel(const TcArgs a) {
-  extern __shared__ uint8_t dyn_smem[];
-  uint8_t* smem = align1024(dyn_smem);
+// Head epilogue of one task: logits +- of the warp's 32 vocabulary rows for
+// probe p; per (sequence, sign) max and sum-exp over the warp, merged over the
+// four quarters of the half through shared memory (`red`, [P][Bp][2][4]);
+// the lane whose row is the target byte writes the target logit.
+__device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
+                              int q4, int p, float2* red) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  KernelShared* ks = reinterpret_cast<KernelShared*>(smem + kStages * stage_layout(g).bytes);
-  const int task = blockIdx.x;
-  const int grp = task % g.G;
-  const int vh = (task / g.G) % 2;
-  const int e = task / (g.G * 2);
-  const int H = g.H;
   const Layout& L = s.lay;
-  const float* th = s.params + (int64_t)e * L.P;
-
-  __shared__ ProbeKey pks[16];
-  if (threadIdx.x < g.P)
-    pks[threadIdx.x] = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)(grp * g.P + threadIdx.x));
-  uint32_t tmem;
-  kernel_setup(ks, tmem);
-
-  TaskIO io;
-  io.a = a.wo16 + (((size_t)e * 2 + vh) * g.Sh) * kTileA;
-  io.a_stride = kTileA;
-  io.b = a.op_in + (((size_t)e * g.S + g.Sx) * g.G + grp) * g.tileB;
-  io.b_stride = (size_t)g.G * g.tileB;
-  io.nst = g.Sh;
-  io.p_valid = min(g.P, s.n_pert - grp * g.P);
-  io.do_z = s.eps != 0.f;
-  auto zparam = [&](int r, int st) -> int64_t {
-    return L.w_out + (int64_t)(128 * vh + r) * H + (int64_t)kKt * st;
-  };
-  if (!tc_mainloop(g, io, smem, ks->load_full, ks->mma_done, tmem, pks, zparam, &ks->abort,
-                   a.status)) {
-    kernel_teardown(tmem);
-    return;
-  }
-
-  // ---- epilogue: logits +-, per-half max / sum-exp, target logit ----------
-  // the stage buffers are free now: reuse them for the cross-warp reduction
-  float2* red = reinterpret_cast<float2*>(smem);  // [P][Bp][2][4]
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int q4 = warp & 3, half = warp >> 2;
-  const int v = 128 * vh + 32 * q4 + lane;
-  const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16);
+  const int lane = threadIdx.x & 31;
+  const int v = 128 * T.m + 32 * q4 + lane;
+  const uint32_t tl = tacc + ((uint32_t)(32 * q4) << 16);
   const float eps = s.eps;
+  const bool do_z = eps != 0.f;
+  const float* th = s.params + (int64_t)T.e * L.P;
   const float bo = th[L.b_out + v];
   const int t = a.t;
-  for (int p = half; p < io.p_valid; p += 2) {
-    const int i = grp * g.P + p;
-    const float dbo = io.do_z ? ((probe_bits32(pks[p], L.b_out + v) & 1u) ? -eps : eps) : 0.f;
-    const int64_t lane_plus = ((int64_t)e * s.n_pert + i) * 2;
+  if (p < T.p_valid) {
+    const int i = T.grp * g.P + p;
+    const float dbo = do_z ? ((probe_bits32(pk, L.b_out + v) & 1u) ? -eps : eps) : 0.f;
+    const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
     for (int b0 = 0; b0 < g.Bp; b0 += 8) {
       float wv[8], wd[8], zv[8], zd[8];
-      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0);
-      tmem_ld8(tl + cw, wv);
-      tmem_ld8(tl + cw + g.Bp, wd);
-      if (io.do_z) {
-        tmem_ld8(tl + kZCols + cw, zv);
-        tmem_ld8(tl + kZCols + cw + g.Bp, zd);
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) zv[j] = zd[j] = 0.f;
-      }
+      load_chunk(tl, (uint32_t)(2 * g.Bp * p + b0), g.Bp, do_z, wv, wd, zv, zd);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         const int b = b0 + j;
@@ -464,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1) head_tc_kernel(const TcArgs a) {
           red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
         }
         if (b < s.B) {
-          const int y = s.bytes[((int64_t)e * s.B + b) * (s.T + 1) + t + 1];
+          const int y = s.bytes[((int64_t)T.e * s.B + b) * (s.T + 1) + t + 1];
           if (y == v) {
             a.ply[((lane_plus + 0) * s.B + b) * (int64_t)s.T + t] = lp;
             a.ply[((lane_plus + 1) * s.B + b) * (int64_t)s.T + t] = lm;
@@ -473,35 +390,220 @@ __global__ void __launch_bounds__(kThreads, 1) head_tc_kernel(const TcArgs a) {
       }
     }
   }
-  __syncthreads();
-  // merge the four 32-row quarters of this half
-  const int n_red = io.p_valid * g.Bp * 2;
-  for (int idx = tid; idx < n_red; idx += kThreads) {
+  // all eight epilogue warps: partials of this task are in `red`
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+  const int et = threadIdx.x - kEpiWarp0 * 32;
+  const int n_red = T.p_valid * g.Bp * 2;
+  for (int idx = et; idx < n_red; idx += kEpiWarps * 32) {
     const int sgn = idx & 1;
     const int pb = idx >> 1;
-    const int p = pb / g.Bp, b = pb % g.Bp;
+    const int pp = pb / g.Bp, b = pb % g.Bp;
     if (b >= s.B) continue;
     const float2* q = red + (size_t)idx * 4;
-    float M = fmaxf(fmaxf(q[0].x, q[1].x), fmaxf(q[2].x, q[3].x));
+    const float M = fmaxf(fmaxf(q[0].x, q[1].x), fmaxf(q[2].x, q[3].x));
     float S = 0.f;
 #pragma unroll
     for (int k = 0; k < 4; ++k) S += q[k].y * __expf(q[k].x - M);
-    const int i = grp * g.P + p;
-    const int64_t ln = ((int64_t)e * s.n_pert + i) * 2 + sgn;
-    const int64_t o = ((ln * s.B + b) * (int64_t)s.T + t) * 2 + vh;
+    const int i = T.grp * g.P + pp;
+    const int64_t ln = ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
+    const int64_t o = ((ln * s.B + b) * (int64_t)s.T + t) * 2 + T.m;
     a.pm[o] = M;
     a.ps[o] = S;
   }
-  kernel_teardown(tmem);
+  // `red` is reused by the next task
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk);
+
+// grid: min(tasks, SMs) persistent CTAs (+ for the head, the embedding-part
+// blocks of the next timestep's operand), kThreads threads.
+template <bool HEAD>
+__global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_tasks,
+                                                                    int n_ctas) {
+  extern __shared__ uint8_t dyn_smem[];
+  const TcGeom& g = a.g;
+  const Sweep& s = a.sw;
+  if (HEAD && (int)blockIdx.x >= n_ctas) {
+    // the embedding part of timestep t + 1's operand (the head reads only
+    // the h part of the same buffer)
+    if (a.t + 1 < s.T)
+      xpart_block(a, const_cast<uint8_t*>(a.op_in), a.t + 1, blockIdx.x - n_ctas);
+    return;
+  }
+  uint8_t* smem = align1024(dyn_smem);
+  const StageLayout SL = stage_layout(g);
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem + kStages * SL.bytes);
+  float2* red = reinterpret_cast<float2*>(smem + kStages * SL.bytes + 1024);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nst = HEAD ? g.Sh : g.S;
+  const bool do_z = s.eps != 0.f;
+  int* status = a.status;
+  volatile int* abort = &ctl->abort;
+
+  if (tid == 0) {
+    ctl->abort = 0;
+    for (int q = 0; q < kStages; ++q) {
+      mbar_init(&ctl->load_full[q], 1);
+      mbar_init(&ctl->z_full[q], kZWarps);
+      mbar_init(&ctl->slot_free[q], 1);
+    }
+    for (int q = 0; q < 2; ++q) {
+      mbar_init(&ctl->acc_full[q], 1);
+      mbar_init(&ctl->acc_empty[q], kEpiWarps);
+    }
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(&ctl->tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl->tmem_slot;
+
+  if (warp < kLoaders) {
+    // ---------------------------------------------------------------- loaders
+    // the whole warp walks the stages (so that it never sits diverged at the
+    // CTA barrier); lane 0 issues the copies
+    uint32_t gs = 0;
+    for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
+      const Task T = make_task<HEAD>(a, task);
+      for (int st = 0; st < nst; ++st, ++gs) {
+        if ((int)(gs % kLoaders) != warp) continue;
+        const int q = gs % kStages;
+        const uint32_t use = gs / kStages;
+        if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
+          continue;
+        if (lane == 0 && !*abort) {
+          uint8_t* slot = smem + q * SL.bytes;
+          mbar_arrive_expect_tx(&ctl->load_full[q], kTileA + g.tileB);
+          bulk_g2s(slot + SL.a_off, T.a + (size_t)st * kTileA, kTileA, &ctl->load_full[q]);
+          bulk_g2s(slot + SL.b_off, T.b + (size_t)st * g.G * g.tileB, g.tileB, &ctl->load_full[q]);
+        }
+        __syncwarp();
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    // the whole warp waits; lane 0 issues the MMAs and commits
+    {
+      const uint32_t idesc_w = idesc_f16_f32(128, g.rowsB);
+      const uint32_t idesc_z = idesc_f16_f32(128, 2 * g.Bp);
+      // descriptors of slot 0; slot q is q * SL.bytes further, k16 = 1 is
+      // 256 bytes further (two core matrices along K)
+      const uint64_t d0 = smem_desc(smem_u32(smem), kLbo, kSbo);
+      const uint32_t hi = (uint32_t)(d0 >> 32);
+      const uint32_t lo0 = (uint32_t)d0;
+      const uint32_t slot_step = SL.bytes >> 4;
+      const uint32_t a_lo0 = lo0 + (SL.a_off >> 4), b_lo0 = lo0 + (SL.b_off >> 4);
+      const uint32_t z_lo0 = lo0 + (SL.z_off >> 4);
+      const uint32_t zp_step = kTileA >> 4;                       // next probe's Z tile
+      const uint32_t bp_step = (uint32_t)(2 * g.Bp / 8) * (kSbo >> 4);  // next probe's rows
+      uint32_t gs = 0;
+      int k = 0;
+      for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
+        const Task T = make_task<HEAD>(a, task);
+        const int buf = k & 1;
+        if (k >= 2) wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status);
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(buf * kAccCols);
+        const int np = do_z ? T.p_valid : 0;
+        for (int st = 0; st < nst; ++st, ++gs) {
+          const int q = gs % kStages;
+          const uint32_t use = gs / kStages;
+          bool ok = wait_or_abort(&ctl->load_full[q], use & 1u, abort, status);
+          if (do_z) ok = wait_or_abort(&ctl->z_full[q], use & 1u, abort, status) && ok;
+          tc_fence_after();
+          if (ok && lane == 0) {
+            const uint32_t so = (uint32_t)q * slot_step;
+            const uint32_t acc0 = st > 0 ? 1u : 0u;
+#pragma unroll
+            for (int k16 = 0; k16 < kKt / 16; ++k16) {
+              const uint32_t ko = so + (uint32_t)k16 * 16;
+              const uint32_t acc = acc0 | (uint32_t)k16;
+              mma_f16_ss_lohi(d, a_lo0 + ko, hi, b_lo0 + ko, hi, idesc_w, acc);
+              for (int p = 0; p < np; ++p)
+                mma_f16_ss_lohi(d + kZCols + (uint32_t)(2 * g.Bp * p), z_lo0 + ko + p * zp_step, hi,
+                                b_lo0 + ko + p * bp_step, hi, idesc_z, acc);
+            }
+          }
+          if (lane == 0) mma_commit(&ctl->slot_free[q]);
+          __syncwarp();
+        }
+        if (lane == 0) mma_commit(&ctl->acc_full[buf]);
+        __syncwarp();
+      }
+    }
+  } else if (warp < kEpiWarp0) {
+    // --------------------------------------------------------- Z generators
+    if (do_z) {
+      const int gtid = tid - kZWarp0 * 32;
+      const int p = gtid >> 7, r = gtid & 127;  // one (probe, row) pair per thread
+      uint32_t gs = 0;
+      for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
+        const Task T = make_task<HEAD>(a, task);
+        const bool active = p < T.p_valid;
+        ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
+        ZSlot cache;
+        cache.blk = 0xFFFFFFFFu;
+        const int split = HEAD ? nst : g.Sx;
+        const int64_t seg0 = z_param<HEAD>(a, T, r, 0);
+        const int64_t seg1 = z_param<HEAD>(a, T, r, split) - (int64_t)kKt * split;
+        uint8_t* zrow = smem + SL.z_off + p * kTileA + kmajor_offset(r, 0, kKt);
+        for (int st = 0; st < nst; ++st, ++gs) {
+          const int q = gs % kStages;
+          const uint32_t use = gs / kStages;
+          if (gs >= kStages) wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status);
+          if (active && !*abort) {
+            const int64_t p0 = (st < split ? seg0 : seg1) + (int64_t)kKt * st;
+            const uint32_t raw = z_run_raw(pk, p0, cache);
+            store_z_row_at(zrow + q * SL.bytes, raw);
+          }
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ctl->z_full[q]);
+        }
+      }
+    }
+  } else {
+    // --------------------------------------------------------------- epilogue
+    const int ew = warp - kEpiWarp0;
+    const int q4 = warp & 3;
+    const int p = ew >> 2;  // probe of the group handled by this warp
+    int k = 0;
+    for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
+      const Task T = make_task<HEAD>(a, task);
+      const int buf = k & 1;
+      wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status);
+      tc_fence_after();
+      const uint32_t tacc = tmem + (uint32_t)(buf * kAccCols);
+      const ProbeKey pk =
+          make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
+      if (HEAD) {
+        head_epilogue(a, T, tacc, pk, q4, p, red);
+      } else if (p < T.p_valid) {
+        gate_epilogue(a, T, tacc, pk, q4, p);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 }
 
 // Embedding part of the operand of timestep t: x = Emb[byte_t], dx = eps z_emb.
-// grid (Sx * G, N), 128 threads.
-__global__ void xpart_kernel(const TcArgs a, uint8_t* op) {
+// Block `blk` of Sx * G * N writes one (expert, stage, group) tile.
+__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  const int st = blockIdx.x / g.G, grp = blockIdx.x % g.G;
-  const int e = blockIdx.y;
+  const int st = (blk / g.G) % g.Sx, grp = blk % g.G;
+  const int e = blk / (g.G * g.Sx);
   const Layout& L = s.lay;
   const float* th = s.params + (int64_t)e * L.P;
   uint8_t* tile = op + (((size_t)e * g.S + st) * g.G + grp) * g.tileB;
@@ -515,7 +617,7 @@ __global__ void xpart_kernel(const TcArgs a, uint8_t* op) {
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
     if (i < s.n_pert && b < s.B) {
-      const int y = s.bytes[((int64_t)e * s.B + b) * (s.T + 1) + a.t];
+      const int y = s.bytes[((int64_t)e * s.B + b) * (s.T + 1) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
       uint32_t bits = 0;
       if (delta && s.eps != 0.f)
@@ -533,6 +635,10 @@ __global__ void xpart_kernel(const TcArgs a, uint8_t* op) {
     *reinterpret_cast<uint4*>(tile + kmajor_offset(row, 8 * kc, kKt)) =
         *reinterpret_cast<const uint4*>(v);
   }
+}
+
+__global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
+  xpart_block(a, op, t, blockIdx.x);
 }
 
 // fp16 A tiles of the gate weights ([x part | h part], rows unit-major:
@@ -691,10 +797,22 @@ debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, i
 }
 
 size_t kernel_smem_bytes(const TcGeom& g) {
-  // stages + barriers + 1 KB alignment slack; at least 120 KB so that one
-  // CTA owns an SM (and all 512 TMEM columns)
-  size_t b = (size_t)kStages * stage_layout(g).bytes + sizeof(KernelShared) + 1024 + 256;
-  return b < 120 * 1024 ? 120 * 1024 : b;
+  // ring slots, the control block (1 KB), the head's reduction buffer
+  // [P][Bp][2][4] float2 and alignment slack
+  const size_t red = (size_t)g.P * g.Bp * 2 * 4 * sizeof(float2);
+  return (size_t)kStages * stage_layout(g).bytes + 1024 + red + 1024;
+}
+
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (!cached[dev]) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    cached[dev] = n;
+  }
+  return cached[dev];
 }
 
 }  // namespace
@@ -710,8 +828,8 @@ TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T) 
   g.S = g.Sx + g.Sh;
   g.MT = g.Hp / 32;
   g.Bp = (B + 7) / 8 * 8;
-  int P = 128 / g.Bp;
-  if (P > 4) P = 4;
+  int P = 64 / g.Bp;  // rowsB = 2 Bp P <= 128 TMEM columns per product
+  if (P > 2) P = 2;
   if (P > n_pert) P = n_pert;
   if (P < 1) P = 1;
   g.P = P;
@@ -725,7 +843,7 @@ TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T) 
   return g;
 }
 
-bool tc_supported(int B) { return B >= 1 && B <= 128; }
+bool tc_supported(int B) { return B >= 1 && B <= 64; }
 
 TcSizes tc_sizes(const TcGeom& g) {
   TcSizes z;
@@ -733,7 +851,7 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.w16 = N * g.MT * g.S * kTileA;
   z.wo16 = N * 2 * g.Sh * kTileA;
   z.op = N * g.S * g.G * g.tileB;
-  z.cst = N * n * 2 * g.B * (size_t)g.Hp * sizeof(float);
+  z.cst = N * n * 2 * (size_t)g.Hp * g.Bp * sizeof(float);
   z.pm = N * n * 2 * g.B * (size_t)g.T * 2 * sizeof(float);
   z.ply = N * n * 2 * g.B * (size_t)g.T * sizeof(float);
   return z;
@@ -742,10 +860,11 @@ TcSizes tc_sizes(const TcGeom& g) {
 cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
                               cudaStream_t stream) {
   const size_t smem = kernel_smem_bytes(g);
-  cudaError_t e = cudaFuncSetAttribute(gate_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(tc_persistent_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  e = cudaFuncSetAttribute(tc_persistent_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
   if (e != cudaSuccess) return e;
   const TcSizes z = tc_sizes(g);
   TcArgs a;
@@ -754,6 +873,8 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.t = 0;
   a.w16 = tb.w16;
   a.wo16 = tb.wo16;
+  a.op_in = tb.op[0];
+  a.op_out = tb.op[1];
   a.cst = tb.cst;
   a.pm = tb.pm;
   a.ps = tb.ps;
@@ -764,29 +885,29 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   prep_tiles_kernel<<<dim3(g.MT * g.S + 2 * g.Sh, g.n_experts), 128, 0, stream>>>(a);
   cudaMemsetAsync(tb.op[0], 0, z.op, stream);
   cudaMemsetAsync(tb.op[1], 0, z.op, stream);
-  a.t = 0;
-  xpart_kernel<<<dim3(g.Sx * g.G, g.n_experts), 128, 0, stream>>>(a, tb.op[0]);
+  const int xblocks = g.n_experts * g.Sx * g.G;
+  xpart_kernel<<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
   trace_end(SOMA_TRACE_PREP, stream);
 
-  const int gate_blocks = g.n_experts * g.MT * g.G;
-  const int head_blocks = g.n_experts * 2 * g.G;
+  const int sms = sm_count();
+  const int gate_tasks = g.n_experts * g.MT * g.G;
+  const int head_tasks = g.n_experts * 2 * g.G;
+  const int gate_ctas = gate_tasks < sms ? gate_tasks : sms;
+  const int head_ctas = head_tasks < sms ? head_tasks : sms;
   for (int t = 0; t < s.T; ++t) {
     a.t = t;
     a.op_in = tb.op[t & 1];
     a.op_out = tb.op[(t + 1) & 1];
     trace_begin(SOMA_TRACE_GATE, stream);
-    gate_tc_kernel<<<gate_blocks, kThreads, smem, stream>>>(a);
+    tc_persistent_kernel<false><<<gate_ctas, kThreads, smem, stream>>>(a, gate_tasks, gate_ctas);
     trace_end(SOMA_TRACE_GATE, stream);
+    // head of timestep t (h part of the operand of t + 1) and, in the same
+    // launch, the embedding part of that operand
     a.op_in = tb.op[(t + 1) & 1];
     trace_begin(SOMA_TRACE_HEAD, stream);
-    head_tc_kernel<<<head_blocks, kThreads, smem, stream>>>(a);
+    tc_persistent_kernel<true><<<head_ctas + (t + 1 < s.T ? xblocks : 0), kThreads, smem,
+                                 stream>>>(a, head_tasks, head_ctas);
     trace_end(SOMA_TRACE_HEAD, stream);
-    if (t + 1 < s.T) {
-      a.t = t + 1;
-      trace_begin(SOMA_TRACE_PREP, stream);
-      xpart_kernel<<<dim3(g.Sx * g.G, g.n_experts), 128, 0, stream>>>(a, tb.op[(t + 1) & 1]);
-      trace_end(SOMA_TRACE_PREP, stream);
-    }
   }
   return cudaGetLastError();
 }

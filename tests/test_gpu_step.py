@@ -198,3 +198,18 @@ def test_large_batch_uses_the_cuda_core_path(oracle_mod):
     theta = inputs.init_params(N, E, H, seed=21, std=0.3)
     bx = inputs.expert_batch(N, B, T, 1, seed=22, step=0)
     _full_parity(oracle_mod, theta, bx, E, H, n, 1e-3, 1e-2, 3, 1)
+
+
+@pytest.mark.parametrize("n", [160, 304])
+def test_many_tasks_per_cta(oracle_mod, n):
+    # more probe groups than SMs: every persistent CTA runs several gate and
+    # head tasks (and the head launch carries the embedding-operand blocks)
+    N, E, H, B, T = 1, 64, 96, 8, 6
+    theta = inputs.init_params(N, E, H, seed=n, std=None)
+    bx = inputs.expert_batch(N, B, T, 2, seed=31, step=0)
+    g = run_step(theta, bx, E, H, n, 1e-3, 1e-3, 4, 2)
+    assert g["status"] == 0
+    probes = [0, 1, 151, 152, 153, n - 2, n - 1]
+    L, coef = oracle_mod.spsa_losses(theta, E, H, np.float32(1e-3), 4, 2, bx, probes=probes)
+    assert_losses(g["losses"][:, probes], L)
+    assert_coefs(g["coef"][:, probes], coef)
