@@ -44,10 +44,16 @@ using namespace tc;
 namespace {
 
 constexpr int kZWarps = 8;
-constexpr int kLoaders = 4;  // one bulk copy stream per issuing thread: several issuers
-constexpr int kThreads = (kLoaders + 1 + kZWarps + 8) * 32;  // loaders, MMA, Z, epilogue
-constexpr int kStages = 6;
-constexpr int kKt = 32;                 // K per stage (fp16 elements)
+constexpr int kStages = 3;
+constexpr int kLoaders = kStages;  // one issuing thread per ring slot (the copies of
+                                   // one thread complete one after another)
+constexpr int kEpiWarps = 8;
+constexpr int kEpiChunks = kEpiWarps / 8;  // 8-sequence chunks interleaved across warps
+constexpr int kZPer = 256 / (kZWarps * 32);  // (probe, row) pairs per generator thread
+static_assert(kZPer * kZWarps * 32 == 256, "Z generators cover 2 probes x 128 rows");
+static_assert(kEpiWarps % 8 == 0, "epilogue warps cover 4 lane quarters x 2 probes");
+constexpr int kThreads = (kLoaders + 1 + kZWarps + kEpiWarps) * 32;  // loaders, MMA, Z, epilogue
+constexpr int kKt = 64;                 // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
 constexpr uint32_t kSbo = kKt * 16;     // bytes between 8-row groups
 constexpr uint32_t kLbo = 128;          // bytes between core matrices along K
@@ -105,31 +111,19 @@ __device__ __forceinline__ uint32_t z_run_raw(const ProbeKey& pk, int64_t p0, ZS
   return natural_to_raw(probe_bits32(pk, p0));
 }
 
-// Writes the 128 x 32 Z tile row r (one 32-parameter run) in the canonical
-// K-major layout; `row` points at element (r, 0), the four 8-element chunks
-// of the row are 128 bytes apart.
+// Writes 32 elements of a Z tile row in the canonical K-major layout from one
+// raw word; `row` points at the first element, consecutive 8-element chunks
+// are 128 bytes apart.
 __device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw) {
   uint4 c0, c1, c2, c3;
-  c0.x = pm1_pair<0>(raw);  c0.y = pm1_pair<1>(raw);  c0.z = pm1_pair<2>(raw);  c0.w = pm1_pair<3>(raw);
-  c1.x = pm1_pair<4>(raw);  c1.y = pm1_pair<5>(raw);  c1.z = pm1_pair<6>(raw);  c1.w = pm1_pair<7>(raw);
-  c2.x = pm1_pair<8>(raw);  c2.y = pm1_pair<9>(raw);  c2.z = pm1_pair<10>(raw); c2.w = pm1_pair<11>(raw);
-  c3.x = pm1_pair<12>(raw); c3.y = pm1_pair<13>(raw); c3.z = pm1_pair<14>(raw); c3.w = pm1_pair<15>(raw);
+  c0.x = pm_pair<0>(raw, 0x3C003C00u);  c0.y = pm_pair<1>(raw, 0x3C003C00u);  c0.z = pm_pair<2>(raw, 0x3C003C00u);  c0.w = pm_pair<3>(raw, 0x3C003C00u);
+  c1.x = pm_pair<4>(raw, 0x3C003C00u);  c1.y = pm_pair<5>(raw, 0x3C003C00u);  c1.z = pm_pair<6>(raw, 0x3C003C00u);  c1.w = pm_pair<7>(raw, 0x3C003C00u);
+  c2.x = pm_pair<8>(raw, 0x3C003C00u);  c2.y = pm_pair<9>(raw, 0x3C003C00u);  c2.z = pm_pair<10>(raw, 0x3C003C00u); c2.w = pm_pair<11>(raw, 0x3C003C00u);
+  c3.x = pm_pair<12>(raw, 0x3C003C00u); c3.y = pm_pair<13>(raw, 0x3C003C00u); c3.z = pm_pair<14>(raw, 0x3C003C00u); c3.w = pm_pair<15>(raw, 0x3C003C00u);
   *reinterpret_cast<uint4*>(row) = c0;
   *reinterpret_cast<uint4*>(row + 128) = c1;
   *reinterpret_cast<uint4*>(row + 256) = c2;
   *reinterpret_cast<uint4*>(row + 384) = c3;
-}
-
-__device__ __forceinline__ void store_z_row(uint8_t* ztile, int r, uint32_t raw) {
-  uint4 c0, c1, c2, c3;
-  c0.x = pm1_pair<0>(raw);  c0.y = pm1_pair<1>(raw);  c0.z = pm1_pair<2>(raw);  c0.w = pm1_pair<3>(raw);
-  c1.x = pm1_pair<4>(raw);  c1.y = pm1_pair<5>(raw);  c1.z = pm1_pair<6>(raw);  c1.w = pm1_pair<7>(raw);
-  c2.x = pm1_pair<8>(raw);  c2.y = pm1_pair<9>(raw);  c2.z = pm1_pair<10>(raw); c2.w = pm1_pair<11>(raw);
-  c3.x = pm1_pair<12>(raw); c3.y = pm1_pair<13>(raw); c3.z = pm1_pair<14>(raw); c3.w = pm1_pair<15>(raw);
-  *reinterpret_cast<uint4*>(ztile + kmajor_offset(r, 0, kKt)) = c0;
-  *reinterpret_cast<uint4*>(ztile + kmajor_offset(r, 8, kKt)) = c1;
-  *reinterpret_cast<uint4*>(ztile + kmajor_offset(r, 16, kKt)) = c2;
-  *reinterpret_cast<uint4*>(ztile + kmajor_offset(r, 24, kKt)) = c3;
 }
 
 // ---------------------------------------------------------------------------
@@ -137,15 +131,17 @@ __device__ __forceinline__ void store_z_row(uint8_t* ztile, int r, uint32_t raw)
 // tasks (blockIdx.x, blockIdx.x + n_ctas, ...; the head launch appends
 // n_ctas-independent blocks for the embedding operand, so the stride is
 // n_ctas, not the grid size).  Roles:
-//   warps 0..3    loaders: warp j bulk-copies the A tile and the operand
-//                 group tile of every stage gs = j (mod 4) into a ring of
-//                 kStages shared-memory slots (the copies of one issuing
-//                 thread complete one after another, so four issue them);
-//   warp 4        MMA issuer: W x operand and Z_p x operand_p per stage into
+//   warps 0..2    loaders: warp j bulk-copies the A tile and the operand
+//                 group tile of every stage that uses ring slot j (16 KB
+//                 copies; the copies of one issuing thread complete one
+//                 after another, so each slot has its own issuer);
+//   warp 3        MMA issuer: W x operand and Z_p x operand_p per stage into
 //                 one of two TMEM accumulator buffers (256 columns each);
-//   warps 5..12   Z generators: the +-1 tiles of the stage, from Philox;
-//   warps 13..20  epilogue: reads a finished accumulator buffer while the
-//                 MMAs of the next task fill the other one.
+//   warps 4..11   Z generators: the +-1 tiles of the stage, from Philox
+//                 (one (probe, row) pair per thread);
+//   warps 12..19  epilogue: reads a finished accumulator buffer while the
+//                 MMAs of the next task fill the other one; warp w reads the
+//                 TMEM lanes of quarter w % 4 for probe (w - 12) / 4.
 // Barriers: load_full / z_full (slot filled), slot_free (the slot's MMAs are
 // done), acc_full (a buffer's task is accumulated), acc_empty (its epilogue
 // has read it).  Every wait is bounded (wait_or_abort).
@@ -153,7 +149,6 @@ __device__ __forceinline__ void store_z_row(uint8_t* ztile, int r, uint32_t raw)
 constexpr int kMmaWarp = kLoaders;
 constexpr int kZWarp0 = kMmaWarp + 1;
 constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
-constexpr int kEpiWarps = 8;
 constexpr int kAccCols = 256;
 
 struct Ctl {
@@ -255,7 +250,7 @@ __device__ __forceinline__ void load_chunk(uint32_t tl, uint32_t cw, int Bp, boo
 // Gate epilogue of one task for one warp: probe p = half, TMEM lanes of the
 // warp's quarter: gates, cell update (fp32 per sign), next operand.
 __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
-                              int q4, int p) {
+                              int q4, int p, int c0) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
@@ -273,7 +268,10 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
-  uint8_t* out_tile = a.op_out + (((size_t)T.e * g.S + g.Sx + T.m) * g.G + T.grp) * g.tileB;
+  // a 64-wide stage of the next operand holds two 32-unit row tiles
+  uint8_t* out_tile =
+      a.op_out + (((size_t)T.e * g.S + g.Sx + (T.m >> 1)) * g.G + T.grp) * g.tileB;
+  const int kk = 32 * (T.m & 1) + u_loc;
   const int i = T.grp * g.P + p;
   float bias = 0.f, dbias = 0.f;
   if (unit_ok) {
@@ -284,7 +282,7 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
   const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
   const bool owns_cell = sign_lane && unit_ok;
   float* cbase = a.cst + ((lane_plus + (gate & 1)) * g.Hp + U) * (int64_t)g.Bp;
-  for (int b0 = 0; b0 < g.Bp; b0 += 8) {
+  for (int b0 = 8 * c0; b0 < g.Bp; b0 += 8 * kEpiChunks) {
     float cprev[8];
     if (owns_cell && a.t > 0) {
       const float4 x = *reinterpret_cast<const float4*>(cbase + b0);
@@ -323,7 +321,7 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
       if (owns_cell && b < s.B) {
         const float val = plus ? 0.5f * (hp + hm) : 0.5f * (hp - hm);
         const int row = 2 * g.Bp * p + (plus ? b : g.Bp + b);
-        *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, u_loc, kKt)) =
+        *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, kk, kKt)) =
             __float2half_rn(val);
       }
     }
@@ -339,7 +337,7 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
 // four quarters of the half through shared memory (`red`, [P][Bp][2][4]);
 // the lane whose row is the target byte writes the target logit.
 __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
-                              int q4, int p, float2* red) {
+                              int q4, int p, int c0, float2* red) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
@@ -355,7 +353,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
     const int i = T.grp * g.P + p;
     const float dbo = do_z ? ((probe_bits32(pk, L.b_out + v) & 1u) ? -eps : eps) : 0.f;
     const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
-    for (int b0 = 0; b0 < g.Bp; b0 += 8) {
+    for (int b0 = 8 * c0; b0 < g.Bp; b0 += 8 * kEpiChunks) {
       float wv[8], wd[8], zv[8], zd[8];
       load_chunk(tl, (uint32_t)(2 * g.Bp * p + b0), g.Bp, do_z, wv, wd, zv, zd);
 #pragma unroll
@@ -390,7 +388,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
       }
     }
   }
-  // all eight epilogue warps: partials of this task are in `red`
+  // all epilogue warps: partials of this task are in `red`
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
   const int et = threadIdx.x - kEpiWarp0 * 32;
   const int n_red = T.p_valid * g.Bp * 2;
@@ -472,8 +470,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
       const Task T = make_task<HEAD>(a, task);
       for (int st = 0; st < nst; ++st, ++gs) {
-        if ((int)(gs % kLoaders) != warp) continue;
         const int q = gs % kStages;
+        if (q != warp) continue;
         const uint32_t use = gs / kStages;
         if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
           continue;
@@ -540,27 +538,39 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   } else if (warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
     if (do_z) {
+      // pairs (probe, row) gtid + j * 32 kZWarps, row = gtid & 127
       const int gtid = tid - kZWarp0 * 32;
-      const int p = gtid >> 7, r = gtid & 127;  // one (probe, row) pair per thread
+      const int r = gtid & 127, pb = gtid >> 7;
       uint32_t gs = 0;
       for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
         const Task T = make_task<HEAD>(a, task);
-        const bool active = p < T.p_valid;
-        ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
-        ZSlot cache;
-        cache.blk = 0xFFFFFFFFu;
+        ProbeKey pk[kZPer];
+        ZSlot cache[kZPer];
+#pragma unroll
+        for (int j = 0; j < kZPer; ++j) {
+          const int pj = pb + j * (kZWarps / 4);
+          pk[j] = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pj));
+          cache[j].blk = 0xFFFFFFFFu;
+        }
         const int split = HEAD ? nst : g.Sx;
         const int64_t seg0 = z_param<HEAD>(a, T, r, 0);
         const int64_t seg1 = z_param<HEAD>(a, T, r, split) - (int64_t)kKt * split;
-        uint8_t* zrow = smem + SL.z_off + p * kTileA + kmajor_offset(r, 0, kKt);
+        uint8_t* zrow = smem + SL.z_off + kmajor_offset(r, 0, kKt);
         for (int st = 0; st < nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
           if (gs >= kStages) wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status);
-          if (active && !*abort) {
+          if (!*abort) {
             const int64_t p0 = (st < split ? seg0 : seg1) + (int64_t)kKt * st;
-            const uint32_t raw = z_run_raw(pk, p0, cache);
-            store_z_row_at(zrow + q * SL.bytes, raw);
+#pragma unroll
+            for (int j = 0; j < kZPer; ++j) {
+              const int pj = pb + j * (kZWarps / 4);
+              if (pj < T.p_valid) {
+                uint8_t* zr = zrow + q * SL.bytes + pj * kTileA;
+                store_z_row_at(zr, z_run_raw(pk[j], p0, cache[j]));
+                store_z_row_at(zr + 4 * 128, z_run_raw(pk[j], p0 + 32, cache[j]));
+              }
+            }
           }
           fence_async_smem();
           __syncwarp();
@@ -572,7 +582,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // --------------------------------------------------------------- epilogue
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
-    const int p = ew >> 2;  // probe of the group handled by this warp
+    const int p = (ew >> 2) & 1;  // probe of the group handled by this warp
+    const int c0 = ew >> 3;       // first 8-sequence chunk (then every other one)
     int k = 0;
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
       const Task T = make_task<HEAD>(a, task);
@@ -583,9 +594,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const ProbeKey pk =
           make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
       if (HEAD) {
-        head_epilogue(a, T, tacc, pk, q4, p, red);
+        head_epilogue(a, T, tacc, pk, q4, p, c0, red);
       } else if (p < T.p_valid) {
-        gate_epilogue(a, T, tacc, pk, q4, p);
+        gate_epilogue(a, T, tacc, pk, q4, p, c0);
       }
       tc_fence_before();
       __syncwarp();

@@ -145,6 +145,33 @@ __device__ __forceinline__ void mma_f16_ss_lohi(uint32_t d_tmem, uint32_t a_lo, 
       : "memory");
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]^T: A is 128 lanes (rows) x 8 columns, each
+// 32-bit column holding the k pair (2c, 2c + 1) of fp16 values.
+__device__ __forceinline__ void mma_f16_ts_lohi(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo,
+                                                uint32_t b_hi, uint32_t idesc,
+                                                uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n .reg .b64 db;\n setp.ne.b32 p, %5, 0;\n"
+      " mov.b64 db, {%2, %3};\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// 16 consecutive 32-bit columns of this thread's TMEM lane <- r[0..15].
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // D[tmem] (+)= A[smem] * B[smem]^T  (M x N x 16), issued by one thread.
 __device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                            uint32_t idesc, uint32_t accumulate) {
@@ -205,12 +232,13 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
 }
 
 // Expands one raw probe word (parameter 2j of the run at bit j, parameter
-// 2j+1 at bit j+16) into the fp16 pair word j of +-1 values: bit 1 <=> -1.
-// Element 2j lands in the low half (bit 15 = sign), 2j+1 in the high half.
+// 2j+1 at bit j+16) into the fp16 pair word j of +-m values, m given as the
+// doubled fp16 bit pattern mag2 = bits(m) * 0x10001: bit 1 <=> -m.  Element 2j
+// lands in the low half (bit 15 = sign), 2j+1 in the high half.
 template <int J>
-__device__ __forceinline__ uint32_t pm1_pair(uint32_t raw) {
+__device__ __forceinline__ uint32_t pm_pair(uint32_t raw, uint32_t mag2) {
   static_assert(J >= 0 && J < 16, "pair index");
-  return ((raw << (15 - J)) & 0x80008000u) | 0x3C003C00u;
+  return ((raw << (15 - J)) & 0x80008000u) | mag2;
 }
 
 }  // namespace tc
