@@ -49,8 +49,7 @@ constexpr int kLoaders = kStages;  // one issuing thread per ring slot (the copi
                                    // one thread complete one after another)
 constexpr int kEpiWarps = 8;
 constexpr int kEpiChunks = kEpiWarps / 8;  // 8-sequence chunks interleaved across warps
-constexpr int kZPer = 256 / (kZWarps * 32);  // (probe, row) pairs per generator thread
-static_assert(kZPer * kZWarps * 32 == 256, "Z generators cover 2 probes x 128 rows");
+static_assert(kZWarps * 32 == 256, "one Z generator thread per (probe, row): 2 x 128");
 static_assert(kEpiWarps % 8 == 0, "epilogue warps cover 4 lane quarters x 2 probes");
 constexpr int kThreads = (kLoaders + 1 + kZWarps + kEpiWarps) * 32;  // loaders, MMA, Z, epilogue
 constexpr int kKt = 64;                 // K per stage (fp16 elements)
@@ -126,6 +125,28 @@ __device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw) {
   *reinterpret_cast<uint4*>(row + 384) = c3;
 }
 
+// The MMAs of one stage, fully unrolled over K (NP = probes with a Z tile):
+// W x operand into [0, rowsB) and Z_p x operand_p into kZCols + 2 Bp p.  The
+// descriptors arrive as their low words (start address of the stage's tiles;
+// a step along K or to the next probe is an addition), so the issuing thread
+// spends a few instructions per MMA and keeps the tensor pipe fed.
+template <int NP>
+__device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo, uint32_t z_lo,
+                                            uint32_t hi, uint32_t zp_step, uint32_t bp_step,
+                                            uint32_t idesc_w, uint32_t idesc_z, uint32_t dz_step,
+                                            uint32_t acc0) {
+#pragma unroll
+  for (int k16 = 0; k16 < kKt / 16; ++k16) {
+    const uint32_t ko = (uint32_t)k16 * 16;
+    const uint32_t acc = k16 > 0 ? 1u : acc0;
+    mma_f16_ss_lohi(d, a_lo + ko, hi, b_lo + ko, hi, idesc_w, acc);
+    if (NP >= 1) mma_f16_ss_lohi(d + kZCols, z_lo + ko, hi, b_lo + ko, hi, idesc_z, acc);
+    if (NP >= 2)
+      mma_f16_ss_lohi(d + kZCols + dz_step, z_lo + ko + zp_step, hi, b_lo + ko + bp_step, hi,
+                      idesc_z, acc);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Persistent warp-specialised kernel.  One CTA per SM walks a static list of
 // tasks (blockIdx.x, blockIdx.x + n_ctas, ...; the head launch appends
@@ -157,17 +178,24 @@ struct Ctl {
   uint64_t slot_free[kStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
+  uint64_t mma_done;
   uint32_t tmem_slot;
   volatile int abort;
 };
 
 // A wait that times out records SOMA_ERR_TIMEOUT in the status word and sets
-// the CTA's abort flag; later waits return at once and the CTA winds down
-// without issuing further copies or MMAs.
+// the CTA's abort flag; a wait that is still pending sees the flag within 64
+// polls and returns false, so the CTA winds down without issuing further
+// copies or MMAs.  A phase that is already complete costs one poll and no
+// read of the flag (the flag shares the shared-memory pipe with the
+// epilogue's shuffles, and every handoff of the main loop passes here).
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               int* status) {
-  if (*abort) return false;
-  if (mbar_wait(bar, parity)) return true;
+  if (mbar_try_wait(bar, parity)) return true;
+  for (uint32_t n = 1; n < (1u << 22); ++n) {
+    if ((n & 63u) == 0 && *abort) return false;
+    if (mbar_try_wait(bar, parity)) return true;
+  }
   *abort = 1;
   atomicCAS(status, 0, kStatusTimeout);
   return false;
@@ -268,10 +296,10 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
-  // a 64-wide stage of the next operand holds two 32-unit row tiles
+  // a stage of the next operand holds kKt / 32 of the 32-unit row tiles
   uint8_t* out_tile =
-      a.op_out + (((size_t)T.e * g.S + g.Sx + (T.m >> 1)) * g.G + T.grp) * g.tileB;
-  const int kk = 32 * (T.m & 1) + u_loc;
+      a.op_out + (((size_t)T.e * g.S + g.Sx + 32 * T.m / kKt) * g.G + T.grp) * g.tileB;
+  const int kk = 32 * T.m % kKt + u_loc;
   const int i = T.grp * g.P + p;
   float bias = 0.f, dbias = 0.f;
   if (unit_ok) {
@@ -454,6 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       mbar_init(&ctl->acc_full[q], 1);
       mbar_init(&ctl->acc_empty[q], kEpiWarps);
     }
+    mbar_init(&ctl->mma_done, 1);
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(&ctl->tmem_slot, kTmemCols);
@@ -465,8 +494,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   if (warp < kLoaders) {
     // ---------------------------------------------------------------- loaders
     // the whole warp walks the stages (so that it never sits diverged at the
-    // CTA barrier); lane 0 issues the copies
+    // CTA barrier); lanes 0 and 1 issue one copy each (the copies of one
+    // thread complete one after another)
     uint32_t gs = 0;
+    int last_use = -1;
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
       const Task T = make_task<HEAD>(a, task);
       for (int st = 0; st < nst; ++st, ++gs) {
@@ -475,15 +506,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         const uint32_t use = gs / kStages;
         if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
           continue;
-        if (lane == 0 && !*abort) {
-          uint8_t* slot = smem + q * SL.bytes;
-          mbar_arrive_expect_tx(&ctl->load_full[q], kTileA + g.tileB);
+        uint8_t* slot = smem + q * SL.bytes;
+        if (lane == 0) mbar_arrive_expect_tx(&ctl->load_full[q], kTileA + g.tileB);
+        __syncwarp();
+        if (lane == 0)
           bulk_g2s(slot + SL.a_off, T.a + (size_t)st * kTileA, kTileA, &ctl->load_full[q]);
+        else if (lane == 1)
           bulk_g2s(slot + SL.b_off, T.b + (size_t)st * g.G * g.tileB, g.tileB, &ctl->load_full[q]);
-        }
+        last_use = (int)use;
         __syncwarp();
       }
     }
+    // copies still in flight land before the CTA exits (after an abort the
+    // MMA warp no longer consumes them)
+    if (last_use >= 0) mbar_wait(&ctl->load_full[warp], (uint32_t)last_use & 1u);
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     // the whole warp waits; lane 0 issues the MMAs and commits
@@ -500,6 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const uint32_t z_lo0 = lo0 + (SL.z_off >> 4);
       const uint32_t zp_step = kTileA >> 4;                       // next probe's Z tile
       const uint32_t bp_step = (uint32_t)(2 * g.Bp / 8) * (kSbo >> 4);  // next probe's rows
+      const uint32_t dz_step = (uint32_t)(2 * g.Bp);                    // next probe's columns
       uint32_t gs = 0;
       int k = 0;
       for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
@@ -518,15 +555,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           if (ok && lane == 0) {
             const uint32_t so = (uint32_t)q * slot_step;
             const uint32_t acc0 = st > 0 ? 1u : 0u;
-#pragma unroll
-            for (int k16 = 0; k16 < kKt / 16; ++k16) {
-              const uint32_t ko = so + (uint32_t)k16 * 16;
-              const uint32_t acc = acc0 | (uint32_t)k16;
-              mma_f16_ss_lohi(d, a_lo0 + ko, hi, b_lo0 + ko, hi, idesc_w, acc);
-              for (int p = 0; p < np; ++p)
-                mma_f16_ss_lohi(d + kZCols + (uint32_t)(2 * g.Bp * p), z_lo0 + ko + p * zp_step, hi,
-                                b_lo0 + ko + p * bp_step, hi, idesc_z, acc);
-            }
+            if (np == 2)
+              issue_stage<2>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
+                             idesc_z, dz_step, acc0);
+            else if (np == 1)
+              issue_stage<1>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
+                             idesc_z, dz_step, acc0);
+            else
+              issue_stage<0>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
+                             idesc_z, dz_step, acc0);
           }
           if (lane == 0) mma_commit(&ctl->slot_free[q]);
           __syncwarp();
@@ -534,47 +571,53 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         if (lane == 0) mma_commit(&ctl->acc_full[buf]);
         __syncwarp();
       }
+      // every MMA of this CTA completes before its tensor memory is freed
+      if (lane == 0) mma_commit(&ctl->mma_done);
+      mbar_wait(&ctl->mma_done, 0);
     }
   } else if (warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
+    // Thread (probe gtid / 128, row gtid % 128).  The raw words of the next
+    // stage are drawn before waiting for its slot, so the Philox rounds
+    // overlap the wait instead of following it.
     if (do_z) {
-      // pairs (probe, row) gtid + j * 32 kZWarps, row = gtid & 127
       const int gtid = tid - kZWarp0 * 32;
-      const int r = gtid & 127, pb = gtid >> 7;
+      const int r = gtid & 127, pz = gtid >> 7;
       uint32_t gs = 0;
       for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
         const Task T = make_task<HEAD>(a, task);
-        ProbeKey pk[kZPer];
-        ZSlot cache[kZPer];
-#pragma unroll
-        for (int j = 0; j < kZPer; ++j) {
-          const int pj = pb + j * (kZWarps / 4);
-          pk[j] = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pj));
-          cache[j].blk = 0xFFFFFFFFu;
-        }
+        const bool active = pz < T.p_valid;
+        const ProbeKey pk =
+            make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pz));
+        ZSlot cache;
+        cache.blk = 0xFFFFFFFFu;
         const int split = HEAD ? nst : g.Sx;
         const int64_t seg0 = z_param<HEAD>(a, T, r, 0);
         const int64_t seg1 = z_param<HEAD>(a, T, r, split) - (int64_t)kKt * split;
-        uint8_t* zrow = smem + SL.z_off + kmajor_offset(r, 0, kKt);
+        uint8_t* zrow = smem + SL.z_off + pz * kTileA + kmajor_offset(r, 0, kKt);
+        uint32_t raw[kKt / 32] = {};
+        if (active) {
+#pragma unroll
+          for (int w = 0; w < kKt / 32; ++w) raw[w] = z_run_raw(pk, seg0 + 32 * w, cache);
+        }
         for (int st = 0; st < nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
-          if (gs >= kStages) wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status);
-          if (!*abort) {
-            const int64_t p0 = (st < split ? seg0 : seg1) + (int64_t)kKt * st;
+          const bool ok =
+              gs < kStages || wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status);
+          if (active && ok) {
+            uint8_t* zr = zrow + q * SL.bytes;
 #pragma unroll
-            for (int j = 0; j < kZPer; ++j) {
-              const int pj = pb + j * (kZWarps / 4);
-              if (pj < T.p_valid) {
-                uint8_t* zr = zrow + q * SL.bytes + pj * kTileA;
-                store_z_row_at(zr, z_run_raw(pk[j], p0, cache[j]));
-                store_z_row_at(zr + 4 * 128, z_run_raw(pk[j], p0 + 32, cache[j]));
-              }
-            }
+            for (int w = 0; w < kKt / 32; ++w) store_z_row_at(zr + w * 4 * 128, raw[w]);
           }
           fence_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->z_full[q]);
+          if (active && st + 1 < nst) {
+            const int64_t p1 = (st + 1 < split ? seg0 : seg1) + (int64_t)kKt * (st + 1);
+#pragma unroll
+            for (int w = 0; w < kKt / 32; ++w) raw[w] = z_run_raw(pk, p1 + 32 * w, cache);
+          }
         }
       }
     }
