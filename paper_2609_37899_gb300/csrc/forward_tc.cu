@@ -48,9 +48,9 @@ constexpr int kStages = 3;
 constexpr int kLoaders = kStages;  // one issuing thread per ring slot (the copies of
                                    // one thread complete one after another)
 constexpr int kEpiWarps = 8;
-constexpr int kEpiChunks = kEpiWarps / 8;  // 8-sequence chunks interleaved across warps
+constexpr int kEpiProbeStep = kEpiWarps / 4;  // warp ew runs probes ew / 4, + kEpiProbeStep, ...
 static_assert(kZWarps * 32 == 256, "one Z generator thread per (probe, row): 2 x 128");
-static_assert(kEpiWarps % 8 == 0, "epilogue warps cover 4 lane quarters x 2 probes");
+static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps: 4 lane quarters x 1 or 2 probes");
 constexpr int kThreads = (kLoaders + 1 + kZWarps + kEpiWarps) * 32;  // loaders, MMA, Z, epilogue
 constexpr int kKt = 64;                 // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
@@ -163,9 +163,10 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 //   warps 12..19  epilogue: reads a finished accumulator buffer while the
 //                 MMAs of the next task fill the other one; warp w reads the
 //                 TMEM lanes of quarter w % 4 for probe (w - 12) / 4.
-// Barriers: load_full / z_full (slot filled), slot_free (the slot's MMAs are
-// done), acc_full (a buffer's task is accumulated), acc_empty (its epilogue
-// has read it).  Every wait is bounded (wait_or_abort).
+// Barriers: full (the slot's copies landed and its Z tiles are written),
+// slot_free (the slot's MMAs are done), acc_full (a buffer's task is
+// accumulated), acc_empty (its epilogue has read it), mma_done (all MMAs of
+// the CTA completed).  Every wait is bounded (wait_or_abort, mbar_wait).
 // ---------------------------------------------------------------------------
 constexpr int kMmaWarp = kLoaders;
 constexpr int kZWarp0 = kMmaWarp + 1;
@@ -173,8 +174,7 @@ constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
 constexpr int kAccCols = 256;
 
 struct Ctl {
-  uint64_t load_full[kStages];
-  uint64_t z_full[kStages];
+  uint64_t full[kStages];
   uint64_t slot_free[kStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
@@ -200,6 +200,14 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   atomicCAS(status, 0, kStatusTimeout);
   return false;
 }
+
+// Gate tile rows: a 128-row tile covers 32 hidden units.  Tile row r lies in
+// TMEM lane quarter r / 32 and holds gate (r / 8) % 4 of unit 8 (r / 32) +
+// r % 8, so one quarter = 8 units x 4 gates, gate-major.  With this order a
+// 16x128b tensor-memory load (rows l / 4 and 8 + l / 4 of a 16-lane half)
+// gives thread l two gates of unit l / 4, and the two halves give all four.
+__host__ __device__ __forceinline__ int tile_unit(int r) { return 8 * (r >> 5) + (r & 7); }
+__host__ __device__ __forceinline__ int tile_gate(int r) { return (r >> 3) & 3; }
 
 struct TcArgs {
   Sweep sw;
@@ -249,169 +257,208 @@ template <bool HEAD>
 __device__ __forceinline__ int64_t z_param(const TcArgs& a, const Task& T, int r, int st) {
   const Layout& L = a.sw.lay;
   if (HEAD) return L.w_out + (int64_t)(128 * T.m + r) * a.g.H + (int64_t)kKt * st;
-  const int64_t R = (int64_t)(r & 3) * a.g.H + 32 * T.m + (r >> 2);  // W row of tile row r
+  const int64_t R = (int64_t)tile_gate(r) * a.g.H + 32 * T.m + tile_unit(r);  // W row of tile row r
   return st < a.g.Sx ? L.w_ih + R * a.g.E + (int64_t)kKt * st
                      : L.w_hh + R * a.g.H + (int64_t)kKt * (st - a.g.Sx);
 }
 
-// The four products of 8 sequences of one probe: W vbar, W dv (columns cw,
-// cw + Bp) and Z vbar, Z dv (the same columns past kZCols); one wait.
-__device__ __forceinline__ void load_chunk(uint32_t tl, uint32_t cw, int Bp, bool do_z, float* wv,
-                                           float* wd, float* zv, float* zd) {
-  uint32_t r0[8], r1[8], r2[8], r3[8];
-  tmem_ld8_nowait(tl + cw, r0);
-  tmem_ld8_nowait(tl + cw + Bp, r1);
-  if (do_z) {
-    tmem_ld8_nowait(tl + kZCols + cw, r2);
-    tmem_ld8_nowait(tl + kZCols + cw + Bp, r3);
-  }
-  tmem_wait_ld();
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    wv[j] = __uint_as_float(r0[j]);
-    wd[j] = __uint_as_float(r1[j]);
-    zv[j] = do_z ? __uint_as_float(r2[j]) : 0.f;
-    zd[j] = do_z ? __uint_as_float(r3[j]) : 0.f;
-  }
-}
-
-// Gate epilogue of one task for one warp: probe p = half, TMEM lanes of the
-// warp's quarter: gates, cell update (fp32 per sign), next operand.
+// Gate epilogue of one task for one warp: probe p, TMEM lane quarter q4
+// (units 8 q4 .. 8 q4 + 7 of the tile).  Thread l runs the cells of unit
+// l / 4 for sequences b0 + l % 4 and b0 + 4 + l % 4 of every 8-sequence
+// chunk, both signs, in fp32: 16x128b loads give it all four gates of its
+// unit (gate-major rows), so no data moves between threads.  Cell state
+// layout: [e, i][Hp][Bp][sign].
 __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
-                              int q4, int p, int c0) {
+                              int q4, int p) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
   const int lane = threadIdx.x & 31;
   const int H = g.H;
-  const int r = 32 * q4 + lane;
-  const int u_loc = r >> 2, gate = r & 3;
-  const int U = 32 * T.m + u_loc;
-  const bool unit_ok = U < H;
-  const uint32_t tl = tacc + ((uint32_t)(32 * q4) << 16);
-  const float sc = (gate == 2) ? 2.f : 1.f;  // tanh(x) = 2 sigmoid(2x) - 1
-  const float add = (gate == 2) ? -1.f : 0.f;
-  const int base = lane & ~3;
-  const bool sign_lane = gate < 2;  // gate 0 lane: sign +, gate 1 lane: sign -
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
+  // bias and its probe sign for the row in this lane's TMEM lane, handed to
+  // the threads that run that row's unit
+  float bias_r = 0.f, dbias_r = 0.f;
+  {
+    const int Ur = 32 * T.m + tile_unit(32 * q4 + lane);
+    if (Ur < H) {
+      const int64_t pb = L.b + (int64_t)tile_gate(32 * q4 + lane) * H + Ur;
+      bias_r = th[pb];
+      if (do_z) dbias_r = (probe_bits32(pk, pb) & 1u) ? -eps : eps;
+    }
+  }
+  const int u8 = lane >> 2, bq = lane & 3;
+  float bias[4], dbias[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    bias[k] = __shfl_sync(0xffffffffu, bias_r, 8 * k + u8);
+    dbias[k] = __shfl_sync(0xffffffffu, dbias_r, 8 * k + u8);
+  }
+  const int U = 32 * T.m + 8 * q4 + u8;
+  const bool unit_ok = U < H;
   // a stage of the next operand holds kKt / 32 of the 32-unit row tiles
   uint8_t* out_tile =
       a.op_out + (((size_t)T.e * g.S + g.Sx + 32 * T.m / kKt) * g.G + T.grp) * g.tileB;
-  const int kk = 32 * T.m % kKt + u_loc;
+  const int kk = 32 * T.m % kKt + 8 * q4 + u8;
   const int i = T.grp * g.P + p;
-  float bias = 0.f, dbias = 0.f;
-  if (unit_ok) {
-    const int64_t pb = L.b + (int64_t)gate * H + U;
-    bias = th[pb];
-    if (do_z) dbias = (probe_bits32(pk, pb) & 1u) ? -eps : eps;
-  }
-  const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
-  const bool owns_cell = sign_lane && unit_ok;
-  float* cbase = a.cst + ((lane_plus + (gate & 1)) * g.Hp + U) * (int64_t)g.Bp;
-  for (int b0 = 8 * c0; b0 < g.Bp; b0 += 8 * kEpiChunks) {
-    float cprev[8];
-    if (owns_cell && a.t > 0) {
-      const float4 x = *reinterpret_cast<const float4*>(cbase + b0);
-      const float4 y = *reinterpret_cast<const float4*>(cbase + b0 + 4);
-      cprev[0] = x.x; cprev[1] = x.y; cprev[2] = x.z; cprev[3] = x.w;
-      cprev[4] = y.x; cprev[5] = y.y; cprev[6] = y.z; cprev[7] = y.w;
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j) cprev[j] = 0.f;
+  float2* cell = reinterpret_cast<float2*>(a.cst) +
+                 (((int64_t)T.e * s.n_pert + i) * g.Hp + U) * (int64_t)g.Bp;
+  const uint32_t tq = tacc + ((uint32_t)(32 * q4) << 16);  // gates 0, 1
+  const uint32_t tq2 = tq + (16u << 16);                    // gates 2, 3
+  for (int b0 = 0; b0 < g.Bp; b0 += 8) {
+    float2 cprev[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    if (unit_ok && a.t > 0) {
+      cprev[0] = cell[b0 + bq];
+      cprev[1] = cell[b0 + 4 + bq];
     }
-    float wv[8], wd[8], zv[8], zd[8], cnew[8];
-    load_chunk(tl, (uint32_t)(2 * g.Bp * p + b0), g.Bp, do_z, wv, wd, zv, zd);
+    // [seq half][gate]: W vbar, W dv, Z vbar, Z dv
+    uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int b = b0 + j;
-      const float C = fmaf(eps, zd[j], wv[j]) + bias;
-      const float D = fmaf(eps, zv[j], wd[j]) + dbias;
-      const float actp = fmaf(sigm(sc * (C + D)), sc, add);
-      const float actm = fmaf(sigm(sc * (C - D)), sc, add);
-      const float ip = __shfl_sync(0xffffffffu, actp, base);
-      const float fp = __shfl_sync(0xffffffffu, actp, base + 1);
-      const float gp = __shfl_sync(0xffffffffu, actp, base + 2);
-      const float op = __shfl_sync(0xffffffffu, actp, base + 3);
-      const float im = __shfl_sync(0xffffffffu, actm, base);
-      const float fm = __shfl_sync(0xffffffffu, actm, base + 1);
-      const float gm = __shfl_sync(0xffffffffu, actm, base + 2);
-      const float om = __shfl_sync(0xffffffffu, actm, base + 3);
-      const bool plus = gate == 0;
-      // lanes of gates 0 and 1 run the cell of sign + and sign - (the other
-      // two lanes compute a copy that is never stored)
-      const float c = plus ? fmaf(fp, cprev[j], ip * gp) : fmaf(fm, cprev[j], im * gm);
-      cnew[j] = c;
-      const float h = (plus ? op : om) * fmaf(sigm(2.f * c), 2.f, -1.f);
-      const float hp = __shfl_sync(0xffffffffu, h, base);
-      const float hm = __shfl_sync(0xffffffffu, h, base + 1);
-      if (owns_cell && b < s.B) {
-        const float val = plus ? 0.5f * (hp + hm) : 0.5f * (hp - hm);
-        const int row = 2 * g.Bp * p + (plus ? b : g.Bp + b);
-        *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, kk, kKt)) =
-            __float2half_rn(val);
+    for (int h = 0; h < 2; ++h) {
+      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0 + 4 * h);
+      tmem_ld_16x128b(tq + cw, wv[h][0], wv[h][1]);
+      tmem_ld_16x128b(tq2 + cw, wv[h][2], wv[h][3]);
+      tmem_ld_16x128b(tq + cw + g.Bp, wd[h][0], wd[h][1]);
+      tmem_ld_16x128b(tq2 + cw + g.Bp, wd[h][2], wd[h][3]);
+      if (do_z) {
+        tmem_ld_16x128b(tq + kZCols + cw, zv[h][0], zv[h][1]);
+        tmem_ld_16x128b(tq2 + kZCols + cw, zv[h][2], zv[h][3]);
+        tmem_ld_16x128b(tq + kZCols + cw + g.Bp, zd[h][0], zd[h][1]);
+        tmem_ld_16x128b(tq2 + kZCols + cw + g.Bp, zd[h][2], zd[h][3]);
       }
     }
-    if (owns_cell) {
-      *reinterpret_cast<float4*>(cbase + b0) = make_float4(cnew[0], cnew[1], cnew[2], cnew[3]);
-      *reinterpret_cast<float4*>(cbase + b0 + 4) = make_float4(cnew[4], cnew[5], cnew[6], cnew[7]);
+    tmem_wait_ld();
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float actp[4], actm[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float zvk = do_z ? __uint_as_float(zv[h][k]) : 0.f;
+        const float zdk = do_z ? __uint_as_float(zd[h][k]) : 0.f;
+        const float C = fmaf(eps, zdk, __uint_as_float(wv[h][k])) + bias[k];
+        const float D = fmaf(eps, zvk, __uint_as_float(wd[h][k])) + dbias[k];
+        if (k == 2) {  // g: tanh(x) = 2 sigmoid(2x) - 1
+          actp[k] = fmaf(sigm(2.f * (C + D)), 2.f, -1.f);
+          actm[k] = fmaf(sigm(2.f * (C - D)), 2.f, -1.f);
+        } else {
+          actp[k] = sigm(C + D);
+          actm[k] = sigm(C - D);
+        }
+      }
+      const float cp = fmaf(actp[1], cprev[h].x, actp[0] * actp[2]);
+      const float cm = fmaf(actm[1], cprev[h].y, actm[0] * actm[2]);
+      const float hp = actp[3] * fmaf(sigm(2.f * cp), 2.f, -1.f);
+      const float hm = actm[3] * fmaf(sigm(2.f * cm), 2.f, -1.f);
+      const int b = b0 + 4 * h + bq;
+      if (unit_ok) {
+        cell[b] = make_float2(cp, cm);
+        if (b < s.B) {
+          const int row = 2 * g.Bp * p + b;
+          *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, kk, kKt)) =
+              __float2half_rn(0.5f * (hp + hm));
+          *reinterpret_cast<__half*>(out_tile + kmajor_offset(row + g.Bp, kk, kKt)) =
+              __float2half_rn(0.5f * (hp - hm));
+        }
+      }
     }
   }
 }
 
-// Head epilogue of one task: logits +- of the warp's 32 vocabulary rows for
-// probe p; per (sequence, sign) max and sum-exp over the warp, merged over the
-// four quarters of the half through shared memory (`red`, [P][Bp][2][4]);
-// the lane whose row is the target byte writes the target logit.
-__device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
-                              int q4, int p, int c0, float2* red) {
+// Head epilogue of one task: logits +- of the 32 vocabulary rows of the
+// warp's lane quarter for each probe the warp runs.  16x128b loads give
+// thread l four rows (l / 4 + {0, 8, 16, 24}) of sequence b0 + l % 4, so
+// the per-(sequence, sign) max and sum-exp over the quarter reduce four rows
+// in registers and then across the eight threads of that sequence (three
+// shuffle rounds).  The four quarters of the half merge through shared
+// memory (`red`, [P][Bp][2][4]); the thread holding the target byte's row
+// writes the target logit.
+__device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int q4, int ew,
+                              float2* red) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
   const int lane = threadIdx.x & 31;
-  const int v = 128 * T.m + 32 * q4 + lane;
-  const uint32_t tl = tacc + ((uint32_t)(32 * q4) << 16);
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
-  const float bo = th[L.b_out + v];
+  const int vq = 128 * T.m + 32 * q4;  // first vocabulary row of the quarter
+  const float bo_r = th[L.b_out + vq + lane];
   const int t = a.t;
-  if (p < T.p_valid) {
+  const int bq = lane & 3, r4 = lane >> 2;
+  // rows of this thread: vq + r4 + 8 k, k = 0..3 (k = 2 h + reg)
+  float bo[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) bo[k] = __shfl_sync(0xffffffffu, bo_r, r4 + 8 * k);
+  const uint32_t tq = tacc + ((uint32_t)(32 * q4) << 16);
+  const uint32_t tq2 = tq + (16u << 16);
+  for (int p = ew >> 2; p < g.P; p += kEpiProbeStep) {
+    if (p >= T.p_valid) continue;
     const int i = T.grp * g.P + p;
-    const float dbo = do_z ? ((probe_bits32(pk, L.b_out + v) & 1u) ? -eps : eps) : 0.f;
+    float dbo[4] = {0.f, 0.f, 0.f, 0.f};
+    if (do_z) {
+      const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)i);
+      const float dbo_r = (probe_bits32(pk, L.b_out + vq + lane) & 1u) ? -eps : eps;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) dbo[k] = __shfl_sync(0xffffffffu, dbo_r, r4 + 8 * k);
+    }
     const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
-    for (int b0 = 8 * c0; b0 < g.Bp; b0 += 8 * kEpiChunks) {
-      float wv[8], wd[8], zv[8], zd[8];
-      load_chunk(tl, (uint32_t)(2 * g.Bp * p + b0), g.Bp, do_z, wv, wd, zv, zd);
+    for (int b0 = 0; b0 < g.Bp; b0 += 4) {
+      // [k]: W vbar, W dv, Z vbar, Z dv of row r4 + 8 k, sequence b0 + bq
+      uint32_t wv[4], wd[4], zv[4] = {0u, 0u, 0u, 0u}, zd[4] = {0u, 0u, 0u, 0u};
+      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0);
+      tmem_ld_16x128b(tq + cw, wv[0], wv[1]);
+      tmem_ld_16x128b(tq2 + cw, wv[2], wv[3]);
+      tmem_ld_16x128b(tq + cw + g.Bp, wd[0], wd[1]);
+      tmem_ld_16x128b(tq2 + cw + g.Bp, wd[2], wd[3]);
+      if (do_z) {
+        tmem_ld_16x128b(tq + kZCols + cw, zv[0], zv[1]);
+        tmem_ld_16x128b(tq2 + kZCols + cw, zv[2], zv[3]);
+        tmem_ld_16x128b(tq + kZCols + cw + g.Bp, zd[0], zd[1]);
+        tmem_ld_16x128b(tq2 + kZCols + cw + g.Bp, zd[2], zd[3]);
+      }
+      tmem_wait_ld();
+      float lp[4], lm[4];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int b = b0 + j;
-        const float C = fmaf(eps, zd[j], wv[j]) + bo;
-        const float D = fmaf(eps, zv[j], wd[j]) + dbo;
-        const float lp = C + D, lm = C - D;
-        float mp = lp, mm = lm;
+      for (int k = 0; k < 4; ++k) {
+        const float C = fmaf(eps, __uint_as_float(zd[k]), __uint_as_float(wv[k])) + bo[k];
+        const float D = fmaf(eps, __uint_as_float(zv[k]), __uint_as_float(wd[k])) + dbo[k];
+        lp[k] = C + D;
+        lm[k] = C - D;
+      }
+      float mp = fmaxf(fmaxf(lp[0], lp[1]), fmaxf(lp[2], lp[3]));
+      float mm = fmaxf(fmaxf(lm[0], lm[1]), fmaxf(lm[2], lm[3]));
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          mp = fmaxf(mp, __shfl_xor_sync(0xffffffffu, mp, o));
-          mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
-        }
-        float sp = __expf(lp - mp), sm_ = __expf(lm - mm);
+      for (int o = 4; o < 32; o <<= 1) {
+        mp = fmaxf(mp, __shfl_xor_sync(0xffffffffu, mp, o));
+        mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
+      }
+      float sp = 0.f, sm_ = 0.f;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          sp += __shfl_xor_sync(0xffffffffu, sp, o);
-          sm_ += __shfl_xor_sync(0xffffffffu, sm_, o);
-        }
-        if (lane == 0) {
-          red[((p * g.Bp + b) * 2 + 0) * 4 + q4] = make_float2(mp, sp);
-          red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
-        }
-        if (b < s.B) {
-          const int y = s.bytes[((int64_t)T.e * s.B + b) * (s.T + 1) + t + 1];
-          if (y == v) {
-            a.ply[((lane_plus + 0) * s.B + b) * (int64_t)s.T + t] = lp;
-            a.ply[((lane_plus + 1) * s.B + b) * (int64_t)s.T + t] = lm;
-          }
+      for (int k = 0; k < 4; ++k) {
+        sp += __expf(lp[k] - mp);
+        sm_ += __expf(lm[k] - mm);
+      }
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        sp += __shfl_xor_sync(0xffffffffu, sp, o);
+        sm_ += __shfl_xor_sync(0xffffffffu, sm_, o);
+      }
+      const int b = b0 + bq;
+      if (r4 == 0) {
+        red[((p * g.Bp + b) * 2 + 0) * 4 + q4] = make_float2(mp, sp);
+        red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
+      }
+      if (b < s.B) {
+        const int y = s.bytes[((int64_t)T.e * s.B + b) * (s.T + 1) + t + 1] - vq - r4;
+        // y = 8 k for the thread that holds the target row
+        if (y >= 0 && y < 32 && (y & 7) == 0) {
+          const int k = y >> 3;
+          const float vp = k == 0 ? lp[0] : k == 1 ? lp[1] : k == 2 ? lp[2] : lp[3];
+          const float vm = k == 0 ? lm[0] : k == 1 ? lm[1] : k == 2 ? lm[2] : lm[3];
+          a.ply[((lane_plus + 0) * s.B + b) * (int64_t)s.T + t] = vp;
+          a.ply[((lane_plus + 1) * s.B + b) * (int64_t)s.T + t] = vm;
         }
       }
     }
@@ -474,8 +521,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   if (tid == 0) {
     ctl->abort = 0;
     for (int q = 0; q < kStages; ++q) {
-      mbar_init(&ctl->load_full[q], 1);
-      mbar_init(&ctl->z_full[q], kZWarps);
+      // the loader's arrival (with the copies' bytes) and, when probes are
+      // generated, one arrival per Z warp: the MMA warp waits once per stage
+      mbar_init(&ctl->full[q], do_z ? 1 + kZWarps : 1);
       mbar_init(&ctl->slot_free[q], 1);
     }
     for (int q = 0; q < 2; ++q) {
@@ -507,19 +555,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
           continue;
         uint8_t* slot = smem + q * SL.bytes;
-        if (lane == 0) mbar_arrive_expect_tx(&ctl->load_full[q], kTileA + g.tileB);
+        if (lane == 0) mbar_arrive_expect_tx(&ctl->full[q], kTileA + g.tileB);
         __syncwarp();
         if (lane == 0)
-          bulk_g2s(slot + SL.a_off, T.a + (size_t)st * kTileA, kTileA, &ctl->load_full[q]);
+          bulk_g2s(slot + SL.a_off, T.a + (size_t)st * kTileA, kTileA, &ctl->full[q]);
         else if (lane == 1)
-          bulk_g2s(slot + SL.b_off, T.b + (size_t)st * g.G * g.tileB, g.tileB, &ctl->load_full[q]);
+          bulk_g2s(slot + SL.b_off, T.b + (size_t)st * g.G * g.tileB, g.tileB, &ctl->full[q]);
         last_use = (int)use;
         __syncwarp();
       }
     }
-    // copies still in flight land before the CTA exits (after an abort the
-    // MMA warp no longer consumes them)
-    if (last_use >= 0) mbar_wait(&ctl->load_full[warp], (uint32_t)last_use & 1u);
+    // copies still in flight land before the CTA exits.  After an abort the
+    // Z warps stop arriving and this wait runs to its bound instead; copies
+    // take microseconds, the bound is tenths of a second.
+    if (last_use >= 0) mbar_wait(&ctl->full[warp], (uint32_t)last_use & 1u);
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     // the whole warp waits; lane 0 issues the MMAs and commits
@@ -549,8 +598,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         for (int st = 0; st < nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
-          bool ok = wait_or_abort(&ctl->load_full[q], use & 1u, abort, status);
-          if (do_z) ok = wait_or_abort(&ctl->z_full[q], use & 1u, abort, status) && ok;
+          const bool ok = wait_or_abort(&ctl->full[q], use & 1u, abort, status);
           tc_fence_after();
           if (ok && lane == 0) {
             const uint32_t so = (uint32_t)q * slot_step;
@@ -603,16 +651,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         for (int st = 0; st < nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
-          const bool ok =
-              gs < kStages || wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status);
-          if (active && ok) {
+          // after an abort the generators stop: an arrival on a phase that
+          // can no longer complete would overfill it
+          if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
+            break;
+          if (active) {
             uint8_t* zr = zrow + q * SL.bytes;
 #pragma unroll
             for (int w = 0; w < kKt / 32; ++w) store_z_row_at(zr + w * 4 * 128, raw[w]);
           }
           fence_async_smem();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&ctl->z_full[q]);
+          if (lane == 0) mbar_arrive(&ctl->full[q]);
           if (active && st + 1 < nst) {
             const int64_t p1 = (st + 1 < split ? seg0 : seg1) + (int64_t)kKt * (st + 1);
 #pragma unroll
@@ -625,8 +675,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // --------------------------------------------------------------- epilogue
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
-    const int p = (ew >> 2) & 1;  // probe of the group handled by this warp
-    const int c0 = ew >> 3;       // first 8-sequence chunk (then every other one)
     int k = 0;
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
       const Task T = make_task<HEAD>(a, task);
@@ -634,12 +682,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status);
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)(buf * kAccCols);
-      const ProbeKey pk =
-          make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
       if (HEAD) {
-        head_epilogue(a, T, tacc, pk, q4, p, c0, red);
-      } else if (p < T.p_valid) {
-        gate_epilogue(a, T, tacc, pk, q4, p, c0);
+        head_epilogue(a, T, tacc, q4, ew, red);
+      } else {
+        for (int p = ew >> 2; p < T.p_valid; p += kEpiProbeStep) {
+          const ProbeKey pk =
+              make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
+          gate_epilogue(a, T, tacc, pk, q4, p);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -710,7 +760,7 @@ __global__ void prep_tiles_kernel(const TcArgs a) {
   uint8_t* tile;
   if (tix < g.MT * g.S) {
     const int m = tix / g.S, st = tix % g.S;
-    const int U = 32 * m + (r >> 2), gate = r & 3;
+    const int U = 32 * m + tile_unit(r), gate = tile_gate(r);
     const int64_t R = (int64_t)gate * g.H + U;
     for (int kk = 0; kk < kKt; ++kk) {
       float w = 0.f;

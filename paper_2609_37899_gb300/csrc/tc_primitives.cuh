@@ -220,6 +220,15 @@ __device__ __forceinline__ void tmem_ld8_nowait(uint32_t taddr, uint32_t* r) {
                : "r"(taddr));
 }
 
+// 16x128b shape, one repetition: thread l receives column c + l % 4 of the
+// lanes l / 4 and 8 + l / 4 of the 16-lane group at taddr (the lane field of
+// taddr is the group's first lane).  Valid after tmem_wait_ld().
+__device__ __forceinline__ void tmem_ld_16x128b(uint32_t taddr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("tcgen05.ld.sync.aligned.16x128b.x1.b32 {%0,%1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(taddr));
+}
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
