@@ -41,7 +41,14 @@ UNIT = "perturbed tokens/s"
 # DRAM traffic of one launch of the dominant kernel from an ncu capture
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel
 # source it was taken on.
-TRAFFIC = {}
+TRAFFIC = {
+    # profiles/tc_persistent_kernel_soma_n2.md: the gate launch, captured on
+    # the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
+    "soma_n2": {"bytes_per_launch": 64.05888e6 + 5.80224e6,
+                "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
+                "source_hash": "0fd1afb54fdcb1e9"},
+}
+
 
 def parse():
     ap = argparse.ArgumentParser()

@@ -60,8 +60,15 @@ def rel_l2(a, b):
     return float(np.linalg.norm(a - b) / np.linalg.norm(b))
 
 
+def report(kind, value):
+    """Achieved error, printed for `pytest -s` (the margins quoted in the
+    design notes come from these lines)."""
+    print(f"PARITY {kind} {value:.3e}")
+
+
 def assert_losses(gpu, ref):
     err = np.abs(np.asarray(gpu, np.float64) - ref).max()
+    report("loss_abs", err)
     assert err <= TOL_LOSS, f"loss error {err:.3e} > {TOL_LOSS}"
 
 
@@ -71,6 +78,7 @@ def assert_coefs(gpu, ref):
         r = ref[e]
         d = np.abs(gpu[e] - r)
         rms = np.sqrt(np.mean(r ** 2))
+        report("coef_rel_l2", np.linalg.norm(d) / np.linalg.norm(r))
         assert np.linalg.norm(d) <= TOL_COEF * np.linalg.norm(r), \
             f"expert {e}: coefficient error {np.linalg.norm(d) / np.linalg.norm(r):.3e}"
         assert np.all(d <= TOL_COEF * np.maximum(np.abs(r), rms)), \
