@@ -59,6 +59,13 @@ def parse():
     ap.add_argument("--seq-len", type=int, default=None,
                     help="override the workload's sequence length (small profiling cases)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adam"],
+                    help="sgd: the SPSA step of Eq. main-spsa (dense probes); adam: the "
+                         "paper's optimizer step (Eq. localspsa: --accum estimates, then Adam)")
+    ap.add_argument("--probes", default=None, choices=["dense", "sparse"],
+                    help="probe kind of --optimizer adam (default sparse, as the paper)")
+    ap.add_argument("--accum", type=int, default=1,
+                    help="accumulation batches per --optimizer adam update")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seqs", type=int, default=32,
                     help="sequences in the one-probe sample of the cpu_baseline timing")
@@ -158,7 +165,7 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def cpu_baseline(cfg_name, c, n_seqs):
+def cpu_baseline(cfg_name, c, n_seqs, kind="dense"):
     """The fp64 oracle, as it stands, on the host cores: one probe pair of
     expert 0 over `n_seqs` of its sequences (both signs)."""
     import oracle
@@ -169,11 +176,11 @@ def cpu_baseline(cfg_name, c, n_seqs):
     oracle.build()
     t0 = time.perf_counter()
     oracle.spsa_losses(theta, c["E"], c["H"], np.float32(c["eps"]), 0, 0, bx, probes=[0],
-                       n_threads=cores)
+                       n_threads=cores, kind=kind)
     dt = time.perf_counter() - t0
     toks = 2 * n_seqs * c["seq_len"]
     return {"value": toks / dt, "unit": UNIT, "cores": min(cores, n_seqs), "kind": "oracle",
-            "sample": f"expert 0, probe 0, both signs, {n_seqs} of {c['batch']} sequences x "
+            "sample": f"expert 0, {kind} probe 0, both signs, {n_seqs} of {c['batch']} sequences x "
                       f"{c['seq_len']} bytes ({toks} perturbed tokens) in {dt:.2f} s; OpenMP "
                       f"over sequences, so {min(cores, n_seqs)} of {cores} cores busy"}
 
@@ -251,14 +258,28 @@ def our_arm(args):
         c["seq_len"] = args.seq_len
     N, E, H, n, B, T = c["n_experts"], c["E"], c["H"], c["n_pert"], c["batch"], c["seq_len"]
     K, W = args.steps, args.warmup
+    adam = args.optimizer == "adam"
+    A = args.accum if adam else 1
+    kind = (args.probes or "sparse") if adam else "dense"
+    if not 1 <= A <= api.MAX_ACCUM:
+        raise SystemExit(f"--accum must be in 1..{api.MAX_ACCUM}")
     experts = api.SomaExperts(N, E, H, n, B, T, device=dev)
     experts.init(seed=1000 + rank, std=c["init_std"] or 0.0)
-    # every step gets its own batch: W + K host batches, pinned, and their
-    # HBM-resident copies for the device-timed run
-    host = [torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=s,
-                                                 seq_len=c["seq_len"])).pin_memory()
-            for s in range(W + K)]
-    resident = [h.to(dev) for h in host]
+    # every step gets its own A batches: (W + K) A host batches, pinned, and
+    # their HBM-resident copies for the device-timed run
+    host = [[torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=A * s + a,
+                                                  seq_len=c["seq_len"])).pin_memory()
+             for a in range(A)] for s in range(W + K)]
+    resident = [[h.to(dev) for h in hs] for hs in host]
+
+    def do_step(batches, s):
+        """One step: the SGD step, or A estimates plus the Adam update t = s + 1
+        (App. E hyper-parameters: beta 0.9 / 0.999, delta 1e-8, decay 1e-4)."""
+        if not adam:
+            return experts.step(batches[0], c["eps"], c["lr"], 0, s)[0]
+        losses, _ = experts.adam_step(batches, c["eps"], 0, [A * s + a for a in range(A)],
+                                      t=s + 1, lr=c["lr"], kind=kind)
+        return losses
     stream = torch.cuda.current_stream(dev)
     # written between timed steps so that no step starts with the previous
     # step's data in L2 (129 MB)
@@ -270,7 +291,7 @@ def our_arm(args):
         torch.cuda.synchronize(dev)
 
     for s in range(W):
-        experts.step(resident[s], c["eps"], c["lr"], 0, s)
+        do_step(resident[s], s)
     barrier()
     api.trace_enable(True)
     api.trace_read(reset=True)
@@ -280,7 +301,7 @@ def our_arm(args):
         start.record(stream)
         for s in range(K):
             flush.fill_(s & 0xFF)
-            experts.step(resident[W + s], c["eps"], c["lr"], 0, W + s)
+            do_step(resident[W + s], W + s)
         stop.record(stream)
         barrier()
     api.trace_enable(False)
@@ -290,16 +311,17 @@ def our_arm(args):
 
     # end to end through the public API: H2D of the step's bytes, the step,
     # D2H of its losses, every step
-    losses_host = torch.empty(N, n, 2, dtype=torch.float32).pin_memory()
-    dev_bytes = torch.empty_like(resident[0])
+    losses_host = torch.empty(A, N, n, 2, dtype=torch.float32).pin_memory()
+    dev_bytes = [torch.empty_like(r) for r in resident[0]]
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for s in range(K):
         flush.fill_(s & 0xFF)
-        dev_bytes.copy_(host[W + s], non_blocking=True)
-        losses, _ = experts.step(dev_bytes, c["eps"], c["lr"], 0, W + K + s)
-        losses_host.copy_(losses, non_blocking=True)
+        for a in range(A):
+            dev_bytes[a].copy_(host[W + s][a], non_blocking=True)
+        losses = do_step(dev_bytes, W + K + s)
+        losses_host.copy_(losses.reshape(losses_host.shape), non_blocking=True)
     e1.record(stream)
     barrier()
     ms_e2e = e0.elapsed_time(e1)
@@ -312,7 +334,7 @@ def our_arm(args):
         dist.destroy_process_group()
         return 0
 
-    tok = tokens_per_step(c) * world
+    tok = tokens_per_step(c) * A * world
     value = tok * K / (ms / 1e3)
     gate_ms, gate_n = traced["gate"]
     peaks, peak_src = measured_peaks()
@@ -329,7 +351,10 @@ def our_arm(args):
         "steps_per_s": K / (ms / 1e3),
         "config": {
             "workload": workload_desc(args.config, c),
-            "tokens_per_step_per_gpu": tokens_per_step(c),
+            "optimizer": ("SGD, dense probes (Eq. main-spsa)" if not adam else
+                          f"Adam with coupled decay, {kind} probes, {A} accumulation batch(es) "
+                          "per update (Eq. localspsa)"),
+            "tokens_per_step_per_gpu": tokens_per_step(c) * A,
             "seq_len": T,
             "l2": "flushed between timed steps (a 256 MiB buffer is written before each "
                   "step, inside the timed region)",
@@ -347,14 +372,14 @@ def our_arm(args):
         },
         "kernel_ms": {k: v[0] / K for k, v in traced.items()},
         "e2e": {"value": tok * K / (ms_e2e / 1e3), "unit": UNIT,
-                "h2d_bytes_per_step": int(resident[0].numel()),
-                "d2h_bytes_per_step": int(N * n * 2 * 4)},
+                "h2d_bytes_per_step": int(sum(r.numel() for r in resident[0])),
+                "d2h_bytes_per_step": int(A * N * n * 2 * 4)},
         "gpu_launches": launches,
         "clocks": clk.summary(),
         "status": api.STATUS_NAMES.get(status, status),
     }
     if not args.no_cpu_baseline and world == 1:
-        line["cpu_baseline"] = cpu_baseline(args.config, c, min(args.cpu_sample_seqs, B))
+        line["cpu_baseline"] = cpu_baseline(args.config, c, min(args.cpu_sample_seqs, B), kind)
     print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

@@ -28,7 +28,14 @@
  * parameter index p, regenerated from Philox4x32-10 (Salmon et al., SC'11):
  *   key = (seed & 0xffffffff, seed >> 32)
  *   counter = (p >> 7, i, step & 0xffffffff, e)
- *   bit = bit (p & 31) of output word ((p & 127) >> 5);  z = 1 - 2 bit.
+ *   o = p & 31;  bit = bit (o >> 1) + 16 (o & 1) of output word ((p & 127) >> 5)
+ *   z = 1 - 2 bit   (even offsets of a 32-parameter run read the low half-word,
+ *                    odd offsets the high half-word).
+ * Sparse probes (App. E, the paper's training probes; soma_spsa_estimate and
+ * soma_adam_update): a second, activity bit per coordinate, read with the same
+ * map from the blocks whose counter word 1 is i | 0x80000000;
+ *   z = activity ? 1 - 2 bit : 0,
+ * so a coordinate is 0 with probability 1/2 and -1 or +1 with probability 1/4.
  * No probe is ever stored.
  *
  * Conventions for every entry point:
@@ -119,6 +126,53 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
 int soma_spsa_update(float* params, int n_experts, soma_dims d, int n_pert, float lr,
                      uint64_t seed, uint64_t step, const float* coef, void* stream);
 
+/* ---- The paper's optimizer step (App. E, Eq. localspsa) ----------------
+ * One update averages A accumulation batches, each with its own batch and
+ * probes (step counter steps[a]):
+ *   ghat  = (1/A) sum_a (1/n_pert) sum_i c_{a,e,i} z^{(a)}_{e,i}
+ *   g     = ghat + weight_decay * theta      (coupled decay, before the moments)
+ *   m     = beta1 m + (1 - beta1) g,  v = beta2 v + (1 - beta2) g^2
+ *   theta = theta - lr * (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + delta)
+ * A caller runs soma_spsa_estimate once per accumulation batch (writing its
+ * coefficients into row a of a [A][n_experts][n_pert] buffer), then
+ * soma_adam_update once. */
+typedef enum soma_probe_kind {
+  SOMA_PROBE_DENSE = 0,  /* Rademacher +-1 (Sec. 5, App. F) */
+  SOMA_PROBE_SPARSE = 1  /* 0 w.p. 1/2, -1 or +1 w.p. 1/4 each (App. E) */
+} soma_probe_kind;
+
+#define SOMA_MAX_ACCUM 64
+
+typedef struct soma_adam_config {
+  float lr;           /* eta_t, finite */
+  float beta1;        /* in [0, 1) */
+  float beta2;        /* in [0, 1) */
+  float delta;        /* delta_Adam > 0 (the paper: 1e-8) */
+  float weight_decay; /* lambda >= 0, coupled (the paper: 1e-4) */
+  int32_t t;          /* 1-based update count; m = v = 0 before update 1 */
+} soma_adam_config;
+
+/* Losses and coefficients of one accumulation batch; params are not changed.
+ * Arguments as soma_spsa_step, plus probe_kind (soma_probe_kind); coef_out is
+ * required.  Same workspace size as soma_spsa_step. */
+int soma_spsa_estimate(const float* params, int n_experts, soma_dims d, int n_pert,
+                       int probe_kind, float eps, uint64_t seed, uint64_t step,
+                       const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
+                       float* coef_out, void* workspace, size_t workspace_bytes, void* stream);
+
+/* The Adam update of Eq. localspsa from the coefficients of n_acc
+ * accumulation batches.
+ *   params, m, v  device fp32 [n_experts][P]; updated in place (m, v start at
+ *                 0 and are owned and kept by the caller between updates).
+ *   steps         HOST uint64 [n_acc]: the step counter each batch's probes
+ *                 were drawn with; 1 <= n_acc <= SOMA_MAX_ACCUM.
+ *   coef          device fp32 [n_acc][n_experts][n_pert].
+ * An expert with a non-finite coefficient is left unchanged (params, m, v).
+ * No workspace. */
+int soma_adam_update(float* params, float* m, float* v, int n_experts, soma_dims d, int n_pert,
+                     int probe_kind, uint64_t seed, const uint64_t* steps, int n_acc,
+                     const float* coef, soma_adam_config cfg, void* stream);
+
 /* Synchronises `stream`, then returns and clears the current device's status
  * word (SOMA_OK if no device-side error was recorded since the last call).
  * Returns SOMA_ERR_CUDA if the synchronisation itself failed. */
@@ -127,8 +181,8 @@ int soma_get_status(void* stream);
 /* Static, human-readable name of a status code. */
 const char* soma_status_string(int code);
 
-/* Tracing.  While enabled, every kernel that soma_spsa_step, soma_eval_loss
- * and soma_spsa_update launch is bracketed by two CUDA events recorded on the
+/* Tracing.  While enabled, every kernel that soma_spsa_step, soma_eval_loss,
+ * soma_spsa_estimate, soma_spsa_update and soma_adam_update launch is bracketed by two CUDA events recorded on the
  * caller's stream; soma_trace_read() waits for the recorded events and sums
  * device time and launch counts per kernel class.  Tracing is process-wide
  * and off by default; events are created on first use and reused. */
@@ -152,11 +206,14 @@ int soma_trace_read(soma_kernel_times* out, int reset);
  * soma_debug_philox: out4[j] = Philox4x32-10(ctr4[j], key = seed halves) for
  *   j < count; ctr4 and out4 are device uint32 [count][4].
  * soma_debug_rademacher: z_out[q] = z_{expert,pert}[p0 + q] for q < count,
- *   device int8, using the same bit extraction the kernels use. */
+ *   device int8, using the same bit extraction the kernels use.
+ * soma_debug_probe: the same for either probe kind (soma_probe_kind). */
 int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
                       void* stream);
 int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
                           int64_t count, int8_t* z_out, void* stream);
+int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int probe_kind,
+                     int64_t p0, int64_t count, int8_t* z_out, void* stream);
 /* soma_debug_tc_gemm: d[128][n] = a[128][k] * b[n][k]^T (fp16 inputs as
  *   uint16 bit patterns, row-major; fp32 output) through the same shared-
  *   memory descriptors, tcgen05.mma and tensor-memory read-back as the

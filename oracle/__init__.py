@@ -83,6 +83,24 @@ def _load():
                                            ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
                                            c_dp, c_dp, ctypes.c_int]
         lib.oracle_spsa_losses.restype = ctypes.c_int
+        lib.oracle_spsa_losses_kind.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_double, ctypes.c_int,
+                                                ctypes.c_uint64, ctypes.c_uint64,
+                                                c_u8p, ctypes.c_int, ctypes.c_int,
+                                                ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
+                                                c_dp, c_dp, ctypes.c_int]
+        lib.oracle_spsa_losses_kind.restype = ctypes.c_int
+        lib.oracle_probe.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32,
+                                     ctypes.c_uint32, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
+                                     ctypes.POINTER(ctypes.c_int8)]
+        lib.oracle_probe.restype = ctypes.c_int
+        lib.oracle_adam_update.argtypes = [c_dp, c_dp, c_dp, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_uint64, ctypes.POINTER(ctypes.c_uint64),
+                                           ctypes.c_int, c_dp, ctypes.c_double, ctypes.c_double,
+                                           ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                           ctypes.c_int, c_dp, c_dp, c_dp]
+        lib.oracle_adam_update.restype = ctypes.c_int
         lib.oracle_spsa_update.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            ctypes.c_int, ctypes.c_double, ctypes.c_uint64,
                                            ctypes.c_uint64, c_dp, c_dp]
@@ -129,6 +147,21 @@ def rademacher(seed: int, step: int, expert: int, probe: int, p0: int, count: in
     return z
 
 
+PROBE_KINDS = {"dense": 0, "sparse": 1}
+
+
+def probe(seed: int, step: int, expert: int, probe_index: int, p0: int, count: int,
+          kind: str = "dense") -> np.ndarray:
+    """Probe entries z_{expert,probe}[p0 : p0+count] (int8): dense in {-1, +1},
+    sparse in {-1, 0, +1} (App. E)."""
+    z = np.zeros(count, dtype=np.int8)
+    rc = _load().oracle_probe(seed, step, expert, probe_index, PROBE_KINDS[kind], p0, count,
+                              _ptr(z, ctypes.c_int8))
+    if rc != 0:
+        raise RuntimeError(f"oracle_probe failed ({rc})")
+    return z
+
+
 def loss(theta, E: int, H: int, bytes_, n_threads: int = 0, per_token: bool = False):
     """Mean next-byte cross entropy (nats/byte) of ONE expert.
 
@@ -147,7 +180,7 @@ def loss(theta, E: int, H: int, bytes_, n_threads: int = 0, per_token: bool = Fa
 
 def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
                 probes=None, n_pert: int | None = None, n_threads: int = 0,
-                first_expert: int = 0):
+                first_expert: int = 0, kind: str = "dense"):
     """Antithetic losses and coefficients for the selected probes.
 
     theta [N, P] (fp32 or fp64), bytes_ [N, B, T+1] uint8.  ``probes`` lists
@@ -165,8 +198,8 @@ def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
     sel = np.ascontiguousarray(list(probes), dtype=np.int32)
     L = np.zeros((N, sel.size, 2), dtype=np.float64)
     coef = np.zeros((N, sel.size), dtype=np.float64)
-    rc = _load().oracle_spsa_losses(_ptr(th, ctypes.c_double), N, first_expert, E, H, float(eps),
-                                    seed, step,
+    rc = _load().oracle_spsa_losses_kind(_ptr(th, ctypes.c_double), N, first_expert, E, H,
+                                    float(eps), PROBE_KINDS[kind], seed, step,
                                     _ptr(bx, ctypes.c_uint8), B, T,
                                     _ptr(sel, ctypes.c_int32), sel.size,
                                     _ptr(L, ctypes.c_double), _ptr(coef, ctypes.c_double),
@@ -197,6 +230,33 @@ def spsa_step(theta, E: int, H: int, n_pert: int, eps: float, lr: float, seed: i
                           n_threads=n_threads)
     new = spsa_update(theta, E, H, lr, seed, step, coef)
     return L, coef, new
+
+
+def adam_update(theta, m, v, E: int, H: int, seed: int, steps, coef, lr: float, beta1: float,
+                beta2: float, delta: float, wd: float, t: int, kind: str = "sparse"):
+    """The paper's optimizer step (Eq. localspsa with coupled weight decay).
+
+    theta, m, v [N, P]; steps[A] the probe step counter of each accumulation
+    batch; coef [A, N, n_pert].  Returns (theta', m', v') in fp64."""
+    th = _f64(theta)
+    mm = _f64(m)
+    vv = _f64(v)
+    N = th.shape[0]
+    cf = np.ascontiguousarray(coef, dtype=np.float64)
+    A, n_pert = cf.shape[0], cf.shape[2]
+    st = np.ascontiguousarray(steps, dtype=np.uint64)
+    assert st.size == A and cf.shape[1] == N
+    to, mo, vo = np.zeros_like(th), np.zeros_like(th), np.zeros_like(th)
+    rc = _load().oracle_adam_update(_ptr(th, ctypes.c_double), _ptr(mm, ctypes.c_double),
+                                    _ptr(vv, ctypes.c_double), N, E, H, n_pert,
+                                    PROBE_KINDS[kind], seed, _ptr(st, ctypes.c_uint64), A,
+                                    _ptr(cf, ctypes.c_double), float(lr), float(beta1),
+                                    float(beta2), float(delta), float(wd), int(t),
+                                    _ptr(to, ctypes.c_double), _ptr(mo, ctypes.c_double),
+                                    _ptr(vo, ctypes.c_double))
+    if rc != 0:
+        raise RuntimeError(f"oracle_adam_update failed ({rc})")
+    return to, mo, vo
 
 
 def bptt_grad(theta, E: int, H: int, bytes_):

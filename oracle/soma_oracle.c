@@ -25,7 +25,12 @@
  *     theta <- theta - lr * (1/n_pert) sum_j coef_j z_j (Eq. main-spsa; the
  *     plain-SGD form of Eq. localspsa without moments);
  *   - the exact batch gradient by back-propagation through time (used only
- *     to pin the epsilon -> 0 limit of the estimator, App. F, Prop. 1 proof).
+ *     to pin the epsilon -> 0 limit of the estimator, App. F, Prop. 1 proof);
+ *   - the paper's own optimizer step (App. E, Eq. localspsa): sparse
+ *     Rademacher probes (a coordinate is 0 with probability 1/2 and -1 or +1
+ *     with probability 1/4 each), the estimate averaged over A accumulation
+ *     batches, coupled weight decay added before the moments, and Adam with
+ *     bias-corrected moments.
  *
  * Parameter layout of one expert (flat, row-major, gate blocks i,f,g,o):
  *   Emb[V][E], W_ih[4H][E], W_hh[4H][H], b[4H], W_out[V][H], b_out[V].
@@ -40,6 +45,13 @@
  *   z       = 1 - 2 * bit.
  * Within each word, parameters 2j and 2j+1 of the run read bits j and
  * j + 16: an even/odd interleave of the two 16-bit halves.
+ *
+ * Sparse probes (App. E) use two bits per coordinate from the same key,
+ * step and expert: the sign bit above, and an activity bit taken at the same
+ * position of the block whose counter word 1 is probe | 0x80000000.
+ *   z = (activity bit set) ? 1 - 2 * bit : 0.
+ * A coordinate is therefore nonzero with probability 1/2, and a nonzero
+ * sparse coordinate equals the dense probe's coordinate.
  */
 #include <math.h>
 #include <stdint.h>
@@ -102,6 +114,24 @@ void oracle_rademacher(uint64_t seed, uint64_t step, uint32_t expert,
     uint32_t bit = (w[k >> 5] >> ((o >> 1) + 16 * (o & 1))) & 1u;
     z[q] = (int8_t)(1 - 2 * (int)bit);
   }
+}
+
+/* z_{e,i}[p] for p in [p0, p0 + count) of the given kind: 0 = dense
+ * Rademacher (as above), 1 = sparse (file header).  One Philox call per
+ * parameter and stream, no caching. */
+int oracle_probe(uint64_t seed, uint64_t step, uint32_t expert, uint32_t probe, int kind,
+                 int64_t p0, int64_t count, int8_t* z) {
+  if (kind != 0 && kind != 1) return 1;
+  oracle_rademacher(seed, step, expert, probe, p0, count, z);
+  if (kind == 0) return 0;
+  int8_t* act = (int8_t*)malloc((size_t)(count > 0 ? count : 1));
+  if (!act) return 2;
+  /* the activity stream: same bit map, counter word 1 with its top bit set */
+  oracle_rademacher(seed, step, expert, probe | 0x80000000u, p0, count, act);
+  for (int64_t q = 0; q < count; ++q)
+    if (act[q] == 1) z[q] = 0; /* bit 0 (z would be +1): inactive */
+  free(act);
+  return 0;
 }
 
 /* ------------------------------------------------------------------ */
@@ -226,12 +256,12 @@ double oracle_loss(const double* theta, int E, int H, const uint8_t* bytes,
  *   out_L  [N][n_sel][2] = L(theta_e + eps z), L(theta_e - eps z)
  *   out_coef [N][n_sel]  = (L+ - L-) / (2 eps); 0 when eps == 0.
  * Returns 0 on success. */
-int oracle_spsa_losses(const double* theta, int N, int e0, int E, int H, double eps,
-                       uint64_t seed, uint64_t step, const uint8_t* bytes,
-                       int B, int T, const int32_t* sel, int n_sel,
-                       double* out_L, double* out_coef, int n_threads) {
+int oracle_spsa_losses_kind(const double* theta, int N, int e0, int E, int H, double eps,
+                            int kind, uint64_t seed, uint64_t step, const uint8_t* bytes,
+                            int B, int T, const int32_t* sel, int n_sel,
+                            double* out_L, double* out_coef, int n_threads) {
   int64_t P = oracle_param_count(E, H);
-  if (P <= 0 || N <= 0 || B <= 0 || T <= 0 || n_sel < 0) return 1;
+  if (P <= 0 || N <= 0 || B <= 0 || T <= 0 || n_sel < 0 || (kind != 0 && kind != 1)) return 1;
   double* theta_s = (double*)malloc(sizeof(double) * (size_t)P);
   int8_t* z = (int8_t*)malloc((size_t)P);
   if (!theta_s || !z) { free(theta_s); free(z); return 2; }
@@ -240,7 +270,7 @@ int oracle_spsa_losses(const double* theta, int N, int e0, int E, int H, double 
     const uint8_t* bx = bytes + (int64_t)e * B * (T + 1);
     for (int q = 0; q < n_sel; ++q) {
       int i = sel[q];
-      oracle_rademacher(seed, step, (uint32_t)(e0 + e), (uint32_t)i, 0, P, z);
+      oracle_probe(seed, step, (uint32_t)(e0 + e), (uint32_t)i, kind, 0, P, z);
       double L[2];
       for (int s = 0; s < 2; ++s) {
         double sign = (s == 0) ? 1.0 : -1.0;
@@ -255,6 +285,15 @@ int oracle_spsa_losses(const double* theta, int N, int e0, int E, int H, double 
   free(theta_s);
   free(z);
   return 0;
+}
+
+/* The same with dense probes (Eq. main-spsa). */
+int oracle_spsa_losses(const double* theta, int N, int e0, int E, int H, double eps,
+                       uint64_t seed, uint64_t step, const uint8_t* bytes,
+                       int B, int T, const int32_t* sel, int n_sel,
+                       double* out_L, double* out_coef, int n_threads) {
+  return oracle_spsa_losses_kind(theta, N, e0, E, H, eps, 0, seed, step, bytes, B, T, sel,
+                                 n_sel, out_L, out_coef, n_threads);
 }
 
 /* theta_out = theta - lr * (1/n_pert) * sum_i coef[e][i] z_{e,i}, in fp64.
@@ -277,6 +316,55 @@ int oracle_spsa_update(const double* theta, int N, int E, int H, int n_pert,
     const double* th = theta + (int64_t)e * P;
     double* to = theta_out + (int64_t)e * P;
     for (int64_t p = 0; p < P; ++p) to[p] = th[p] - lr * (g[p] / (double)n_pert);
+  }
+  free(g);
+  free(z);
+  return 0;
+}
+
+/* The paper's optimizer step (App. E, Eq. localspsa), in fp64, for every
+ * expert e:
+ *   ghat[p]  = (1/A) sum_a (1/n_pert) sum_i coef[a][e][i] z_{e,i}^{(a)}[p],
+ *              z^{(a)} drawn with step counter steps[a] (kind 0 dense, 1 sparse)
+ *   g        = ghat + wd * theta            (coupled weight decay, before the moments)
+ *   m        = beta1 m + (1 - beta1) g,     v = beta2 v + (1 - beta2) g^2
+ *   mhat     = m / (1 - beta1^t),           vhat = v / (1 - beta2^t)
+ *   theta'   = theta - lr * mhat / (sqrt(vhat) + delta)
+ * t >= 1 is the update count (m = v = 0 before the first update).
+ * theta, m, v and the outputs are [N][P]; coef is [A][N][n_pert]. */
+int oracle_adam_update(const double* theta, const double* m, const double* v, int N, int E,
+                       int H, int n_pert, int kind, uint64_t seed, const uint64_t* steps, int A,
+                       const double* coef, double lr, double beta1, double beta2, double delta,
+                       double wd, int t, double* theta_out, double* m_out, double* v_out) {
+  int64_t P = oracle_param_count(E, H);
+  if (P <= 0 || N <= 0 || n_pert <= 0 || A <= 0 || t < 1 || (kind != 0 && kind != 1)) return 1;
+  double* g = (double*)malloc(sizeof(double) * (size_t)P);
+  int8_t* z = (int8_t*)malloc((size_t)P);
+  if (!g || !z) { free(g); free(z); return 2; }
+  double bc1 = 1.0 - pow(beta1, (double)t), bc2 = 1.0 - pow(beta2, (double)t);
+  for (int e = 0; e < N; ++e) {
+    for (int64_t p = 0; p < P; ++p) g[p] = 0.0;
+    for (int a = 0; a < A; ++a) {
+      for (int i = 0; i < n_pert; ++i) {
+        double ci = coef[((int64_t)a * N + e) * n_pert + i];
+        oracle_probe(seed, steps[a], (uint32_t)e, (uint32_t)i, kind, 0, P, z);
+        for (int64_t p = 0; p < P; ++p) g[p] += ci * (double)z[p];
+      }
+    }
+    const double* th = theta + (int64_t)e * P;
+    const double* me = m + (int64_t)e * P;
+    const double* ve = v + (int64_t)e * P;
+    double* to = theta_out + (int64_t)e * P;
+    double* mo = m_out + (int64_t)e * P;
+    double* vo = v_out + (int64_t)e * P;
+    for (int64_t p = 0; p < P; ++p) {
+      double gp = g[p] / ((double)A * (double)n_pert) + wd * th[p];
+      double mp = beta1 * me[p] + (1.0 - beta1) * gp;
+      double vp = beta2 * ve[p] + (1.0 - beta2) * gp * gp;
+      mo[p] = mp;
+      vo[p] = vp;
+      to[p] = th[p] - lr * (mp / bc1) / (sqrt(vp / bc2) + delta);
+    }
   }
   free(g);
   free(z);

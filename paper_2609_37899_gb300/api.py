@@ -39,6 +39,16 @@ class soma_dims(ctypes.Structure):
 TRACE_KINDS = ("gate", "head", "reduce", "update", "prep")
 
 
+class soma_adam_config(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("delta", ctypes.c_float), ("weight_decay", ctypes.c_float),
+                ("t", ctypes.c_int32)]
+
+
+PROBE_KINDS = {"dense": 0, "sparse": 1}
+MAX_ACCUM = 64
+
+
 class soma_kernel_times(ctypes.Structure):
     _fields_ = [("ms", ctypes.c_double * 5), ("launches", ctypes.c_int64 * 5)]
 
@@ -75,6 +85,12 @@ def lib():
         _sig(L, "soma_debug_philox", i32, [u64, vp, vp, i32, vp])
         _sig(L, "soma_debug_rademacher", i32, [u64, u64, i32, i32, i64, i64, vp, vp])
         _sig(L, "soma_debug_tc_gemm", i32, [vp, vp, vp, i32, i32, vp])
+        _sig(L, "soma_spsa_estimate", i32, [vp, i32, soma_dims, i32, i32, f32, u64, u64, vp, i32,
+                                            i32, vp, vp, vp, sz, vp])
+        _sig(L, "soma_adam_update", i32, [vp, vp, vp, i32, soma_dims, i32, i32, u64,
+                                          ctypes.POINTER(ctypes.c_uint64), i32, vp,
+                                          soma_adam_config, vp])
+        _sig(L, "soma_debug_probe", i32, [u64, u64, i32, i32, i32, i64, i64, vp, vp])
         _lib = L
         return L
 
@@ -145,6 +161,37 @@ def spsa_step(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int, n_
         "soma_spsa_step")
 
 
+def spsa_estimate(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int, n_pert: int,
+                  kind: str, eps: float, seed: int, step: int, losses: torch.Tensor,
+                  coef: torch.Tensor, workspace: torch.Tensor, stream=None):
+    """Losses [N, n_pert, 2] and coefficients [N, n_pert] of one accumulation
+    batch with dense or sparse probes; params are read only."""
+    N, B, T1 = byte_batch.shape
+    P = param_count(E, H)
+    _check(lib().soma_spsa_estimate(
+        _dev(params, torch.float32, "params", N * P), N, dims(E, H), n_pert, PROBE_KINDS[kind],
+        eps, seed, step, _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
+        _dev(losses, torch.float32, "losses", N * n_pert * 2),
+        _dev(coef, torch.float32, "coef", N * n_pert),
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_spsa_estimate")
+
+
+def adam_update(params: torch.Tensor, m: torch.Tensor, v: torch.Tensor, E: int, H: int,
+                kind: str, seed: int, steps, coef: torch.Tensor, lr: float, beta1: float,
+                beta2: float, delta: float, weight_decay: float, t: int, stream=None):
+    """The Adam step of Eq. localspsa; coef [A, N, n_pert], steps: A host ints."""
+    A, N, n_pert = coef.shape
+    P = param_count(E, H)
+    st = (ctypes.c_uint64 * A)(*[int(x) for x in steps])
+    cfg = soma_adam_config(lr, beta1, beta2, delta, weight_decay, t)
+    _check(lib().soma_adam_update(
+        _dev(params, torch.float32, "params", N * P), _dev(m, torch.float32, "m", N * P),
+        _dev(v, torch.float32, "v", N * P), N, dims(E, H), n_pert, PROBE_KINDS[kind], seed, st,
+        A, _dev(coef, torch.float32, "coef", A * N * n_pert), cfg, _stream(stream)),
+        "soma_adam_update")
+
+
 def eval_loss(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int,
               loss_out: torch.Tensor, workspace: torch.Tensor, stream=None):
     N, B, T1 = byte_batch.shape
@@ -199,6 +246,15 @@ def debug_rademacher(seed: int, step: int, expert: int, probe: int, p0: int, cou
     return z
 
 
+def debug_probe(seed: int, step: int, expert: int, probe: int, kind: str, p0: int, count: int,
+                device="cuda", stream=None) -> torch.Tensor:
+    z = torch.empty(count, dtype=torch.int8, device=device)
+    _check(lib().soma_debug_probe(seed, step, expert, probe, PROBE_KINDS[kind], p0, count,
+                                  _dev(z, torch.int8, "z"), _stream(stream)),
+           "soma_debug_probe")
+    return z
+
+
 def debug_tc_gemm(a: torch.Tensor, b: torch.Tensor, stream=None) -> torch.Tensor:
     """a [128, K] fp16, b [N, K] fp16 (CUDA) -> a @ b.T [128, N] fp32 on the tensor cores."""
     n, k = b.shape
@@ -237,3 +293,27 @@ class SomaExperts:
     def eval(self, byte_batch: torch.Tensor, stream=None):
         eval_loss(self.params, byte_batch, self.E, self.H, self.loss, self.workspace, stream)
         return self.loss
+
+    def adam_step(self, byte_batches, eps: float, seed: int, steps, t: int, lr: float,
+                  beta1: float = 0.9, beta2: float = 0.999, delta: float = 1e-8,
+                  weight_decay: float = 1e-4, kind: str = "sparse", stream=None):
+        """The paper's optimizer step: one estimate per accumulation batch
+        (byte_batches[a] with probe step counter steps[a]), then the Adam
+        update with bias correction for update t.  Moments live on this
+        object (zeros before the first update)."""
+        A = len(byte_batches)
+        if getattr(self, "m", None) is None:
+            self.m = torch.zeros_like(self.params)
+            self.v = torch.zeros_like(self.params)
+        if getattr(self, "coef_acc", None) is None or self.coef_acc.shape[0] != A:
+            self.coef_acc = torch.zeros(A, self.N, self.n_pert, dtype=torch.float32,
+                                        device=self.params.device)
+            self.losses_acc = torch.zeros(A, self.N, self.n_pert, 2, dtype=torch.float32,
+                                          device=self.params.device)
+        for a in range(A):
+            spsa_estimate(self.params, byte_batches[a], self.E, self.H, self.n_pert, kind, eps,
+                          seed, steps[a], self.losses_acc[a], self.coef_acc[a], self.workspace,
+                          stream)
+        adam_update(self.params, self.m, self.v, self.E, self.H, kind, seed, steps, self.coef_acc,
+                    lr, beta1, beta2, delta, weight_decay, t, stream)
+        return self.losses_acc, self.coef_acc

@@ -81,24 +81,27 @@ __global__ void __launch_bounds__(128) gate_step_kernel(const GateStep g) {
     {  // perturbed weights: row wrow, reduction indices k0 .. k0 + kc - 1
       const int64_t p = xpart ? L.w_ih + (int64_t)wrow * E + k0
                               : L.w_hh + (int64_t)wrow * H + (k0 - E);
-      const uint32_t bits = (pert && wrow_ok) ? probe_bits32(pk, p) : 0u;
+      ProbeBits bits = {0u, 0u};
+      if (pert && wrow_ok) bits = probe_bits(pk, p, s.sparse);
 #pragma unroll
       for (int k = 0; k < kKc; ++k) {
         float w = 0.f;
-        if (wrow_ok && k < kc) w = perturb(th[p + k], (bits >> k) & 1u, se);
+        if (wrow_ok && k < kc) w = perturb(th[p + k], (bits.neg >> k) & 1u, (bits.act >> k) & 1u, se);
         Wt[k][lu][lg] = w;
       }
     }
     {  // inputs: perturbed embedding row of byte_t, or h_{t-1}
-      uint32_t xbits = 0u;
-      if (xpart && pert && col_ok) xbits = probe_bits32(pk, L.emb + (int64_t)xbyte * E + k0 + lk0);
+      ProbeBits xbits = {0u, 0u};
+      if (xpart && pert && col_ok)
+        xbits = probe_bits(pk, L.emb + (int64_t)xbyte * E + k0 + lk0, s.sparse);
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const int k = lk0 + kk;
         float v = 0.f;
         if (col_ok && k < kc) {
           if (xpart) {
-            v = perturb(th[L.emb + (int64_t)xbyte * E + k0 + k], (xbits >> kk) & 1u, se);
+            v = perturb(th[L.emb + (int64_t)xbyte * E + k0 + k], (xbits.neg >> kk) & 1u,
+                        (xbits.act >> kk) & 1u, se);
           } else if (hprev) {
             v = hprev[k0 - E + k];
           }
@@ -131,8 +134,9 @@ __global__ void __launch_bounds__(128) gate_step_kernel(const GateStep g) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int64_t p = L.b + (int64_t)q * H + u;
-    const uint32_t bit = pert ? (probe_bits32(pk, p) & 1u) : 0u;
-    bias[q] = perturb(th[p], bit, se);
+    ProbeBits bit = {0u, 0u};
+    if (pert) bit = probe_bits(pk, p, s.sparse);
+    bias[q] = perturb(th[p], bit.neg & 1u, bit.act & 1u, se);
   }
 #pragma unroll
   for (int j = 0; j < kColsPerThr; ++j) {
@@ -201,10 +205,12 @@ __global__ void __launch_bounds__(256) head_nll_kernel(const HeadChunk hc) {
     const int kc = min(kKc, H - k0);
     {
       const int64_t p = L.w_out + (int64_t)tid * H + k0;
-      const uint32_t bits = pert ? probe_bits32(pk, p) : 0u;
+      ProbeBits bits = {0u, 0u};
+      if (pert) bits = probe_bits(pk, p, s.sparse);
 #pragma unroll
       for (int k = 0; k < kKc; ++k)
-        sm.g.Wt[k][tid] = (k < kc) ? perturb(th[p + k], (bits >> k) & 1u, se) : 0.f;
+        sm.g.Wt[k][tid] =
+            (k < kc) ? perturb(th[p + k], (bits.neg >> k) & 1u, (bits.act >> k) & 1u, se) : 0.f;
     }
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
@@ -227,8 +233,9 @@ __global__ void __launch_bounds__(256) head_nll_kernel(const HeadChunk hc) {
   }
   {
     const int64_t p = L.b_out + tid;
-    const uint32_t bit = pert ? (probe_bits32(pk, p) & 1u) : 0u;
-    const float bo = perturb(th[p], bit, se);
+    ProbeBits bit = {0u, 0u};
+    if (pert) bit = probe_bits(pk, p, s.sparse);
+    const float bo = perturb(th[p], bit.neg & 1u, bit.act & 1u, se);
 #pragma unroll
     for (int j = 0; j < kHeadCols; ++j) sm.Lg[tid][j] = acc[j] + bo;
   }

@@ -110,15 +110,30 @@ __device__ __forceinline__ uint32_t z_run_raw(const ProbeKey& pk, int64_t p0, ZS
   return natural_to_raw(probe_bits32(pk, p0));
 }
 
+// fp16 pair word J of a run: +-1 for dense probes; for sparse probes the
+// magnitude is kept only where the activity bit (same position in `act`) is
+// set, so inactive coordinates are +-0.
+template <bool SPARSE, int J>
+__device__ __forceinline__ uint32_t z_pair(uint32_t raw, uint32_t act) {
+  if (!SPARSE) return pm_pair<J>(raw, 0x3C003C00u);
+  const uint32_t a = (act << (15 - J)) & 0x80008000u;  // activity at the sign positions
+  return ((raw << (15 - J)) & 0x80008000u) | (0x3C003C00u & (a - (a >> 15)));
+}
+
 // Writes 32 elements of a Z tile row in the canonical K-major layout from one
-// raw word; `row` points at the first element, consecutive 8-element chunks
-// are 128 bytes apart.
-__device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw) {
+// raw sign word (and, for sparse probes, its activity word); `row` points at
+// the first element, consecutive 8-element chunks are 128 bytes apart.
+template <bool SPARSE>
+__device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw, uint32_t act) {
   uint4 c0, c1, c2, c3;
-  c0.x = pm_pair<0>(raw, 0x3C003C00u);  c0.y = pm_pair<1>(raw, 0x3C003C00u);  c0.z = pm_pair<2>(raw, 0x3C003C00u);  c0.w = pm_pair<3>(raw, 0x3C003C00u);
-  c1.x = pm_pair<4>(raw, 0x3C003C00u);  c1.y = pm_pair<5>(raw, 0x3C003C00u);  c1.z = pm_pair<6>(raw, 0x3C003C00u);  c1.w = pm_pair<7>(raw, 0x3C003C00u);
-  c2.x = pm_pair<8>(raw, 0x3C003C00u);  c2.y = pm_pair<9>(raw, 0x3C003C00u);  c2.z = pm_pair<10>(raw, 0x3C003C00u); c2.w = pm_pair<11>(raw, 0x3C003C00u);
-  c3.x = pm_pair<12>(raw, 0x3C003C00u); c3.y = pm_pair<13>(raw, 0x3C003C00u); c3.z = pm_pair<14>(raw, 0x3C003C00u); c3.w = pm_pair<15>(raw, 0x3C003C00u);
+  c0.x = z_pair<SPARSE, 0>(raw, act);   c0.y = z_pair<SPARSE, 1>(raw, act);
+  c0.z = z_pair<SPARSE, 2>(raw, act);   c0.w = z_pair<SPARSE, 3>(raw, act);
+  c1.x = z_pair<SPARSE, 4>(raw, act);   c1.y = z_pair<SPARSE, 5>(raw, act);
+  c1.z = z_pair<SPARSE, 6>(raw, act);   c1.w = z_pair<SPARSE, 7>(raw, act);
+  c2.x = z_pair<SPARSE, 8>(raw, act);   c2.y = z_pair<SPARSE, 9>(raw, act);
+  c2.z = z_pair<SPARSE, 10>(raw, act);  c2.w = z_pair<SPARSE, 11>(raw, act);
+  c3.x = z_pair<SPARSE, 12>(raw, act);  c3.y = z_pair<SPARSE, 13>(raw, act);
+  c3.z = z_pair<SPARSE, 14>(raw, act);  c3.w = z_pair<SPARSE, 15>(raw, act);
   *reinterpret_cast<uint4*>(row) = c0;
   *reinterpret_cast<uint4*>(row + 128) = c1;
   *reinterpret_cast<uint4*>(row + 256) = c2;
@@ -286,7 +301,10 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
     if (Ur < H) {
       const int64_t pb = L.b + (int64_t)tile_gate(32 * q4 + lane) * H + Ur;
       bias_r = th[pb];
-      if (do_z) dbias_r = (probe_bits32(pk, pb) & 1u) ? -eps : eps;
+      if (do_z) {
+        const ProbeBits zb = probe_bits(pk, pb, s.sparse);
+        dbias_r = eps_z(zb.neg & 1u, zb.act & 1u, eps);
+      }
     }
   }
   const int u8 = lane >> 2, bq = lane & 3;
@@ -399,7 +417,8 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     float dbo[4] = {0.f, 0.f, 0.f, 0.f};
     if (do_z) {
       const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)i);
-      const float dbo_r = (probe_bits32(pk, L.b_out + vq + lane) & 1u) ? -eps : eps;
+      const ProbeBits zb = probe_bits(pk, L.b_out + vq + lane, s.sparse);
+      const float dbo_r = eps_z(zb.neg & 1u, zb.act & 1u, eps);
 #pragma unroll
       for (int k = 0; k < 4; ++k) dbo[k] = __shfl_sync(0xffffffffu, dbo_r, r4 + 8 * k);
     }
@@ -495,7 +514,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk);
 
 // grid: min(tasks, SMs) persistent CTAs (+ for the head, the embedding-part
 // blocks of the next timestep's operand), kThreads threads.
-template <bool HEAD>
+template <bool HEAD, bool SPARSE>
 __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_tasks,
                                                                     int n_ctas) {
   extern __shared__ uint8_t dyn_smem[];
@@ -637,16 +656,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         const bool active = pz < T.p_valid;
         const ProbeKey pk =
             make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pz));
-        ZSlot cache;
+        const ProbeKey pka = activity_key(pk);
+        ZSlot cache, cache_a;
         cache.blk = 0xFFFFFFFFu;
+        cache_a.blk = 0xFFFFFFFFu;
         const int split = HEAD ? nst : g.Sx;
         const int64_t seg0 = z_param<HEAD>(a, T, r, 0);
         const int64_t seg1 = z_param<HEAD>(a, T, r, split) - (int64_t)kKt * split;
         uint8_t* zrow = smem + SL.z_off + pz * kTileA + kmajor_offset(r, 0, kKt);
-        uint32_t raw[kKt / 32] = {};
+        uint32_t raw[kKt / 32] = {}, act[kKt / 32] = {};
         if (active) {
 #pragma unroll
-          for (int w = 0; w < kKt / 32; ++w) raw[w] = z_run_raw(pk, seg0 + 32 * w, cache);
+          for (int w = 0; w < kKt / 32; ++w) {
+            raw[w] = z_run_raw(pk, seg0 + 32 * w, cache);
+            if (SPARSE) act[w] = z_run_raw(pka, seg0 + 32 * w, cache_a);
+          }
         }
         for (int st = 0; st < nst; ++st, ++gs) {
           const int q = gs % kStages;
@@ -658,7 +682,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           if (active) {
             uint8_t* zr = zrow + q * SL.bytes;
 #pragma unroll
-            for (int w = 0; w < kKt / 32; ++w) store_z_row_at(zr + w * 4 * 128, raw[w]);
+            for (int w = 0; w < kKt / 32; ++w)
+              store_z_row_at<SPARSE>(zr + w * 4 * 128, raw[w], act[w]);
           }
           fence_async_smem();
           __syncwarp();
@@ -666,7 +691,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           if (active && st + 1 < nst) {
             const int64_t p1 = (st + 1 < split ? seg0 : seg1) + (int64_t)kKt * (st + 1);
 #pragma unroll
-            for (int w = 0; w < kKt / 32; ++w) raw[w] = z_run_raw(pk, p1 + 32 * w, cache);
+            for (int w = 0; w < kKt / 32; ++w) {
+              raw[w] = z_run_raw(pk, p1 + 32 * w, cache);
+              if (SPARSE) act[w] = z_run_raw(pka, p1 + 32 * w, cache_a);
+            }
           }
         }
       }
@@ -723,13 +751,14 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
     if (i < s.n_pert && b < s.B) {
       const int y = s.bytes[((int64_t)e * s.B + b) * (s.T + 1) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
-      uint32_t bits = 0;
+      ProbeBits bits = {0u, 0u};
       if (delta && s.eps != 0.f)
-        bits = probe_bits32(make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i), p0);
+        bits = probe_bits(make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i), p0, s.sparse);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         float x = 0.f;
-        if (k0 + j < g.E) x = delta ? (((bits >> j) & 1u) ? -s.eps : s.eps) : th[p0 + j];
+        if (k0 + j < g.E)
+          x = delta ? eps_z((bits.neg >> j) & 1u, (bits.act >> j) & 1u, s.eps) : th[p0 + j];
         v[j] = __float2half_rn(x);
       }
     } else {
@@ -964,11 +993,12 @@ TcSizes tc_sizes(const TcGeom& g) {
 cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
                               cudaStream_t stream) {
   const size_t smem = kernel_smem_bytes(g);
-  cudaError_t e = cudaFuncSetAttribute(tc_persistent_kernel<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto gate_kernel = s.sparse ? tc_persistent_kernel<false, true> : tc_persistent_kernel<false, false>;
+  auto head_kernel = s.sparse ? tc_persistent_kernel<true, true> : tc_persistent_kernel<true, false>;
+  cudaError_t e = cudaFuncSetAttribute(gate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(tc_persistent_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
+  e = cudaFuncSetAttribute(head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const TcSizes z = tc_sizes(g);
   TcArgs a;
@@ -1003,14 +1033,14 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
     a.op_in = tb.op[t & 1];
     a.op_out = tb.op[(t + 1) & 1];
     trace_begin(SOMA_TRACE_GATE, stream);
-    tc_persistent_kernel<false><<<gate_ctas, kThreads, smem, stream>>>(a, gate_tasks, gate_ctas);
+    gate_kernel<<<gate_ctas, kThreads, smem, stream>>>(a, gate_tasks, gate_ctas);
     trace_end(SOMA_TRACE_GATE, stream);
     // head of timestep t (h part of the operand of t + 1) and, in the same
     // launch, the embedding part of that operand
     a.op_in = tb.op[(t + 1) & 1];
     trace_begin(SOMA_TRACE_HEAD, stream);
-    tc_persistent_kernel<true><<<head_ctas + (t + 1 < s.T ? xblocks : 0), kThreads, smem,
-                                 stream>>>(a, head_tasks, head_ctas);
+    head_kernel<<<head_ctas + (t + 1 < s.T ? xblocks : 0), kThreads, smem, stream>>>(
+        a, head_tasks, head_ctas);
     trace_end(SOMA_TRACE_HEAD, stream);
   }
   return cudaGetLastError();

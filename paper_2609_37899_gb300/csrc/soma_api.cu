@@ -156,10 +156,11 @@ int soma_init_experts(float* params, int n_experts, soma_dims d, uint64_t seed, 
   return cuda_status(launch_init(params, lay, n_experts, seed, std, (cudaStream_t)stream));
 }
 
-int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float eps, float lr,
-                   uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
-                   int seq_len, float* losses_out, float* coef_out, void* workspace,
-                   size_t workspace_bytes, void* stream) {
+// Forward sweep, reduction and (optionally) the SGD update of one step.
+static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, int sparse,
+                        float eps, float lr, bool update, uint64_t seed, uint64_t step,
+                        const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
+                        float* coef_out, void* workspace, size_t workspace_bytes, void* stream) {
   if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
   if (!params || !byte_batch || !losses_out || !aligned16(params) ||
       !sizes_ok(n_experts, n_pert, batch, seq_len) || !(eps >= 0.f) || !std::isfinite(eps) ||
@@ -181,6 +182,7 @@ int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float 
   s.B = batch;
   s.T = seq_len;
   s.eps = eps;
+  s.sparse = sparse;
   s.seed = seed;
   s.step = step;
   float* coef_ws = coef_scratch(w, workspace);
@@ -200,9 +202,59 @@ int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float 
   }
   // eps == 0 makes every coefficient 0 and lr == 0 every step 0: theta stays
   // bit-identical, so the update is not launched at all.
-  if (e == cudaSuccess && eps != 0.f && lr != 0.f)
+  if (update && e == cudaSuccess && eps != 0.f && lr != 0.f)
     e = launch_spsa_update(params, s.lay, n_experts, n_pert, lr, seed, step, coef_ws, st);
   return cuda_status(e);
+}
+
+int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float eps, float lr,
+                   uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
+                   int seq_len, float* losses_out, float* coef_out, void* workspace,
+                   size_t workspace_bytes, void* stream) {
+  return spsa_forward(params, n_experts, d, n_pert, 0, eps, lr, true, seed, step, byte_batch,
+                      batch, seq_len, losses_out, coef_out, workspace, workspace_bytes, stream);
+}
+
+int soma_spsa_estimate(const float* params, int n_experts, soma_dims d, int n_pert,
+                       int probe_kind, float eps, uint64_t seed, uint64_t step,
+                       const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
+                       float* coef_out, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!coef_out || (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE))
+    return SOMA_ERR_INVALID_ARG;
+  // the forward sweep only reads params
+  return spsa_forward(const_cast<float*>(params), n_experts, d, n_pert, probe_kind, eps, 0.f,
+                      false, seed, step, byte_batch, batch, seq_len, losses_out, coef_out,
+                      workspace, workspace_bytes, stream);
+}
+
+int soma_adam_update(float* params, float* m, float* v, int n_experts, soma_dims d, int n_pert,
+                     int probe_kind, uint64_t seed, const uint64_t* steps, int n_acc,
+                     const float* coef, soma_adam_config cfg, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !m || !v || !coef || !steps || !aligned16(params) || !aligned16(m) ||
+      !aligned16(v) || n_experts < 1 || n_pert < 1 || n_pert > kMaxPert || n_acc < 1 ||
+      n_acc > SOMA_MAX_ACCUM || (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE))
+    return SOMA_ERR_INVALID_ARG;
+  if (!std::isfinite(cfg.lr) || !(cfg.beta1 >= 0.f && cfg.beta1 < 1.f) ||
+      !(cfg.beta2 >= 0.f && cfg.beta2 < 1.f) || !(cfg.delta > 0.f) || !std::isfinite(cfg.delta) ||
+      !(cfg.weight_decay >= 0.f) || !std::isfinite(cfg.weight_decay) || cfg.t < 1)
+    return SOMA_ERR_INVALID_ARG;
+  AdamSteps st;
+  st.n_acc = n_acc;
+  for (int a = 0; a < n_acc; ++a) st.step[a] = steps[a];
+  AdamArgs h;
+  h.lr = cfg.lr;
+  h.b1 = cfg.beta1;
+  h.b2 = cfg.beta2;
+  h.delta = cfg.delta;
+  h.wd = cfg.weight_decay;
+  // bias corrections in double, then rounded once
+  h.inv_bc1 = (float)(1.0 / (1.0 - std::pow((double)cfg.beta1, (double)cfg.t)));
+  h.inv_bc2 = (float)(1.0 / (1.0 - std::pow((double)cfg.beta2, (double)cfg.t)));
+  const Layout lay = make_layout(d.embed, d.hidden);
+  return cuda_status(launch_adam_update(params, m, v, lay, n_experts, n_pert, probe_kind, seed, st,
+                                        coef, h, (cudaStream_t)stream));
 }
 
 int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_t* byte_batch,
@@ -227,6 +279,7 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
   s.B = batch;
   s.T = seq_len;
   s.eps = 0.f;
+  s.sparse = 0;
   s.seed = 0;
   s.step = 0;
   cudaError_t e;
@@ -305,7 +358,17 @@ int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, in
   if (!z_out || count < 0 || p0 < 0 || expert < 0 || pert < 0) return SOMA_ERR_INVALID_ARG;
   if (count == 0) return SOMA_OK;
   return cuda_status(
-      launch_debug_rademacher(seed, step, expert, pert, p0, count, z_out, (cudaStream_t)stream));
+      launch_debug_rademacher(seed, step, expert, pert, 0, p0, count, z_out, (cudaStream_t)stream));
+}
+
+int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int probe_kind,
+                     int64_t p0, int64_t count, int8_t* z_out, void* stream) {
+  if (!z_out || count < 0 || p0 < 0 || expert < 0 || pert < 0 ||
+      (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE))
+    return SOMA_ERR_INVALID_ARG;
+  if (count == 0) return SOMA_OK;
+  return cuda_status(launch_debug_rademacher(seed, step, expert, pert, probe_kind, p0, count, z_out,
+                                             (cudaStream_t)stream));
 }
 
 }  // extern "C"

@@ -103,9 +103,42 @@ __host__ __device__ __forceinline__ uint32_t probe_bits32(const ProbeKey& k, int
 // Raw bit position of offset o (0..31) inside a run.
 __host__ __device__ constexpr int raw_bit(int o) { return (o >> 1) + 16 * (o & 1); }
 
+// Sparse probes (App. E: a coordinate is 0 with probability 1/2, else -1 or
+// +1) take a second bit per coordinate: the activity bit, read with the same
+// map from the blocks whose counter word 1 is the probe index with its top
+// bit set.  z = active ? 1 - 2 * sign bit : 0, so a nonzero sparse
+// coordinate equals the dense probe's coordinate.
+__host__ __device__ __forceinline__ ProbeKey activity_key(ProbeKey k) {
+  k.probe |= 0x80000000u;
+  return k;
+}
+
+// Sign and activity bits of the 32 parameters p .. p+31 (natural order).
+struct ProbeBits {
+  uint32_t neg, act;
+};
+
+__host__ __device__ __forceinline__ ProbeBits probe_bits(const ProbeKey& k, int64_t p,
+                                                         bool sparse) {
+  ProbeBits b;
+  b.neg = probe_bits32(k, p);
+  b.act = sparse ? probe_bits32(activity_key(k), p) : 0xFFFFFFFFu;
+  return b;
+}
+
 // w + s*eps*z for a z bit: the perturbed parameter in fp32.
 __host__ __device__ __forceinline__ float perturb(float w, uint32_t bit, float se) {
   return w + (bit ? -se : se);
+}
+
+// The same for a probe coordinate with sign bit `neg` and activity bit `act`.
+__host__ __device__ __forceinline__ float perturb(float w, uint32_t neg, uint32_t act, float se) {
+  return act ? w + (neg ? -se : se) : w;
+}
+
+// eps z of one coordinate.
+__host__ __device__ __forceinline__ float eps_z(uint32_t neg, uint32_t act, float eps) {
+  return act ? (neg ? -eps : eps) : 0.f;
 }
 
 // ---------------------------------------------------------------------------
@@ -144,6 +177,7 @@ struct Sweep {
   int n_experts, n_pert, n_sign;
   int B, T;
   float eps;
+  int sparse;              // probe kind: 0 dense Rademacher, 1 sparse (App. E)
   uint64_t seed, step;
   __host__ __device__ int lanes() const { return n_experts * n_pert * n_sign; }
 };

@@ -6,6 +6,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "soma_api.h"
 #include "soma_device.cuh"
 
 namespace soma {
@@ -72,7 +73,23 @@ cudaError_t launch_init(float* params, const Layout& lay, int n_experts, uint64_
                         cudaStream_t stream);
 cudaError_t launch_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
                                 cudaStream_t stream);
-cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
-                                    int64_t count, int8_t* z, cudaStream_t stream);
+cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int sparse,
+                                    int64_t p0, int64_t count, int8_t* z, cudaStream_t stream);
+
+// Probe step counters of the accumulation batches of one Adam update.
+struct AdamSteps {
+  int n_acc;
+  uint64_t step[SOMA_MAX_ACCUM];
+};
+
+// Adam hyper-parameters with the bias corrections of update t folded in:
+// inv_bc1 = 1 / (1 - b1^t), inv_bc2 = 1 / (1 - b2^t).
+struct AdamArgs {
+  float lr, b1, b2, delta, wd, inv_bc1, inv_bc2;
+};
+
+cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
+                               int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
+                               const float* coef, const AdamArgs& h, cudaStream_t stream);
 
 }  // namespace soma

@@ -111,6 +111,63 @@ spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr,
   }
 }
 
+// The paper's optimizer step (App. E, Eq. localspsa) for expert e:
+//   g = (1/(A n)) sum_a sum_i coef[a][e][i] z_{e,i}^{(a)} + wd * theta,
+//   m = b1 m + (1 - b1) g,  v = b2 v + (1 - b2) g^2,
+//   theta -= lr * (m / bc1) / (sqrt(v / bc2) + delta),
+// with z^{(a)} drawn with step counter steps[a] (dense or sparse).  As in the
+// SGD kernel, thread q owns the 32 parameters 32q .. 32q + 31 and reads one
+// raw Philox word per probe (two for sparse probes).  An expert whose
+// coefficients are not all finite is left unchanged, moments included.
+__global__ void __launch_bounds__(kUpdThreads)
+adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __restrict__ v,
+                   Layout lay, int n_experts, int n_pert, int sparse, uint64_t seed,
+                   AdamSteps steps, const float* __restrict__ coef, AdamArgs h) {
+  __shared__ int all_finite;
+  const int e = blockIdx.y;
+  if (threadIdx.x == 0) all_finite = 1;
+  __syncthreads();
+  for (int j = threadIdx.x; j < steps.n_acc * n_pert; j += kUpdThreads) {
+    const int a = j / n_pert, i = j % n_pert;
+    if (!isfinite(coef[((int64_t)a * n_experts + e) * n_pert + i])) all_finite = 0;
+  }
+  __syncthreads();
+  if (!all_finite) return;
+  const int64_t q = (int64_t)blockIdx.x * kUpdThreads + threadIdx.x;
+  const int64_t p0 = q * 32;
+  if (p0 >= lay.P) return;
+  float acc[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+  for (int a = 0; a < steps.n_acc; ++a) {
+    const float* ca = coef + ((int64_t)a * n_experts + e) * n_pert;
+    for (int i = 0; i < n_pert; ++i) {
+      const ProbeKey pk = make_probe_key(seed, steps.step[a], (uint32_t)e, (uint32_t)i);
+      const uint32_t w = (uint32_t)(p0 >> 5);  // p0 is 32-aligned
+      const uint32_t raw = probe_raw_word(pk, w);
+      const uint32_t act = sparse ? probe_raw_word(activity_key(pk), w) : 0xFFFFFFFFu;
+      const float c = ca[i];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const uint32_t rb = (uint32_t)raw_bit(j);
+        if ((act >> rb) & 1u) acc[j] += ((raw >> rb) & 1u) ? -c : c;
+      }
+    }
+  }
+  const float inv = 1.f / ((float)steps.n_acc * (float)n_pert);
+  const int64_t base = (int64_t)e * lay.P + p0;
+  const int cnt = lay.P - p0 < 32 ? (int)(lay.P - p0) : 32;
+  for (int j = 0; j < cnt; ++j) {
+    const float th = params[base + j];
+    const float g = fmaf(h.wd, th, acc[j] * inv);
+    const float mj = fmaf(h.b1, m[base + j], (1.f - h.b1) * g);
+    const float vj = fmaf(h.b2, v[base + j], (1.f - h.b2) * g * g);
+    m[base + j] = mj;
+    v[base + j] = vj;
+    params[base + j] = th - h.lr * (mj * h.inv_bc1) / (sqrtf(vj * h.inv_bc2) + h.delta);
+  }
+}
+
 // Box-Muller normals from Philox4x32-10 in the init domain (counter word 3
 // = 0x80000001): parameters 2q and 2q+1 of expert e use counter (q, e, 0, .).
 __global__ void init_kernel(float* __restrict__ params, Layout lay, uint64_t seed, float std) {
@@ -157,13 +214,15 @@ __global__ void debug_philox_kernel(uint64_t seed, const uint32_t* ctr4, uint32_
   out4[4 * j + 3] = o.w;
 }
 
-// z[q] for p = p0 + q, through probe_bits32 at an arbitrary (unaligned) start
+// z[q] for p = p0 + q, through probe_bits at an arbitrary (unaligned) start
 // so that the two-block path of the helper is exercised as well.
-__global__ void debug_rademacher_kernel(ProbeKey pk, int64_t p0, int64_t count, int8_t* z) {
+__global__ void debug_rademacher_kernel(ProbeKey pk, int sparse, int64_t p0, int64_t count,
+                                        int8_t* z) {
   const int64_t q0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 32;
   if (q0 >= count) return;
-  const uint32_t bits = probe_bits32(pk, p0 + q0);
-  for (int j = 0; j < 32 && q0 + j < count; ++j) z[q0 + j] = ((bits >> j) & 1u) ? -1 : 1;
+  const ProbeBits bits = probe_bits(pk, p0 + q0, sparse != 0);
+  for (int j = 0; j < 32 && q0 + j < count; ++j)
+    z[q0 + j] = ((bits.act >> j) & 1u) ? (((bits.neg >> j) & 1u) ? -1 : 1) : 0;
 }
 
 }  // namespace
@@ -204,11 +263,24 @@ cudaError_t launch_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* o
   return cudaGetLastError();
 }
 
-cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
-                                    int64_t count, int8_t* z, cudaStream_t stream) {
+cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int sparse,
+                                    int64_t p0, int64_t count, int8_t* z, cudaStream_t stream) {
   const ProbeKey pk = make_probe_key(seed, step, (uint32_t)expert, (uint32_t)pert);
   const int64_t words = (count + 31) / 32;
-  debug_rademacher_kernel<<<(unsigned)((words + 127) / 128), 128, 0, stream>>>(pk, p0, count, z);
+  debug_rademacher_kernel<<<(unsigned)((words + 127) / 128), 128, 0, stream>>>(pk, sparse, p0,
+                                                                                count, z);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
+                               int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
+                               const float* coef, const AdamArgs& h, cudaStream_t stream) {
+  const int64_t words = (lay.P + 31) / 32;
+  dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
+  trace_begin(SOMA_TRACE_UPDATE, stream);
+  adam_update_kernel<<<grid, kUpdThreads, 0, stream>>>(params, m, v, lay, n_experts, n_pert, sparse,
+                                                       seed, steps, coef, h);
+  trace_end(SOMA_TRACE_UPDATE, stream);
   return cudaGetLastError();
 }
 

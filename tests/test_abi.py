@@ -29,7 +29,8 @@ def test_header_declares_the_entry_points():
     for required in ["soma_init_experts", "soma_spsa_step", "soma_eval_loss",
                      "soma_workspace_bytes", "soma_param_count", "soma_get_status",
                      "soma_status_string", "soma_spsa_update", "soma_debug_philox",
-                     "soma_debug_rademacher"]:
+                     "soma_debug_rademacher", "soma_spsa_estimate", "soma_adam_update",
+                     "soma_debug_probe"]:
         assert required in names
 
 
@@ -96,3 +97,23 @@ def test_host_validation_rejects_before_launch(soma):
     assert L.soma_init_experts(fake, 1, d, 0, -1.0, None) == 1
     assert L.soma_spsa_update(fake, 1, d, 8, float("nan"), 0, 0, fake, None) == 1
     assert L.soma_debug_rademacher(0, 0, 0, 0, -1, 4, fake, None) == 1
+    # the optimizer step's entry points
+    est = (fake, 1, d, 8)
+    assert L.soma_spsa_estimate(*est, 2, 1e-3, 0, 0, fake, 4, 64, fake, fake, fake, ws,
+                                None) == 1  # unknown probe kind
+    assert L.soma_spsa_estimate(*est, 1, 1e-3, 0, 0, fake, 4, 64, fake, None, fake, ws,
+                                None) == 1  # coef_out is required
+    cfg = soma.soma_adam_config(1e-3, 0.9, 0.999, 1e-8, 1e-4, 1)
+    steps = (ctypes.c_uint64 * 2)(0, 1)
+    assert L.soma_adam_update(fake, fake, fake, 1, d, 8, 1, 0, steps, 0, fake, cfg,
+                              None) == 1  # n_acc = 0
+    assert L.soma_adam_update(fake, fake, fake, 1, d, 8, 1, 0, steps, 65, fake, cfg,
+                              None) == 1  # n_acc > SOMA_MAX_ACCUM
+    assert L.soma_adam_update(fake, fake, fake, 1, d, 8, 1, 0, None, 2, fake, cfg, None) == 1
+    for bad in (soma.soma_adam_config(1e-3, 1.0, 0.999, 1e-8, 0.0, 1),
+                soma.soma_adam_config(1e-3, 0.9, 0.999, 0.0, 0.0, 1),
+                soma.soma_adam_config(1e-3, 0.9, 0.999, 1e-8, -1.0, 1),
+                soma.soma_adam_config(1e-3, 0.9, 0.999, 1e-8, 0.0, 0)):
+        assert L.soma_adam_update(fake, fake, fake, 1, d, 8, 1, 0, steps, 2, fake, bad,
+                                  None) == 1
+    assert L.soma_debug_probe(0, 0, 0, 0, 3, 0, 4, fake, None) == 1
