@@ -160,6 +160,30 @@ int soma_spsa_estimate(const float* params, int n_experts, soma_dims d, int n_pe
                        const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
                        float* coef_out, void* workspace, size_t workspace_bytes, void* stream);
 
+/* Options of soma_spsa_estimate_opts: the probe kind and the two variants
+ * the paper measures its mechanism with (App. D).
+ *   batch_per_probe = 0  byte_batch [n_experts][batch][seq_len + 1], one batch
+ *                        per expert shared by every probe (Sec. 4);
+ *                   = 1  byte_batch [n_experts][n_pert][batch][seq_len + 1],
+ *                        an independently drawn batch per probe (both signs
+ *                        of a probe share it).
+ *   summed_loss     = 0  each expert's own loss (SOMA);
+ *                   = 1  the control arm that sums the N experts' losses
+ *                        before each finite difference: coef_out[e][i] =
+ *                        sum_e' (L+_{e',i} - L-_{e',i}) / (2 eps) for every e
+ *                        (losses_out still holds each expert's L+, L-). */
+typedef struct soma_estimate_options {
+  int32_t probe_kind;
+  int32_t batch_per_probe;
+  int32_t summed_loss;
+} soma_estimate_options;
+
+int soma_spsa_estimate_opts(const float* params, int n_experts, soma_dims d, int n_pert,
+                            const soma_estimate_options* opts, float eps, uint64_t seed,
+                            uint64_t step, const uint8_t* byte_batch, int batch, int seq_len,
+                            float* losses_out, float* coef_out, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
 /* The Adam update of Eq. localspsa from the coefficients of n_acc
  * accumulation batches.
  *   params, m, v  device fp32 [n_experts][P]; updated in place (m, v start at

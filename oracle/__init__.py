@@ -90,6 +90,14 @@ def _load():
                                                 ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
                                                 c_dp, c_dp, ctypes.c_int]
         lib.oracle_spsa_losses_kind.restype = ctypes.c_int
+        lib.oracle_spsa_losses_opts.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_double, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_uint64, ctypes.c_uint64,
+                                                c_u8p, ctypes.c_int, ctypes.c_int,
+                                                ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
+                                                c_dp, c_dp, ctypes.c_int]
+        lib.oracle_spsa_losses_opts.restype = ctypes.c_int
         lib.oracle_probe.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32,
                                      ctypes.c_uint32, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
                                      ctypes.POINTER(ctypes.c_int8)]
@@ -180,7 +188,8 @@ def loss(theta, E: int, H: int, bytes_, n_threads: int = 0, per_token: bool = Fa
 
 def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
                 probes=None, n_pert: int | None = None, n_threads: int = 0,
-                first_expert: int = 0, kind: str = "dense"):
+                first_expert: int = 0, kind: str = "dense", batch_per_probe: bool = False,
+                summed_loss: bool = False):
     """Antithetic losses and coefficients for the selected probes.
 
     theta [N, P] (fp32 or fp64), bytes_ [N, B, T+1] uint8.  ``probes`` lists
@@ -192,14 +201,16 @@ def spsa_losses(theta, E: int, H: int, eps: float, seed: int, step: int, bytes_,
     N = th.shape[0]
     bx = _u8(bytes_)
     assert bx.shape[0] == N
-    B, T = bx.shape[1], bx.shape[2] - 1
+    B, T = bx.shape[-2], bx.shape[-1] - 1
+    n_total = bx.shape[1] if batch_per_probe else 0  # bytes [N, n_pert, B, T+1]
     if probes is None:
         probes = range(n_pert)
     sel = np.ascontiguousarray(list(probes), dtype=np.int32)
     L = np.zeros((N, sel.size, 2), dtype=np.float64)
     coef = np.zeros((N, sel.size), dtype=np.float64)
-    rc = _load().oracle_spsa_losses_kind(_ptr(th, ctypes.c_double), N, first_expert, E, H,
-                                    float(eps), PROBE_KINDS[kind], seed, step,
+    rc = _load().oracle_spsa_losses_opts(_ptr(th, ctypes.c_double), N, first_expert, E, H,
+                                    float(eps), PROBE_KINDS[kind], int(batch_per_probe),
+                                    int(summed_loss), n_total, seed, step,
                                     _ptr(bx, ctypes.c_uint8), B, T,
                                     _ptr(sel, ctypes.c_int32), sel.size,
                                     _ptr(L, ctypes.c_double), _ptr(coef, ctypes.c_double),

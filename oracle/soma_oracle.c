@@ -251,25 +251,33 @@ double oracle_loss(const double* theta, int E, int H, const uint8_t* bytes,
 
 /* Antithetic losses of the selected probes.
  *   theta [N][P] (fp64), bytes [N][B][T+1] (one batch per expert, shared by
- *   every probe and both signs), sel[n_sel] probe indices in [0, n_pert).
+ *   every probe and both signs) or, with batch_per_probe, [N][n_pert][B][T+1]
+ *   (one batch per probe, App. D), sel[n_sel] probe indices in [0, n_pert).
+ *   summed_loss: the control arm of App. D, whose coefficient for probe sel[q]
+ *   is (sum_e L+_e - sum_e L-_e) / (2 eps) for every expert.
  *   Row e of theta is expert e0 + e (its index in the probe counter).
  *   out_L  [N][n_sel][2] = L(theta_e + eps z), L(theta_e - eps z)
  *   out_coef [N][n_sel]  = (L+ - L-) / (2 eps); 0 when eps == 0.
  * Returns 0 on success. */
-int oracle_spsa_losses_kind(const double* theta, int N, int e0, int E, int H, double eps,
-                            int kind, uint64_t seed, uint64_t step, const uint8_t* bytes,
-                            int B, int T, const int32_t* sel, int n_sel,
-                            double* out_L, double* out_coef, int n_threads) {
+int oracle_spsa_losses_opts(const double* theta, int N, int e0, int E, int H, double eps,
+                            int kind, int batch_per_probe, int summed_loss, int n_pert,
+                            uint64_t seed, uint64_t step, const uint8_t* bytes, int B, int T,
+                            const int32_t* sel, int n_sel, double* out_L, double* out_coef,
+                            int n_threads) {
   int64_t P = oracle_param_count(E, H);
   if (P <= 0 || N <= 0 || B <= 0 || T <= 0 || n_sel < 0 || (kind != 0 && kind != 1)) return 1;
+  if (batch_per_probe && n_pert <= 0) return 1;
   double* theta_s = (double*)malloc(sizeof(double) * (size_t)P);
   int8_t* z = (int8_t*)malloc((size_t)P);
   if (!theta_s || !z) { free(theta_s); free(z); return 2; }
+  int64_t seq_block = (int64_t)B * (T + 1);
   for (int e = 0; e < N; ++e) {
     const double* th = theta + (int64_t)e * P;
-    const uint8_t* bx = bytes + (int64_t)e * B * (T + 1);
     for (int q = 0; q < n_sel; ++q) {
       int i = sel[q];
+      /* one batch per expert (Sec. 4), or one per (expert, probe) */
+      const uint8_t* bx = bytes + (batch_per_probe ? ((int64_t)e * n_pert + i) * seq_block
+                                                   : (int64_t)e * seq_block);
       oracle_probe(seed, step, (uint32_t)(e0 + e), (uint32_t)i, kind, 0, P, z);
       double L[2];
       for (int s = 0; s < 2; ++s) {
@@ -282,9 +290,32 @@ int oracle_spsa_losses_kind(const double* theta, int N, int e0, int E, int H, do
       out_coef[(int64_t)e * n_sel + q] = (eps == 0.0) ? 0.0 : (L[0] - L[1]) / (2.0 * eps);
     }
   }
+  if (summed_loss) {
+    /* the control arm (App. D): the experts' losses are summed, then the
+     * finite difference of the sums is every expert's coefficient */
+    for (int q = 0; q < n_sel; ++q) {
+      double Lp = 0.0, Lm = 0.0;
+      for (int e = 0; e < N; ++e) {
+        Lp += out_L[((int64_t)e * n_sel + q) * 2 + 0];
+        Lm += out_L[((int64_t)e * n_sel + q) * 2 + 1];
+      }
+      double c = (eps == 0.0) ? 0.0 : (Lp - Lm) / (2.0 * eps);
+      for (int e = 0; e < N; ++e) out_coef[(int64_t)e * n_sel + q] = c;
+    }
+  }
   free(theta_s);
   free(z);
   return 0;
+}
+
+/* Antithetic losses of the selected probes with probe kind `kind`, one batch
+ * per expert shared by every probe, each expert's own loss. */
+int oracle_spsa_losses_kind(const double* theta, int N, int e0, int E, int H, double eps,
+                            int kind, uint64_t seed, uint64_t step, const uint8_t* bytes,
+                            int B, int T, const int32_t* sel, int n_sel,
+                            double* out_L, double* out_coef, int n_threads) {
+  return oracle_spsa_losses_opts(theta, N, e0, E, H, eps, kind, 0, 0, 0, seed, step, bytes, B, T,
+                                 sel, n_sel, out_L, out_coef, n_threads);
 }
 
 /* The same with dense probes (Eq. main-spsa). */

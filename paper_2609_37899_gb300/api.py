@@ -45,6 +45,11 @@ class soma_adam_config(ctypes.Structure):
                 ("t", ctypes.c_int32)]
 
 
+class soma_estimate_options(ctypes.Structure):
+    _fields_ = [("probe_kind", ctypes.c_int32), ("batch_per_probe", ctypes.c_int32),
+                ("summed_loss", ctypes.c_int32)]
+
+
 PROBE_KINDS = {"dense": 0, "sparse": 1}
 MAX_ACCUM = 64
 
@@ -91,6 +96,9 @@ def lib():
                                           ctypes.POINTER(ctypes.c_uint64), i32, vp,
                                           soma_adam_config, vp])
         _sig(L, "soma_debug_probe", i32, [u64, u64, i32, i32, i32, i64, i64, vp, vp])
+        _sig(L, "soma_spsa_estimate_opts", i32, [vp, i32, soma_dims, i32,
+                                                 ctypes.POINTER(soma_estimate_options), f32, u64,
+                                                 u64, vp, i32, i32, vp, vp, vp, sz, vp])
         _lib = L
         return L
 
@@ -163,13 +171,20 @@ def spsa_step(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int, n_
 
 def spsa_estimate(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int, n_pert: int,
                   kind: str, eps: float, seed: int, step: int, losses: torch.Tensor,
-                  coef: torch.Tensor, workspace: torch.Tensor, stream=None):
+                  coef: torch.Tensor, workspace: torch.Tensor, stream=None,
+                  batch_per_probe: bool = False, summed_loss: bool = False):
     """Losses [N, n_pert, 2] and coefficients [N, n_pert] of one accumulation
-    batch with dense or sparse probes; params are read only."""
-    N, B, T1 = byte_batch.shape
+    batch with dense or sparse probes; params are read only.  byte_batch is
+    [N, B, T+1], or [N, n_pert, B, T+1] with batch_per_probe; summed_loss
+    gives every expert the coefficient of the summed loss (control arm)."""
+    N = params.shape[0]
+    B, T1 = byte_batch.shape[-2], byte_batch.shape[-1]
+    if batch_per_probe:
+        assert tuple(byte_batch.shape[:2]) == (N, n_pert), "byte_batch [N, n_pert, B, T+1]"
     P = param_count(E, H)
-    _check(lib().soma_spsa_estimate(
-        _dev(params, torch.float32, "params", N * P), N, dims(E, H), n_pert, PROBE_KINDS[kind],
+    opts = soma_estimate_options(PROBE_KINDS[kind], int(batch_per_probe), int(summed_loss))
+    _check(lib().soma_spsa_estimate_opts(
+        _dev(params, torch.float32, "params", N * P), N, dims(E, H), n_pert, ctypes.byref(opts),
         eps, seed, step, _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
         _dev(losses, torch.float32, "losses", N * n_pert * 2),
         _dev(coef, torch.float32, "coef", N * n_pert),

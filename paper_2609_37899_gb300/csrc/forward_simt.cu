@@ -58,7 +58,7 @@ __global__ void __launch_bounds__(128) gate_step_kernel(const GateStep g) {
   const int lc = tid & 31, lk0 = (tid >> 5) * 8;  // input column lc, k range lk0..+7
   const int bcol = b0 + lc;
   const bool col_ok = bcol < B;
-  const uint8_t* seq = s.bytes + ((int64_t)e * B + (col_ok ? bcol : 0)) * (s.T + 1);
+  const uint8_t* seq = s.bytes + seq_offset(s, e, i, col_ok ? bcol : 0);
   const int xbyte = seq[g.t];
   const float* hprev =
       (g.t == 0 || !col_ok)
@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(256) head_nll_kernel(const HeadChunk hc) {
     if (ln == 0) {
       const int tc = cidx2 / B, b = cidx2 % B;
       const int t = hc.t0 + tc;
-      const int y = s.bytes[((int64_t)e * B + b) * (s.T + 1) + t + 1];
+      const int y = s.bytes[seq_offset(s, e, i, b) + t + 1];
       const float nll = (mx + logf(se_)) - sm.Lg[y][j];
       hc.nll[((int64_t)lane_id * B + b) * s.T + t] = nll;
     }

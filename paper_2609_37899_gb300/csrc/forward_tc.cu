@@ -470,7 +470,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
         red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
       }
       if (b < s.B) {
-        const int y = s.bytes[((int64_t)T.e * s.B + b) * (s.T + 1) + t + 1] - vq - r4;
+        const int y = s.bytes[seq_offset(s, T.e, i, b) + t + 1] - vq - r4;
         // y = 8 k for the thread that holds the target row
         if (y >= 0 && y < 32 && (y & 7) == 0) {
           const int k = y >> 3;
@@ -749,7 +749,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
     if (i < s.n_pert && b < s.B) {
-      const int y = s.bytes[((int64_t)e * s.B + b) * (s.T + 1) + t];
+      const int y = s.bytes[seq_offset(s, e, i, b) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
       ProbeBits bits = {0u, 0u};
       if (delta && s.eps != 0.f)

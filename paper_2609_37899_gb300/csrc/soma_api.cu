@@ -158,6 +158,7 @@ int soma_init_experts(float* params, int n_experts, soma_dims d, uint64_t seed, 
 
 // Forward sweep, reduction and (optionally) the SGD update of one step.
 static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, int sparse,
+                        int batch_per_probe, int summed_loss,
                         float eps, float lr, bool update, uint64_t seed, uint64_t step,
                         const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
                         float* coef_out, void* workspace, size_t workspace_bytes, void* stream) {
@@ -183,6 +184,7 @@ static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, i
   s.T = seq_len;
   s.eps = eps;
   s.sparse = sparse;
+  s.batch_per_probe = batch_per_probe;
   s.seed = seed;
   s.step = step;
   float* coef_ws = coef_scratch(w, workspace);
@@ -200,6 +202,7 @@ static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, i
       e = launch_reduce_losses(fb.nll, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
                                coef_out, coef_ws, status, st);
   }
+  if (summed_loss && e == cudaSuccess) e = launch_sum_over_experts(coef_out, n_experts, n_pert, st);
   // eps == 0 makes every coefficient 0 and lr == 0 every step 0: theta stays
   // bit-identical, so the update is not launched at all.
   if (update && e == cudaSuccess && eps != 0.f && lr != 0.f)
@@ -211,21 +214,36 @@ int soma_spsa_step(float* params, int n_experts, soma_dims d, int n_pert, float 
                    uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
                    int seq_len, float* losses_out, float* coef_out, void* workspace,
                    size_t workspace_bytes, void* stream) {
-  return spsa_forward(params, n_experts, d, n_pert, 0, eps, lr, true, seed, step, byte_batch,
+  return spsa_forward(params, n_experts, d, n_pert, 0, 0, 0, eps, lr, true, seed, step, byte_batch,
                       batch, seq_len, losses_out, coef_out, workspace, workspace_bytes, stream);
+}
+
+int soma_spsa_estimate_opts(const float* params, int n_experts, soma_dims d, int n_pert,
+                            const soma_estimate_options* opts, float eps, uint64_t seed,
+                            uint64_t step, const uint8_t* byte_batch, int batch, int seq_len,
+                            float* losses_out, float* coef_out, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!coef_out || !opts ||
+      (opts->probe_kind != SOMA_PROBE_DENSE && opts->probe_kind != SOMA_PROBE_SPARSE) ||
+      (opts->batch_per_probe != 0 && opts->batch_per_probe != 1) ||
+      (opts->summed_loss != 0 && opts->summed_loss != 1))
+    return SOMA_ERR_INVALID_ARG;
+  // the forward sweep only reads params
+  return spsa_forward(const_cast<float*>(params), n_experts, d, n_pert, opts->probe_kind,
+                      opts->batch_per_probe, opts->summed_loss, eps, 0.f, false, seed, step,
+                      byte_batch, batch, seq_len, losses_out, coef_out, workspace,
+                      workspace_bytes, stream);
 }
 
 int soma_spsa_estimate(const float* params, int n_experts, soma_dims d, int n_pert,
                        int probe_kind, float eps, uint64_t seed, uint64_t step,
                        const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
                        float* coef_out, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
-  if (!coef_out || (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE))
-    return SOMA_ERR_INVALID_ARG;
-  // the forward sweep only reads params
-  return spsa_forward(const_cast<float*>(params), n_experts, d, n_pert, probe_kind, eps, 0.f,
-                      false, seed, step, byte_batch, batch, seq_len, losses_out, coef_out,
-                      workspace, workspace_bytes, stream);
+  const soma_estimate_options opts = {probe_kind, 0, 0};
+  return soma_spsa_estimate_opts(params, n_experts, d, n_pert, &opts, eps, seed, step,
+                                 byte_batch, batch, seq_len, losses_out, coef_out, workspace,
+                                 workspace_bytes, stream);
 }
 
 int soma_adam_update(float* params, float* m, float* v, int n_experts, soma_dims d, int n_pert,
@@ -280,6 +298,7 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
   s.T = seq_len;
   s.eps = 0.f;
   s.sparse = 0;
+  s.batch_per_probe = 0;
   s.seed = 0;
   s.step = 0;
   cudaError_t e;

@@ -88,6 +88,7 @@ struct AdamArgs {
   float lr, b1, b2, delta, wd, inv_bc1, inv_bc2;
 };
 
+cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cudaStream_t stream);
 cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                                const float* coef, const AdamArgs& h, cudaStream_t stream);

@@ -168,6 +168,18 @@ adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __r
   }
 }
 
+// The summed-loss control arm (App. D): the N experts' losses are summed
+// before each finite difference, so every expert's coefficient of probe i is
+// sum_e (L+_{e,i} - L-_{e,i}) / (2 eps) = sum_e c_{e,i}.  One thread per
+// probe, experts summed in order in fp64.
+__global__ void sum_over_experts_kernel(float* coef, int n_experts, int n_pert) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_pert) return;
+  double acc = 0.0;
+  for (int e = 0; e < n_experts; ++e) acc += (double)coef[(int64_t)e * n_pert + i];
+  for (int e = 0; e < n_experts; ++e) coef[(int64_t)e * n_pert + i] = (float)acc;
+}
+
 // Box-Muller normals from Philox4x32-10 in the init domain (counter word 3
 // = 0x80000001): parameters 2q and 2q+1 of expert e use counter (q, e, 0, .).
 __global__ void init_kernel(float* __restrict__ params, Layout lay, uint64_t seed, float std) {
@@ -269,6 +281,13 @@ cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, in
   const int64_t words = (count + 31) / 32;
   debug_rademacher_kernel<<<(unsigned)((words + 127) / 128), 128, 0, stream>>>(pk, sparse, p0,
                                                                                 count, z);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cudaStream_t stream) {
+  trace_begin(SOMA_TRACE_REDUCE, stream);
+  sum_over_experts_kernel<<<(n_pert + 127) / 128, 128, 0, stream>>>(coef, n_experts, n_pert);
+  trace_end(SOMA_TRACE_REDUCE, stream);
   return cudaGetLastError();
 }
 
