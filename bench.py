@@ -44,9 +44,9 @@ UNIT = "perturbed tokens/s"
 TRAFFIC = {
     # profiles/tc_persistent_kernel_soma_n2.md: the gate launch, captured on
     # the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
-    "soma_n2": {"bytes_per_launch": 64.05888e6 + 5.80224e6,
+    "soma_n2": {"bytes_per_launch": 64.060416e6 + 5.587968e6,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "0fd1afb54fdcb1e9"},
+                "source_hash": "e83525c8c502e592"},
 }
 
 
@@ -66,6 +66,11 @@ def parse():
                     help="probe kind of --optimizer adam (default sparse, as the paper)")
     ap.add_argument("--accum", type=int, default=1,
                     help="accumulation batches per --optimizer adam update")
+    ap.add_argument("--batch-per-probe", action="store_true",
+                    help="--optimizer adam: an independent batch for every probe (App. D)")
+    ap.add_argument("--summed-loss", action="store_true",
+                    help="--optimizer adam: the control arm that sums the experts' losses "
+                         "before each finite difference (App. D)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seqs", type=int, default=32,
                     help="sequences in the one-probe sample of the cpu_baseline timing")
@@ -267,9 +272,19 @@ def our_arm(args):
     experts.init(seed=1000 + rank, std=c["init_std"] or 0.0)
     # every step gets its own A batches: (W + K) A host batches, pinned, and
     # their HBM-resident copies for the device-timed run
-    host = [[torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=A * s + a,
-                                                  seq_len=c["seq_len"])).pin_memory()
-             for a in range(A)] for s in range(W + K)]
+    per_probe = adam and args.batch_per_probe
+    summed = adam and args.summed_loss
+
+    def host_batch(k):
+        if not per_probe:
+            return torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=k,
+                                                        seq_len=c["seq_len"])).pin_memory()
+        # [N, n, B, T+1]: probe i of batch k draws its own sequences
+        return torch.from_numpy(np.stack(
+            [inputs.config_batch(args.config, seed=rank, step=k * n + i, seq_len=c["seq_len"])
+             for i in range(n)], axis=1)).pin_memory()
+
+    host = [[host_batch(A * s + a) for a in range(A)] for s in range(W + K)]
     resident = [[h.to(dev) for h in hs] for hs in host]
 
     def do_step(batches, s):
@@ -278,7 +293,8 @@ def our_arm(args):
         if not adam:
             return experts.step(batches[0], c["eps"], c["lr"], 0, s)[0]
         losses, _ = experts.adam_step(batches, c["eps"], 0, [A * s + a for a in range(A)],
-                                      t=s + 1, lr=c["lr"], kind=kind)
+                                      t=s + 1, lr=c["lr"], kind=kind,
+                                      batch_per_probe=per_probe, summed_loss=summed)
         return losses
     stream = torch.cuda.current_stream(dev)
     # written between timed steps so that no step starts with the previous
@@ -353,7 +369,9 @@ def our_arm(args):
             "workload": workload_desc(args.config, c),
             "optimizer": ("SGD, dense probes (Eq. main-spsa)" if not adam else
                           f"Adam with coupled decay, {kind} probes, {A} accumulation batch(es) "
-                          "per update (Eq. localspsa)"),
+                          "per update (Eq. localspsa)"
+                          + ("; a batch per probe" if per_probe else "")
+                          + ("; summed-loss control arm" if summed else "")),
             "tokens_per_step_per_gpu": tokens_per_step(c) * A,
             "seq_len": T,
             "l2": "flushed between timed steps (a 256 MiB buffer is written before each "

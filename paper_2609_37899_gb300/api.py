@@ -311,7 +311,8 @@ class SomaExperts:
 
     def adam_step(self, byte_batches, eps: float, seed: int, steps, t: int, lr: float,
                   beta1: float = 0.9, beta2: float = 0.999, delta: float = 1e-8,
-                  weight_decay: float = 1e-4, kind: str = "sparse", stream=None):
+                  weight_decay: float = 1e-4, kind: str = "sparse", stream=None,
+                  batch_per_probe: bool = False, summed_loss: bool = False):
         """The paper's optimizer step: one estimate per accumulation batch
         (byte_batches[a] with probe step counter steps[a]), then the Adam
         update with bias correction for update t.  Moments live on this
@@ -328,7 +329,7 @@ class SomaExperts:
         for a in range(A):
             spsa_estimate(self.params, byte_batches[a], self.E, self.H, self.n_pert, kind, eps,
                           seed, steps[a], self.losses_acc[a], self.coef_acc[a], self.workspace,
-                          stream)
+                          stream, batch_per_probe=batch_per_probe, summed_loss=summed_loss)
         adam_update(self.params, self.m, self.v, self.E, self.H, kind, seed, steps, self.coef_acc,
                     lr, beta1, beta2, delta, weight_decay, t, stream)
         return self.losses_acc, self.coef_acc
