@@ -71,6 +71,11 @@ def parse():
     ap.add_argument("--summed-loss", action="store_true",
                     help="--optimizer adam: the control arm that sums the experts' losses "
                          "before each finite difference (App. D)")
+    ap.add_argument("--inference", action="store_true",
+                    help="routed inference (Eq. main-mixture) on the workload's experts instead "
+                         "of a training step: --requests requests of seq_len bytes, k = min(4, N) "
+                         "random routes each, the last 3/4 of the positions scored")
+    ap.add_argument("--requests", type=int, default=4096)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seqs", type=int, default=32,
                     help="sequences in the one-probe sample of the cpu_baseline timing")
@@ -404,10 +409,92 @@ def our_arm(args):
     return 0
 
 
+def inference_arm(args):
+    """Routed inference: scored tokens/s of soma_mixture_nll, routing included."""
+    import torch
+    from paper_2609_37899_gb300 import api, build, inputs
+    if not os.path.exists(api.LIB_PATH):
+        build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    c = dict(inputs.CONFIGS[args.config])
+    if args.seq_len:
+        c["seq_len"] = args.seq_len
+    N, E, H, T = c["n_experts"], c["E"], c["H"], c["seq_len"]
+    R, k, t0 = args.requests, min(4, c["n_experts"]), c["seq_len"] // 4
+    K, W = args.steps, args.warmup
+    params = torch.empty(N, api.param_count(E, H), dtype=torch.float32, device=dev)
+    api.init_experts(params, E, H, seed=1000, std=c["init_std"] or 0.0)
+    rng = np.random.default_rng(7)
+    # routes: k distinct experts per request, uniformly (the fitted router is
+    # not available); requests: the workload's byte streams
+    routes = [np.stack([rng.choice(N, size=k, replace=False) for _ in range(R)]).astype(np.int32)
+              for _ in range(W + K)]
+    host = []
+    for s in range(W + K):
+        rows = []
+        while sum(len(x) for x in rows) < R:
+            rows.append(inputs.config_batch(args.config, seed=1, step=100 * s + len(rows),
+                                            seq_len=T).reshape(-1, T + 1))
+        host.append(torch.from_numpy(np.concatenate(rows)[:R]).pin_memory())
+    resident = [h.to(dev) for h in host]
+    ws = torch.empty(max(api.mixture_workspace_bytes(E, H, N, r, T) for r in routes),
+                     dtype=torch.uint8, device=dev)
+    out = torch.empty(R, T - t0, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for s in range(W):
+        api.mixture_nll(params, resident[s], E, H, routes[s], t0, out, ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        e0.record(stream)
+        for s in range(K):
+            flush.fill_(s & 0xFF)
+            api.mixture_nll(params, resident[W + s], E, H, routes[W + s], t0, out, ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    out_host = torch.empty_like(out, device="cpu").pin_memory()
+    dev_rq = torch.empty_like(resident[0])
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for s in range(K):
+        flush.fill_(s & 0xFF)
+        dev_rq.copy_(host[W + s], non_blocking=True)
+        api.mixture_nll(params, dev_rq, E, H, routes[W + s], t0, out, ws)
+        out_host.copy_(out, non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    ms_e2e = f0.elapsed_time(f1)
+    status = api.get_status()
+    tok = R * (T - t0)
+    line = {
+        "metric": "scored tokens/s, routed inference (Eq. main-mixture)", "value": tok * K / (ms / 1e3),
+        "unit": "scored tokens/s", "n_gpus": 1, "steps": K, "warmup": W, "ms_per_step": ms / K,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": DTYPE,
+        "data": "synthetic",
+        "config": {"workload": workload_desc(args.config, c) + f"; {R} requests x {T} bytes, "
+                               f"k={k} uniform random routes, positions {t0}..{T - 1} scored, "
+                               "routing (host grouping) inside the timed region",
+                   "l2": "flushed between timed steps (256 MiB written before each)"},
+        "e2e": {"value": tok * K / (ms_e2e / 1e3), "unit": "scored tokens/s",
+                "h2d_bytes_per_step": int(resident[0].numel()),
+                "d2h_bytes_per_step": int(out.numel() * 4)},
+        "clocks": clk.summary(),
+        "status": api.STATUS_NAMES.get(status, status),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return reference_arm(args)
+    if args.inference:
+        return inference_arm(args)
     return our_arm(args)
 
 

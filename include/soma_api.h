@@ -197,6 +197,26 @@ int soma_adam_update(float* params, float* m, float* v, int n_experts, soma_dims
                      int probe_kind, uint64_t seed, const uint64_t* steps, int n_acc,
                      const float* coef, soma_adam_config cfg, void* stream);
 
+/* ---- Routed inference (Sec. 3, Eq. main-mixture) ----------------------
+ * Request r (teacher-forced, LSTM state reset to zero) is scored by the k
+ * experts routes[r][0..k-1]; its prediction averages their probabilities,
+ *   p(y | x_<t) = (1/k) sum_j p_{routes[r][j]}(y | x_<t),
+ * and nll_out[r][t - t0] = -log p(byte_{t+1} | bytes_<=t) for t0 <= t < seq_len.
+ * The routes come from the caller (the paper's router is a fitted tf-idf
+ * model); an expert may be listed more than once.  Requests are grouped by
+ * expert and each expert runs on its group in sweeps of up to 64 sequences.
+ *   params    device fp32 [n_experts][P]
+ *   requests  device uint8 [R][seq_len + 1]
+ *   routes    HOST int32 [R][k], entries in [0, n_experts); 1 <= k <= 16
+ *   nll_out   device fp32 [R][seq_len - t0]; 0 <= t0 < seq_len
+ * The workspace size depends on the routing (the largest group), hence the
+ * routes argument of soma_mixture_workspace_bytes (0 if invalid). */
+size_t soma_mixture_workspace_bytes(soma_dims d, int n_experts, const int32_t* routes, int R,
+                                    int k, int seq_len);
+int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint8_t* requests,
+                     int R, int seq_len, const int32_t* routes, int k, int t0, float* nll_out,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
 /* Synchronises `stream`, then returns and clears the current device's status
  * word (SOMA_OK if no device-side error was recorded since the last call).
  * Returns SOMA_ERR_CUDA if the synchronisation itself failed. */

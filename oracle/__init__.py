@@ -98,6 +98,11 @@ def _load():
                                                 ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
                                                 c_dp, c_dp, ctypes.c_int]
         lib.oracle_spsa_losses_opts.restype = ctypes.c_int
+        lib.oracle_mixture_nll.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int, c_u8p,
+                                           ctypes.c_int, ctypes.c_int,
+                                           ctypes.POINTER(ctypes.c_int32), ctypes.c_int,
+                                           ctypes.c_int, c_dp, ctypes.c_int]
+        lib.oracle_mixture_nll.restype = ctypes.c_int
         lib.oracle_probe.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32,
                                      ctypes.c_uint32, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
                                      ctypes.POINTER(ctypes.c_int8)]
@@ -268,6 +273,24 @@ def adam_update(theta, m, v, E: int, H: int, seed: int, steps, coef, lr: float, 
     if rc != 0:
         raise RuntimeError(f"oracle_adam_update failed ({rc})")
     return to, mo, vo
+
+
+def mixture_nll(theta, E: int, H: int, requests, routes, t0: int, n_threads: int = 0):
+    """Routed-inference NLL [R, T - t0] (Eq. main-mixture): requests [R, T+1]
+    uint8, routes [R, k] expert indices into theta [N, P]."""
+    th = _f64(theta)
+    N = th.shape[0]
+    rq = _u8(requests)
+    R, T = rq.shape[0], rq.shape[1] - 1
+    rt = np.ascontiguousarray(routes, dtype=np.int32)
+    k = rt.shape[1]
+    out = np.zeros((R, T - t0), dtype=np.float64)
+    rc = _load().oracle_mixture_nll(_ptr(th, ctypes.c_double), N, E, H, _ptr(rq, ctypes.c_uint8),
+                                    R, T, _ptr(rt, ctypes.c_int32), k, t0,
+                                    _ptr(out, ctypes.c_double), n_threads)
+    if rc != 0:
+        raise RuntimeError(f"oracle_mixture_nll failed ({rc})")
+    return out
 
 
 def bptt_grad(theta, E: int, H: int, bytes_):

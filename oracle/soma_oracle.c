@@ -30,7 +30,9 @@
  *     Rademacher probes (a coordinate is 0 with probability 1/2 and -1 or +1
  *     with probability 1/4 each), the estimate averaged over A accumulation
  *     batches, coupled weight decay added before the moments, and Adam with
- *     bias-corrected moments.
+ *     bias-corrected moments;
+ *   - routed inference: the average of the routed experts' next-byte
+ *     probabilities (Sec. 3, Eq. main-mixture).
  *
  * Parameter layout of one expert (flat, row-major, gate blocks i,f,g,o):
  *   Emb[V][E], W_ih[4H][E], W_hh[4H][H], b[4H], W_out[V][H], b_out[V].
@@ -399,6 +401,33 @@ int oracle_adam_update(const double* theta, const double* m, const double* v, in
   }
   free(g);
   free(z);
+  return 0;
+}
+
+/* Routed inference (Sec. 3, Eq. main-mixture), in fp64: request r is read by
+ * its k routed experts routes[r][j] (state reset to zero), and
+ *   out[r][t - t0] = -log( (1/k) sum_j p_{routes[r][j]}(byte_{t+1} | bytes_<=t) )
+ * for t0 <= t < T.  theta [N][P], requests [R][T+1]. */
+int oracle_mixture_nll(const double* theta, int N, int E, int H, const uint8_t* requests, int R,
+                       int T, const int32_t* routes, int k, int t0, double* out, int n_threads) {
+  int64_t P = oracle_param_count(E, H);
+  if (P <= 0 || N <= 0 || R <= 0 || T <= 0 || k <= 0 || t0 < 0 || t0 >= T) return 1;
+  double* nll = (double*)malloc(sizeof(double) * (size_t)k * T);
+  if (!nll) return 2;
+  for (int r = 0; r < R; ++r) {
+    const uint8_t* seq = requests + (int64_t)r * (T + 1);
+    for (int j = 0; j < k; ++j) {
+      int e = routes[(int64_t)r * k + j];
+      if (e < 0 || e >= N) { free(nll); return 1; }
+      oracle_loss(theta + (int64_t)e * P, E, H, seq, 1, T, nll + (int64_t)j * T, n_threads);
+    }
+    for (int t = t0; t < T; ++t) {
+      double p = 0.0;
+      for (int j = 0; j < k; ++j) p += exp(-nll[(int64_t)j * T + t]);
+      out[(int64_t)r * (T - t0) + (t - t0)] = -log(p / (double)k);
+    }
+  }
+  free(nll);
   return 0;
 }
 

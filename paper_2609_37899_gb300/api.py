@@ -96,6 +96,10 @@ def lib():
                                           ctypes.POINTER(ctypes.c_uint64), i32, vp,
                                           soma_adam_config, vp])
         _sig(L, "soma_debug_probe", i32, [u64, u64, i32, i32, i32, i64, i64, vp, vp])
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        _sig(L, "soma_mixture_workspace_bytes", sz, [soma_dims, i32, i32p, i32, i32, i32])
+        _sig(L, "soma_mixture_nll", i32, [vp, i32, soma_dims, vp, i32, i32, i32p, i32, i32, vp,
+                                          vp, sz, vp])
         _sig(L, "soma_spsa_estimate_opts", i32, [vp, i32, soma_dims, i32,
                                                  ctypes.POINTER(soma_estimate_options), f32, u64,
                                                  u64, vp, i32, i32, vp, vp, vp, sz, vp])
@@ -205,6 +209,37 @@ def adam_update(params: torch.Tensor, m: torch.Tensor, v: torch.Tensor, E: int, 
         _dev(v, torch.float32, "v", N * P), N, dims(E, H), n_pert, PROBE_KINDS[kind], seed, st,
         A, _dev(coef, torch.float32, "coef", A * N * n_pert), cfg, _stream(stream)),
         "soma_adam_update")
+
+
+def _routes(routes):
+    import numpy as np
+    rt = np.ascontiguousarray(routes, dtype=np.int32)
+    assert rt.ndim == 2, "routes [R, k]"
+    return rt, rt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def mixture_workspace_bytes(E: int, H: int, n_experts: int, routes, seq_len: int) -> int:
+    rt, ptr = _routes(routes)
+    n = int(lib().soma_mixture_workspace_bytes(dims(E, H), n_experts, ptr, rt.shape[0],
+                                               rt.shape[1], seq_len))
+    if n == 0:
+        raise SomaError(1, "soma_mixture_workspace_bytes: invalid sizes or routes")
+    return n
+
+
+def mixture_nll(params: torch.Tensor, requests: torch.Tensor, E: int, H: int, routes, t0: int,
+                nll_out: torch.Tensor, workspace: torch.Tensor, stream=None):
+    """Routed inference (Eq. main-mixture): nll_out [R, T - t0] for requests
+    [R, T+1] (device) and host routes [R, k]."""
+    rt, ptr = _routes(routes)
+    R, T1 = requests.shape
+    N = params.shape[0]
+    _check(lib().soma_mixture_nll(
+        _dev(params, torch.float32, "params", N * param_count(E, H)), N, dims(E, H),
+        _dev(requests, torch.uint8, "requests"), R, T1 - 1, ptr, rt.shape[1], t0,
+        _dev(nll_out, torch.float32, "nll_out", R * (T1 - 1 - t0)),
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_mixture_nll")
 
 
 def eval_loss(params: torch.Tensor, byte_batch: torch.Tensor, E: int, H: int,

@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <vector>
 
 #include "soma_api.h"
 #include "soma_launch.h"
@@ -391,3 +392,130 @@ int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int pro
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Routed inference (Sec. 3, Eq. main-mixture)
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int kMaxRoutes = 16;
+constexpr int kMixChunk = 64;  // sequences per expert and sweep (the tensor path's limit)
+
+struct MixPlan {
+  int b_max, Bc, chunks;
+  WsPlan sweep;
+  size_t gather, route, slot, grouped, nll, total;
+  std::vector<int32_t> gather_h, slot_h;
+};
+
+// Groups the requests by expert: request r's j-th route lands in slot
+// slot_h[r][j] of expert routes[r][j]; gather_h[e][slot] = r.
+bool plan_mixture(const soma_dims& d, int N, const int32_t* routes, int R, int k, int T,
+                  MixPlan& m) {
+  std::vector<int> count((size_t)N, 0);
+  m.slot_h.assign((size_t)R * k, 0);
+  for (int r = 0; r < R; ++r)
+    for (int j = 0; j < k; ++j) {
+      const int e = routes[(size_t)r * k + j];
+      if (e < 0 || e >= N) return false;
+      m.slot_h[(size_t)r * k + j] = count[(size_t)e]++;
+    }
+  m.b_max = 1;
+  for (int e = 0; e < N; ++e) m.b_max = count[(size_t)e] > m.b_max ? count[(size_t)e] : m.b_max;
+  m.gather_h.assign((size_t)N * m.b_max, -1);
+  for (int r = 0; r < R; ++r)
+    for (int j = 0; j < k; ++j)
+      m.gather_h[(size_t)routes[(size_t)r * k + j] * m.b_max + m.slot_h[(size_t)r * k + j]] = r;
+  m.Bc = m.b_max < kMixChunk ? m.b_max : kMixChunk;
+  m.chunks = (m.b_max + m.Bc - 1) / m.Bc;
+  m.sweep = plan_sweep(d, N, 1, 1, m.Bc, T);
+  m.gather = round_up((size_t)N * m.b_max * sizeof(int32_t));
+  m.route = round_up((size_t)R * k * sizeof(int32_t));
+  m.slot = m.route;
+  m.grouped = round_up((size_t)N * m.Bc * (T + 1));
+  m.nll = round_up((size_t)N * m.b_max * T * sizeof(float));
+  m.total = m.sweep.total + m.gather + m.route + m.slot + m.grouped + m.nll;
+  return true;
+}
+
+bool mixture_args_ok(int n_experts, const int32_t* routes, int R, int k, int seq_len, int t0) {
+  return n_experts >= 1 && routes && R >= 1 && k >= 1 && k <= kMaxRoutes && seq_len >= 1 &&
+         t0 >= 0 && t0 < seq_len && sizes_ok(n_experts, 1, 1, seq_len);
+}
+
+}  // namespace
+
+size_t soma_mixture_workspace_bytes(soma_dims d, int n_experts, const int32_t* routes, int R,
+                                    int k, int seq_len) {
+  if (!dims_ok(d) || !mixture_args_ok(n_experts, routes, R, k, seq_len, 0)) return 0;
+  MixPlan m;
+  if (!plan_mixture(d, n_experts, routes, R, k, seq_len, m)) return 0;
+  return m.total;
+}
+
+int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint8_t* requests,
+                     int R, int seq_len, const int32_t* routes, int k, int t0, float* nll_out,
+                     void* workspace, size_t workspace_bytes, void* stream) {
+  if (!dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !requests || !nll_out || !aligned16(params) ||
+      !mixture_args_ok(n_experts, routes, R, k, seq_len, t0))
+    return SOMA_ERR_INVALID_ARG;
+  MixPlan m;
+  if (!plan_mixture(d, n_experts, routes, R, k, seq_len, m)) return SOMA_ERR_INVALID_ARG;
+  if (!workspace || !aligned16(workspace) || workspace_bytes < m.total) return SOMA_ERR_WORKSPACE;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+  char* base = static_cast<char*>(workspace);
+  void* sweep_ws = base;
+  int32_t* gather = reinterpret_cast<int32_t*>(base + m.sweep.total);
+  int32_t* route = reinterpret_cast<int32_t*>(base + m.sweep.total + m.gather);
+  int32_t* slot = reinterpret_cast<int32_t*>(base + m.sweep.total + m.gather + m.route);
+  uint8_t* grouped =
+      reinterpret_cast<uint8_t*>(base + m.sweep.total + m.gather + m.route + m.slot);
+  float* nll = reinterpret_cast<float*>(base + m.sweep.total + m.gather + m.route + m.slot +
+                                        m.grouped);
+  // the routing tables (host, built above) go with the stream's work; the
+  // copies from pageable memory return once the data is staged
+  cudaError_t e = cudaMemcpyAsync(gather, m.gather_h.data(), m.gather_h.size() * sizeof(int32_t),
+                                  cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(route, routes, (size_t)R * k * sizeof(int32_t), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(slot, m.slot_h.data(), m.slot_h.size() * sizeof(int32_t),
+                        cudaMemcpyHostToDevice, st);
+  Sweep s;
+  s.params = params;
+  s.bytes = grouped;
+  s.lay = make_layout(d.embed, d.hidden);
+  s.n_experts = n_experts;
+  s.n_pert = 1;
+  s.n_sign = 1;
+  s.B = m.Bc;
+  s.T = seq_len;
+  s.eps = 0.f;
+  s.sparse = 0;
+  s.batch_per_probe = 0;
+  s.seed = 0;
+  s.step = 0;
+  for (int c = 0; c < m.chunks && e == cudaSuccess; ++c) {
+    const int b0 = c * m.Bc;
+    e = launch_gather_requests(requests, gather, n_experts, m.b_max, b0, m.Bc, seq_len + 1,
+                               grouped, st);
+    if (e != cudaSuccess) break;
+    if (m.sweep.tc) {
+      const TcBuffers tb = carve_tc(m.sweep, sweep_ws);
+      e = launch_forward_tc(s, m.sweep.g, tb, status, st);
+      if (e == cudaSuccess)
+        e = launch_token_nll_tc(tb, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
+    } else {
+      const ForwardBuffers fb = carve(m.sweep, sweep_ws);
+      e = launch_forward_simt(s, fb, st);
+      if (e == cudaSuccess)
+        e = launch_token_nll_copy(fb.nll, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
+    }
+  }
+  if (e == cudaSuccess)
+    e = launch_mixture(nll, route, slot, R, k, seq_len, t0, m.b_max, nll_out, st);
+  return cuda_status(e);
+}

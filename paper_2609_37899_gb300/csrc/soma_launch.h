@@ -88,6 +88,16 @@ struct AdamArgs {
   float lr, b1, b2, delta, wd, inv_bc1, inv_bc2;
 };
 
+// Routed inference (mixture.cu).
+cudaError_t launch_gather_requests(const uint8_t* requests, const int32_t* gather, int N,
+                                   int b_max, int b0, int Bc, int T1, uint8_t* grouped,
+                                   cudaStream_t stream);
+cudaError_t launch_token_nll_tc(const TcBuffers& tb, int N, int Bc, int T, int b_max, int b0,
+                                float* nll, cudaStream_t stream);
+cudaError_t launch_token_nll_copy(const float* src, int N, int Bc, int T, int b_max, int b0,
+                                  float* nll, cudaStream_t stream);
+cudaError_t launch_mixture(const float* nll, const int32_t* route, const int32_t* slot, int R,
+                           int k, int T, int t0, int b_max, float* out, cudaStream_t stream);
 cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cudaStream_t stream);
 cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,

@@ -30,7 +30,8 @@ def test_header_declares_the_entry_points():
                      "soma_workspace_bytes", "soma_param_count", "soma_get_status",
                      "soma_status_string", "soma_spsa_update", "soma_debug_philox",
                      "soma_debug_rademacher", "soma_spsa_estimate", "soma_adam_update",
-                     "soma_debug_probe"]:
+                     "soma_debug_probe", "soma_spsa_estimate_opts", "soma_mixture_nll",
+                     "soma_mixture_workspace_bytes"]:
         assert required in names
 
 
@@ -117,3 +118,12 @@ def test_host_validation_rejects_before_launch(soma):
         assert L.soma_adam_update(fake, fake, fake, 1, d, 8, 1, 0, steps, 2, fake, bad,
                                   None) == 1
     assert L.soma_debug_probe(0, 0, 0, 0, 3, 0, 4, fake, None) == 1
+    # routed inference: routes are checked on the host
+    bad = (ctypes.c_int32 * 2)(0, 5)
+    assert L.soma_mixture_workspace_bytes(d, 2, bad, 1, 2, 8) == 0
+    assert L.soma_mixture_nll(fake, 2, d, fake, 1, 8, bad, 2, 0, fake, fake, 1 << 20, None) == 1
+    good = (ctypes.c_int32 * 2)(0, 1)
+    assert L.soma_mixture_nll(fake, 2, d, fake, 1, 8, good, 2, 8, fake, fake, 1 << 20,
+                              None) == 1  # t0 = seq_len
+    assert L.soma_mixture_nll(fake, 2, d, fake, 1, 8, good, 17, 0, fake, fake, 1 << 20,
+                              None) == 1  # k > 16
