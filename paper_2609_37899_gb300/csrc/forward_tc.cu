@@ -216,14 +216,6 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
-// Gate tile rows: a 128-row tile covers 32 hidden units.  Tile row r lies in
-// TMEM lane quarter r / 32 and holds gate (r / 8) % 4 of unit 8 (r / 32) +
-// r % 8, so one quarter = 8 units x 4 gates, gate-major.  With this order a
-// 16x128b tensor-memory load (rows l / 4 and 8 + l / 4 of a 16-lane half)
-// gives thread l two gates of unit l / 4, and the two halves give all four.
-__host__ __device__ __forceinline__ int tile_unit(int r) { return 8 * (r >> 5) + (r & 7); }
-__host__ __device__ __forceinline__ int tile_gate(int r) { return (r >> 3) & 3; }
-
 struct TcArgs {
   Sweep sw;
   TcGeom g;

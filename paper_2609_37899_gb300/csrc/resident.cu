@@ -1,0 +1,482 @@
+// resident.cu -- the SPSA forward of small experts with the whole recurrence
+// resident in one CTA (tcgen05 / TMEM).
+//
+// One CTA runs one (expert, probe) pair, both signs, over all T timesteps in
+// the mean/difference form of forward_tc.cu:
+//   a+- = C +- D,  C = W vbar + eps (Z dv) + b,  D = W dv + eps (Z vbar) + eps z_b.
+// The gate weights W = [W_ih | W_hh], the head weights W_out and the probe
+// tiles Z of this pair are converted to fp16 tiles in shared memory once,
+// and the probes are therefore drawn once per step, not once per timestep.
+// The operand [vbar | dv] (rows) x [x | h] (K) also lives in shared memory:
+// the gate epilogue writes h of timestep t straight into it, where the head
+// of t and the gate of t + 1 read it.  Cell states stay in registers, and
+// the losses are summed in the CTA.  Per timestep:
+//   MMAs   head(t - 1) and gate(t) (one thread), one commit;
+//   head epilogue of t - 1: max / sum-exp per (sequence, sign) over both
+//          vocabulary halves, target logit, NLL summed in fp64;
+//   gate epilogue of t: gates and cells, h of t into the operand;
+//   the embedding part of the operand of t + 1.
+// The shape limits (H <= 64, B <= 32, the tiles within shared memory) are
+// checked by res_supported(); larger experts use the persistent kernel.
+#include <cuda_fp16.h>
+
+#include "soma_api.h"
+#include "soma_device.cuh"
+#include "soma_launch.h"
+#include "tc_primitives.cuh"
+
+namespace soma {
+
+using namespace tc;
+
+namespace {
+
+constexpr int kResThreads = 256;  // 8 warps: two M tiles x four TMEM lane quarters
+constexpr int kResMaxBp = 32;
+constexpr size_t kResMaxSmem = 220 * 1024;
+constexpr uint32_t kLboRes = 128;  // bytes between core matrices along K
+
+__device__ __forceinline__ float sigm_res(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
+
+struct ResGeom {
+  int E, H, Ek, Hk, K, MTg, Bp, B, T;
+  uint32_t wg, zg, wo, zo, op, red, ylog, acc, ctl, bytes;  // shared-memory offsets
+  uint32_t tmem_cols;
+};
+
+__host__ __device__ inline uint32_t res_align(uint32_t x) { return (x + 1023u) & ~1023u; }
+
+ResGeom make_res_geom(const Layout& lay, int B, int T) {
+  ResGeom r;
+  r.E = lay.E;
+  r.H = lay.H;
+  r.Ek = (lay.E + 15) / 16 * 16;
+  r.Hk = (lay.H + 15) / 16 * 16;
+  r.K = r.Ek + r.Hk;
+  r.MTg = (lay.H + 31) / 32;
+  r.Bp = (B + 7) / 8 * 8;
+  r.B = B;
+  r.T = T;
+  uint32_t o = 0;
+  const uint32_t gate_tile = 128u * r.K * 2, head_tile = 128u * r.Hk * 2;
+  r.wg = o; o = res_align(o + r.MTg * gate_tile);
+  r.zg = o; o = res_align(o + r.MTg * gate_tile);
+  r.wo = o; o = res_align(o + 2 * head_tile);
+  r.zo = o; o = res_align(o + 2 * head_tile);
+  r.op = o; o = res_align(o + 2u * r.Bp * r.K * 2);
+  r.red = o; o += 2u * 4 * 2 * r.Bp * sizeof(float2);  // [half][quarter][sign][Bp]
+  r.ylog = o; o += 2u * r.Bp * sizeof(float);          // [sign][Bp]
+  o = (o + 7u) & ~7u;
+  r.acc = o; o += 3u * r.Bp * sizeof(double);          // per sequence: sum nll+, nll-, diff
+  o = (o + 7u) & ~7u;
+  r.ctl = o; o += 64;
+  r.bytes = o + 1024;  // alignment slack of the dynamic shared-memory base
+  const uint32_t cols = (uint32_t)(r.MTg + 2) * 4 * r.Bp;
+  r.tmem_cols = 32;
+  while (r.tmem_cols < cols) r.tmem_cols <<= 1;
+  return r;
+}
+
+struct ResArgs {
+  Sweep sw;
+  ResGeom g;
+  int n_sign;         // 2: (L+, L-) per pair; 1: L per expert (eps = 0)
+  float* losses_out;  // [N][n][2] or [N]
+  float* coef_out;    // [N][n] or null
+  float* coef_ws;     // [N][n] or null
+  int* status;
+};
+
+// z of flat parameter p as an fp16 +-1 / 0 (sparse) value.
+__device__ __forceinline__ __half z_half(const ProbeBits& b, int j) {
+  return ((b.act >> j) & 1u) ? (((b.neg >> j) & 1u) ? __float2half_rn(-1.f) : __float2half_rn(1.f))
+                             : __float2half_rn(0.f);
+}
+
+__global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
+  extern __shared__ uint8_t dyn_smem[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
+  const ResGeom& g = a.g;
+  const Sweep& s = a.sw;
+  const Layout& L = s.lay;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int e = blockIdx.x / s.n_pert, i = blockIdx.x % s.n_pert;
+  const float* th = s.params + (int64_t)e * L.P;
+  const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
+  const float eps = s.eps;
+  const bool do_z = eps != 0.f;
+  uint64_t* mma_bar = reinterpret_cast<uint64_t*>(smem + g.ctl);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 8);
+  float2* red = reinterpret_cast<float2*>(smem + g.red);
+  float* ylog = reinterpret_cast<float*>(smem + g.ylog);
+  double* acc = reinterpret_cast<double*>(smem + g.acc);
+
+  if (tid == 0) {
+    mbar_init(mma_bar, 1);
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(tmem_slot, g.tmem_cols);
+
+  // ---- resident tiles: W, Z of the gate (gate-major quarters) and the head
+  const int gate_chunks = g.MTg * 128 * (g.K / 8);
+  for (int c = tid; c < gate_chunks; c += kResThreads) {
+    const int m = c / (128 * (g.K / 8)), rem = c % (128 * (g.K / 8));
+    const int r = rem / (g.K / 8), k0 = 8 * (rem % (g.K / 8));
+    const int U = 32 * m + tile_unit(r);
+    const int64_t R = (int64_t)tile_gate(r) * g.H + U;
+    __align__(16) __half w[8], z[8];
+    int64_t p0 = -1;
+    int kmax = 0;  // valid columns of this chunk
+    if (U < g.H) {
+      if (k0 < g.Ek) {
+        p0 = L.w_ih + R * g.E + k0;
+        kmax = min(8, g.E - k0);
+      } else {
+        p0 = L.w_hh + R * g.H + (k0 - g.Ek);
+        kmax = min(8, g.H - (k0 - g.Ek));
+      }
+    }
+    ProbeBits zb = {0u, 0u};
+    if (kmax > 0 && do_z) zb = probe_bits(pk, p0, s.sparse);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const bool ok = j < kmax;
+      w[j] = __float2half_rn(ok ? th[p0 + j] : 0.f);
+      z[j] = ok ? z_half(zb, j) : __float2half_rn(0.f);
+    }
+    const uint32_t off = m * (128u * g.K * 2) + kmajor_offset(r, k0, g.K);
+    *reinterpret_cast<uint4*>(smem + g.wg + off) = *reinterpret_cast<const uint4*>(w);
+    *reinterpret_cast<uint4*>(smem + g.zg + off) = *reinterpret_cast<const uint4*>(z);
+  }
+  const int head_chunks = 2 * 128 * (g.Hk / 8);
+  for (int c = tid; c < head_chunks; c += kResThreads) {
+    const int h = c / (128 * (g.Hk / 8)), rem = c % (128 * (g.Hk / 8));
+    const int r = rem / (g.Hk / 8), k0 = 8 * (rem % (g.Hk / 8));
+    const int64_t p0 = L.w_out + (int64_t)(128 * h + r) * g.H + k0;
+    const int kmax = min(8, g.H - k0);
+    ProbeBits zb = {0u, 0u};
+    if (kmax > 0 && do_z) zb = probe_bits(pk, p0, s.sparse);
+    __align__(16) __half w[8], z[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const bool ok = j < kmax;
+      w[j] = __float2half_rn(ok ? th[p0 + j] : 0.f);
+      z[j] = ok ? z_half(zb, j) : __float2half_rn(0.f);
+    }
+    const uint32_t off = h * (128u * g.Hk * 2) + kmajor_offset(r, k0, g.Hk);
+    *reinterpret_cast<uint4*>(smem + g.wo + off) = *reinterpret_cast<const uint4*>(w);
+    *reinterpret_cast<uint4*>(smem + g.zo + off) = *reinterpret_cast<const uint4*>(z);
+  }
+  for (int c = tid; c < 2 * g.Bp * g.K / 8; c += kResThreads)
+    reinterpret_cast<uint4*>(smem + g.op)[c] = make_uint4(0u, 0u, 0u, 0u);
+  for (int c = tid; c < 3 * g.Bp; c += kResThreads) acc[c] = 0.0;
+
+  // ---- per-thread constants of the epilogues
+  // gate: warp w runs tile w / 4, TMEM lane quarter w % 4; thread l owns unit
+  // 8 (w % 4) + l / 4 of that tile and sequences b0 + l % 4, b0 + 4 + l % 4
+  const int q4 = warp & 3, tile = warp >> 2;
+  const int u8 = lane >> 2, bq = lane & 3;
+  const int U = 32 * tile + 8 * q4 + u8;
+  const bool unit_ok = tile < g.MTg && U < g.H;
+  float bias[4] = {0.f, 0.f, 0.f, 0.f}, dbias[4] = {0.f, 0.f, 0.f, 0.f};
+  if (unit_ok) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t pb = L.b + (int64_t)k * g.H + U;
+      bias[k] = th[pb];
+      if (do_z) {
+        const ProbeBits zb = probe_bits(pk, pb, s.sparse);
+        dbias[k] = eps_z(zb.neg & 1u, zb.act & 1u, eps);
+      }
+    }
+  }
+  float cst[kResMaxBp / 8][2][2];  // [chunk][sequence half][sign]
+#pragma unroll
+  for (int c = 0; c < kResMaxBp / 8; ++c)
+    cst[c][0][0] = cst[c][0][1] = cst[c][1][0] = cst[c][1][1] = 0.f;
+  // head: warp w runs vocabulary half w / 4, quarter w % 4; thread l holds
+  // rows l / 4 + 8 k (k = 0..3) of the quarter
+  const int half = warp >> 2, r4 = lane >> 2;
+  const int vq = 128 * half + 32 * q4;
+  float bo[4], dbo[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int64_t pb = L.b_out + vq + r4 + 8 * k;
+    bo[k] = th[pb];
+    dbo[k] = 0.f;
+    if (do_z) {
+      const ProbeBits zb = probe_bits(pk, pb, s.sparse);
+      dbo[k] = eps_z(zb.neg & 1u, zb.act & 1u, eps);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t gcol0 = 0, hcol0 = (uint32_t)g.MTg * 4 * g.Bp;
+  bool ok = true;
+
+  for (int t = 0; t <= g.T && ok; ++t) {
+    // embedding part of the operand of timestep t: rows [vbar (Bp) | dv (Bp)]
+    if (t < g.T) {
+      for (int c = tid; c < 2 * g.Bp * (g.Ek / 8); c += kResThreads) {
+        const int row = c / (g.Ek / 8), k0 = 8 * (c % (g.Ek / 8));
+        const bool delta = row >= g.Bp;
+        const int b = delta ? row - g.Bp : row;
+        __align__(16) __half v[8];
+        if (b < g.B) {
+          const int y = s.bytes[seq_offset(s, e, i, b) + t];
+          const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
+          const int kmax = min(8, g.E - k0);
+          ProbeBits zb = {0u, 0u};
+          if (delta && do_z && kmax > 0) zb = probe_bits(pk, p0, s.sparse);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float x = 0.f;
+            if (j < kmax)
+              x = delta ? eps_z((zb.neg >> j) & 1u, (zb.act >> j) & 1u, eps) : th[p0 + j];
+            v[j] = __float2half_rn(x);
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[j] = __float2half_rn(0.f);
+        }
+        *reinterpret_cast<uint4*>(smem + g.op + kmajor_offset(row, k0, g.K)) =
+            *reinterpret_cast<const uint4*>(v);
+      }
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t n2 = (uint32_t)(2 * g.Bp);
+      const uint32_t idesc = idesc_f16_f32(128, 2 * g.Bp);
+      const uint32_t sbase = smem_u32(smem);
+      const uint32_t gsbo = (uint32_t)g.K * 16, hsbo = (uint32_t)g.Hk * 16;
+      if (t >= 1) {  // head of t - 1: h part of the operand
+        for (int h = 0; h < 2; ++h) {
+          const uint32_t d = tmem + hcol0 + (uint32_t)h * 2 * n2;
+          for (int k16 = 0; k16 < g.Hk / 16; ++k16) {
+            const uint32_t ko = (uint32_t)k16 * 256;
+            const uint64_t bdesc =
+                smem_desc(sbase + g.op + (uint32_t)(g.Ek / 8) * 128 + ko, kLboRes, gsbo);
+            mma_f16_ss(d, smem_desc(sbase + g.wo + h * (128u * g.Hk * 2) + ko, kLboRes, hsbo),
+                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+            mma_f16_ss(d + n2, smem_desc(sbase + g.zo + h * (128u * g.Hk * 2) + ko, kLboRes, hsbo),
+                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+          }
+        }
+      }
+      if (t < g.T) {  // gate of t
+        for (int m = 0; m < g.MTg; ++m) {
+          const uint32_t d = tmem + gcol0 + (uint32_t)m * 2 * n2;
+          for (int k16 = 0; k16 < g.K / 16; ++k16) {
+            const uint32_t ko = (uint32_t)k16 * 256;
+            const uint64_t bdesc = smem_desc(sbase + g.op + ko, kLboRes, gsbo);
+            mma_f16_ss(d, smem_desc(sbase + g.wg + m * (128u * g.K * 2) + ko, kLboRes, gsbo),
+                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+            mma_f16_ss(d + n2, smem_desc(sbase + g.zg + m * (128u * g.K * 2) + ko, kLboRes, gsbo),
+                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+          }
+        }
+      }
+      mma_commit(mma_bar);
+    }
+    __syncwarp();
+    bool got = mbar_wait(mma_bar, (uint32_t)t & 1u);
+    if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
+    // one decision for the whole CTA: a timed-out wait ends the recurrence
+    // for every thread at the same barrier
+    ok = __syncthreads_and(got) != 0;
+    tc_fence_after();
+
+    if (t >= 1 && ok) {
+      // ---- head epilogue of t - 1
+      const uint32_t tq = tmem + hcol0 + (uint32_t)half * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
+      const uint32_t tq2 = tq + (16u << 16);
+      for (int b0 = 0; b0 < g.Bp; b0 += 4) {
+        uint32_t wv[4], wd[4], zv[4], zd[4];
+        const uint32_t cw = (uint32_t)b0;
+        tmem_ld_16x128b(tq + cw, wv[0], wv[1]);
+        tmem_ld_16x128b(tq2 + cw, wv[2], wv[3]);
+        tmem_ld_16x128b(tq + cw + g.Bp, wd[0], wd[1]);
+        tmem_ld_16x128b(tq2 + cw + g.Bp, wd[2], wd[3]);
+        tmem_ld_16x128b(tq + 2 * g.Bp + cw, zv[0], zv[1]);
+        tmem_ld_16x128b(tq2 + 2 * g.Bp + cw, zv[2], zv[3]);
+        tmem_ld_16x128b(tq + 3 * g.Bp + cw, zd[0], zd[1]);
+        tmem_ld_16x128b(tq2 + 3 * g.Bp + cw, zd[2], zd[3]);
+        tmem_wait_ld();
+        float lp[4], lm[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float C = fmaf(eps, __uint_as_float(zd[k]), __uint_as_float(wv[k])) + bo[k];
+          const float D = fmaf(eps, __uint_as_float(zv[k]), __uint_as_float(wd[k])) + dbo[k];
+          lp[k] = C + D;
+          lm[k] = C - D;
+        }
+        float mp = fmaxf(fmaxf(lp[0], lp[1]), fmaxf(lp[2], lp[3]));
+        float mm = fmaxf(fmaxf(lm[0], lm[1]), fmaxf(lm[2], lm[3]));
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          mp = fmaxf(mp, __shfl_xor_sync(0xffffffffu, mp, o));
+          mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
+        }
+        float sp = 0.f, sm_ = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          sp += __expf(lp[k] - mp);
+          sm_ += __expf(lm[k] - mm);
+        }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          sp += __shfl_xor_sync(0xffffffffu, sp, o);
+          sm_ += __shfl_xor_sync(0xffffffffu, sm_, o);
+        }
+        const int b = b0 + bq;
+        if (r4 == 0) {
+          red[((half * 4 + q4) * 2 + 0) * g.Bp + b] = make_float2(mp, sp);
+          red[((half * 4 + q4) * 2 + 1) * g.Bp + b] = make_float2(mm, sm_);
+        }
+        if (b < g.B) {
+          const int y = s.bytes[seq_offset(s, e, i, b) + t] - vq - r4;  // target of t - 1
+          if (y >= 0 && y < 32 && (y & 7) == 0) {
+            const int k = y >> 3;
+            ylog[b] = k == 0 ? lp[0] : k == 1 ? lp[1] : k == 2 ? lp[2] : lp[3];
+            ylog[g.Bp + b] = k == 0 ? lm[0] : k == 1 ? lm[1] : k == 2 ? lm[2] : lm[3];
+          }
+        }
+      }
+      __syncthreads();
+      if (tid < g.B) {
+        float nll[2];
+        for (int sg = 0; sg < 2; ++sg) {
+          float M = -INFINITY;
+          for (int h = 0; h < 8; ++h) M = fmaxf(M, red[(h * 2 + sg) * g.Bp + tid].x);
+          float S = 0.f;
+          for (int h = 0; h < 8; ++h) {
+            const float2 q = red[(h * 2 + sg) * g.Bp + tid];
+            S += q.y * __expf(q.x - M);
+          }
+          nll[sg] = M + logf(S) - ylog[sg * g.Bp + tid];
+        }
+        acc[tid] += (double)nll[0];
+        acc[g.Bp + tid] += (double)nll[1];
+        acc[2 * g.Bp + tid] += (double)(nll[0] - nll[1]);
+      }
+    }
+
+    if (t < g.T && ok && tile < g.MTg) {
+      // ---- gate epilogue of t: cells in registers, h of t into the operand
+      const uint32_t tq = tmem + gcol0 + (uint32_t)tile * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
+      const uint32_t tq2 = tq + (16u << 16);
+#pragma unroll
+      for (int c = 0; c < kResMaxBp / 8; ++c) {
+        const int b0 = 8 * c;
+        if (b0 >= g.Bp) break;
+        uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const uint32_t cw = (uint32_t)(b0 + 4 * h);
+          tmem_ld_16x128b(tq + cw, wv[h][0], wv[h][1]);
+          tmem_ld_16x128b(tq2 + cw, wv[h][2], wv[h][3]);
+          tmem_ld_16x128b(tq + cw + g.Bp, wd[h][0], wd[h][1]);
+          tmem_ld_16x128b(tq2 + cw + g.Bp, wd[h][2], wd[h][3]);
+          tmem_ld_16x128b(tq + 2 * g.Bp + cw, zv[h][0], zv[h][1]);
+          tmem_ld_16x128b(tq2 + 2 * g.Bp + cw, zv[h][2], zv[h][3]);
+          tmem_ld_16x128b(tq + 3 * g.Bp + cw, zd[h][0], zd[h][1]);
+          tmem_ld_16x128b(tq2 + 3 * g.Bp + cw, zd[h][2], zd[h][3]);
+        }
+        tmem_wait_ld();
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          float actp[4], actm[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float C = fmaf(eps, __uint_as_float(zd[h][k]), __uint_as_float(wv[h][k])) + bias[k];
+            const float D = fmaf(eps, __uint_as_float(zv[h][k]), __uint_as_float(wd[h][k])) + dbias[k];
+            if (k == 2) {
+              actp[k] = fmaf(sigm_res(2.f * (C + D)), 2.f, -1.f);
+              actm[k] = fmaf(sigm_res(2.f * (C - D)), 2.f, -1.f);
+            } else {
+              actp[k] = sigm_res(C + D);
+              actm[k] = sigm_res(C - D);
+            }
+          }
+          const float cp = fmaf(actp[1], cst[c][h][0], actp[0] * actp[2]);
+          const float cm = fmaf(actm[1], cst[c][h][1], actm[0] * actm[2]);
+          cst[c][h][0] = cp;
+          cst[c][h][1] = cm;
+          const float hp = actp[3] * fmaf(sigm_res(2.f * cp), 2.f, -1.f);
+          const float hm = actm[3] * fmaf(sigm_res(2.f * cm), 2.f, -1.f);
+          const int b = b0 + 4 * h + bq;
+          if (unit_ok && b < g.B) {
+            *reinterpret_cast<__half*>(smem + g.op + kmajor_offset(b, g.Ek + U, g.K)) =
+                __float2half_rn(0.5f * (hp + hm));
+            *reinterpret_cast<__half*>(smem + g.op + kmajor_offset(g.Bp + b, g.Ek + U, g.K)) =
+                __float2half_rn(0.5f * (hp - hm));
+          }
+        }
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+  }
+
+  // ---- losses and coefficient of the pair (fp64 sums, sequences in order)
+  if (tid == 0) {
+    double sp = 0.0, sm = 0.0, sd = 0.0;
+    for (int b = 0; b < g.B; ++b) {
+      sp += acc[b];
+      sm += acc[g.Bp + b];
+      sd += acc[2 * g.Bp + b];
+    }
+    const double inv = 1.0 / ((double)g.B * (double)g.T);
+    const double Lp = sp * inv, Lm = sm * inv, D = sd * inv;
+    const double c = (eps == 0.f) ? 0.0 : D / (2.0 * (double)eps);
+    const int64_t pair = blockIdx.x;
+    if (a.n_sign == 2) {
+      a.losses_out[pair * 2] = (float)Lp;
+      a.losses_out[pair * 2 + 1] = (float)Lm;
+    } else {
+      a.losses_out[pair] = (float)Lp;
+    }
+    if (a.coef_out) a.coef_out[pair] = (float)c;
+    if (a.coef_ws) a.coef_ws[pair] = (float)c;
+    if (!(isfinite(Lp) && isfinite(Lm) && isfinite(c))) atomicCAS(a.status, 0, kStatusNonFinite);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, g.tmem_cols);
+}
+
+}  // namespace
+
+bool res_supported(const Layout& lay, int B) {
+  if (B < 1 || B > kResMaxBp || lay.H > 64) return false;
+  const ResGeom g = make_res_geom(lay, B, 1);
+  return g.bytes <= kResMaxSmem;
+}
+
+cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, float* coef_out,
+                               float* coef_ws, int* status, cudaStream_t stream) {
+  ResArgs a;
+  a.sw = s;
+  a.n_sign = n_sign;
+  a.g = make_res_geom(s.lay, s.B, s.T);
+  a.losses_out = losses_out;
+  a.coef_out = coef_out;
+  a.coef_ws = coef_ws;
+  a.status = status;
+  cudaError_t e = cudaFuncSetAttribute(res_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)a.g.bytes);
+  if (e != cudaSuccess) return e;
+  trace_begin(SOMA_TRACE_GATE, stream);
+  res_kernel<<<s.n_experts * s.n_pert, kResThreads, a.g.bytes, stream>>>(a);
+  trace_end(SOMA_TRACE_GATE, stream);
+  return cudaGetLastError();
+}
+
+}  // namespace soma

@@ -47,6 +47,7 @@ size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 // up to 128 sequences run on the tensor cores (both signs always); larger
 // batches on the fp32 CUDA-core kernels.
 struct WsPlan {
+  bool res;  // the resident small-expert kernel: no scratch but the coefficients
   bool tc;
   TcGeom g;
   TcSizes z;
@@ -54,11 +55,17 @@ struct WsPlan {
   size_t hist, cst, nll, coef, total;
 };
 
-WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T) {
+WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T,
+                  bool allow_res = true) {
   WsPlan w;
   std::memset(&w, 0, sizeof(w));
   const Layout lay = make_layout(d.embed, d.hidden);
   w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
+  if (allow_res && res_supported(lay, B)) {
+    w.res = true;
+    w.total = w.coef;
+    return w;
+  }
   if (tc_supported(B)) {
     w.tc = true;
     w.g = make_tc_geom(lay, n_experts, n_pert, B, T);
@@ -190,7 +197,9 @@ static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, i
   s.step = step;
   float* coef_ws = coef_scratch(w, workspace);
   cudaError_t e;
-  if (w.tc) {
+  if (w.res) {
+    e = launch_forward_res(s, 2, losses_out, coef_out, coef_ws, status, st);
+  } else if (w.tc) {
     const TcBuffers tb = carve_tc(w, workspace);
     e = launch_forward_tc(s, w.g, tb, status, st);
     if (e == cudaSuccess)
@@ -303,7 +312,9 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
   s.seed = 0;
   s.step = 0;
   cudaError_t e;
-  if (w.tc) {
+  if (w.res) {
+    e = launch_forward_res(s, 1, loss_out, nullptr, nullptr, status, st);
+  } else if (w.tc) {
     const TcBuffers tb = carve_tc(w, workspace);
     e = launch_forward_tc(s, w.g, tb, status, st);
     if (e == cudaSuccess)
@@ -428,7 +439,8 @@ bool plan_mixture(const soma_dims& d, int N, const int32_t* routes, int R, int k
       m.gather_h[(size_t)routes[(size_t)r * k + j] * m.b_max + m.slot_h[(size_t)r * k + j]] = r;
   m.Bc = m.b_max < kMixChunk ? m.b_max : kMixChunk;
   m.chunks = (m.b_max + m.Bc - 1) / m.Bc;
-  m.sweep = plan_sweep(d, N, 1, 1, m.Bc, T);
+  // the mixture reads per-target NLL, which only the per-timestep kernels keep
+  m.sweep = plan_sweep(d, N, 1, 1, m.Bc, T, false);
   m.gather = round_up((size_t)N * m.b_max * sizeof(int32_t));
   m.route = round_up((size_t)R * k * sizeof(int32_t));
   m.slot = m.route;

@@ -88,6 +88,13 @@ struct AdamArgs {
   float lr, b1, b2, delta, wd, inv_bc1, inv_bc2;
 };
 
+// Small experts with the whole recurrence resident in one CTA (resident.cu).
+bool res_supported(const Layout& lay, int B);
+// n_sign = 2: losses_out [N][n][2] (L+, L-) and the coefficients; n_sign = 1
+// (eps = 0, n = 1): losses_out [N] = L(theta).
+cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, float* coef_out,
+                               float* coef_ws, int* status, cudaStream_t stream);
+
 // Routed inference (mixture.cu).
 cudaError_t launch_gather_requests(const uint8_t* requests, const int32_t* gather, int N,
                                    int b_max, int b0, int Bc, int T1, uint8_t* grouped,
