@@ -16,7 +16,8 @@
 //          vocabulary halves, target logit, NLL summed in fp64;
 //   gate epilogue of t: gates and cells, h of t into the operand;
 //   the embedding part of the operand of t + 1.
-// The shape limits (H <= 64, B <= 32, the tiles within shared memory) are
+// The shape limits (H <= 64, B <= 32, 2 Bp Ek / 8 <= 256 operand chunks, the
+// tiles within shared memory) are
 // checked by res_supported(); larger experts use the persistent kernel.
 #include <cuda_fp16.h>
 
@@ -31,7 +32,8 @@ using namespace tc;
 
 namespace {
 
-constexpr int kResThreads = 256;  // 8 warps: two M tiles x four TMEM lane quarters
+constexpr int kResThreads = 512;  // 16 warps: (two M tiles x four TMEM lane quarters) x two
+                                  // halves of the sequences
 constexpr int kResMaxBp = 32;
 constexpr size_t kResMaxSmem = 220 * 1024;
 constexpr uint32_t kLboRes = 128;  // bytes between core matrices along K
@@ -40,7 +42,7 @@ __device__ __forceinline__ float sigm_res(float x) { return __fdividef(1.0f, 1.0
 
 struct ResGeom {
   int E, H, Ek, Hk, K, MTg, Bp, B, T;
-  uint32_t wg, zg, wo, zo, op, red, ylog, acc, ctl, bytes;  // shared-memory offsets
+  uint32_t wg, zg, wo, zo, op, emb, dx, red, ylog, acc, ctl, bytes;  // shared-memory offsets
   uint32_t tmem_cols;
 };
 
@@ -64,6 +66,8 @@ ResGeom make_res_geom(const Layout& lay, int B, int T) {
   r.wo = o; o = res_align(o + 2 * head_tile);
   r.zo = o; o = res_align(o + 2 * head_tile);
   r.op = o; o = res_align(o + 2u * r.Bp * r.K * 2);
+  r.emb = o; o += 256u * r.Ek * 2;   // fp16 Emb rows [V][Ek]
+  r.dx = o; o += 256u * r.Ek * 2;    // fp16 eps z of the Emb rows
   r.red = o; o += 2u * 4 * 2 * r.Bp * sizeof(float2);  // [half][quarter][sign][Bp]
   r.ylog = o; o += 2u * r.Bp * sizeof(float);          // [sign][Bp]
   o = (o + 7u) & ~7u;
@@ -106,14 +110,16 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
-  uint64_t* mma_bar = reinterpret_cast<uint64_t*>(smem + g.ctl);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 8);
+  uint64_t* gate_bar = reinterpret_cast<uint64_t*>(smem + g.ctl);
+  uint64_t* head_bar = reinterpret_cast<uint64_t*>(smem + g.ctl + 8);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 16);
   float2* red = reinterpret_cast<float2*>(smem + g.red);
   float* ylog = reinterpret_cast<float*>(smem + g.ylog);
   double* acc = reinterpret_cast<double*>(smem + g.acc);
 
   if (tid == 0) {
-    mbar_init(mma_bar, 1);
+    mbar_init(gate_bar, 1);
+    mbar_init(head_bar, 1);
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(tmem_slot, g.tmem_cols);
@@ -170,12 +176,31 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   }
   for (int c = tid; c < 2 * g.Bp * g.K / 8; c += kResThreads)
     reinterpret_cast<uint4*>(smem + g.op)[c] = make_uint4(0u, 0u, 0u, 0u);
+  // the embedding table and its eps z, so that the operand of a timestep is
+  // gathered from shared memory
+  for (int c = tid; c < 256 * (g.Ek / 8); c += kResThreads) {
+    const int v = c / (g.Ek / 8), k0 = 8 * (c % (g.Ek / 8));
+    const int64_t p0 = L.emb + (int64_t)v * g.E + k0;
+    const int kmax = min(8, g.E - k0);
+    ProbeBits zb = {0u, 0u};
+    if (do_z && kmax > 0) zb = probe_bits(pk, p0, s.sparse);
+    __align__(16) __half x[8], d[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const bool ok = j < kmax;
+      x[j] = __float2half_rn(ok ? th[p0 + j] : 0.f);
+      d[j] = __float2half_rn(ok ? eps_z((zb.neg >> j) & 1u, (zb.act >> j) & 1u, eps) : 0.f);
+    }
+    reinterpret_cast<uint4*>(smem + g.emb)[c] = *reinterpret_cast<const uint4*>(x);
+    reinterpret_cast<uint4*>(smem + g.dx)[c] = *reinterpret_cast<const uint4*>(d);
+  }
   for (int c = tid; c < 3 * g.Bp; c += kResThreads) acc[c] = 0.0;
 
   // ---- per-thread constants of the epilogues
-  // gate: warp w runs tile w / 4, TMEM lane quarter w % 4; thread l owns unit
-  // 8 (w % 4) + l / 4 of that tile and sequences b0 + l % 4, b0 + 4 + l % 4
-  const int q4 = warp & 3, tile = warp >> 2;
+  // gate: warp w runs tile (w / 4) % 2, TMEM lane quarter w % 4, and the
+  // 8-sequence chunks c with c % 2 == w / 8; thread l owns unit 8 (w % 4) +
+  // l / 4 of that tile and sequences 8c + l % 4, 8c + 4 + l % 4
+  const int q4 = warp & 3, tile = (warp >> 2) & 1, sp = warp >> 3;
   const int u8 = lane >> 2, bq = lane & 3;
   const int U = 32 * tile + 8 * q4 + u8;
   const bool unit_ok = tile < g.MTg && U < g.H;
@@ -195,9 +220,10 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
 #pragma unroll
   for (int c = 0; c < kResMaxBp / 8; ++c)
     cst[c][0][0] = cst[c][0][1] = cst[c][1][0] = cst[c][1][1] = 0.f;
-  // head: warp w runs vocabulary half w / 4, quarter w % 4; thread l holds
-  // rows l / 4 + 8 k (k = 0..3) of the quarter
-  const int half = warp >> 2, r4 = lane >> 2;
+  // head: warp w runs vocabulary half (w / 4) % 2, quarter w % 4, and the
+  // 4-sequence groups 4 (w / 8) + 8 j; thread l holds rows l / 4 + 8 k
+  // (k = 0..3) of the quarter
+  const int half = (warp >> 2) & 1, r4 = lane >> 2;
   const int vq = 128 * half + 32 * q4;
   float bo[4], dbo[4];
 #pragma unroll
@@ -217,35 +243,25 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const uint32_t tmem = *tmem_slot;
   const uint32_t gcol0 = 0, hcol0 = (uint32_t)g.MTg * 4 * g.Bp;
   bool ok = true;
+  // the operand chunk this thread gathers every timestep (one row, 8 columns)
+  const int xc = tid < 2 * g.Bp * (g.Ek / 8) ? tid : -1;
+  const int xrow = xc / (g.Ek / 8), xk0 = 8 * (xc % (g.Ek / 8));
+  const bool x_delta = xrow >= g.Bp;
+  const int xb = x_delta ? xrow - g.Bp : xrow;
+  int ynext = (xc >= 0 && xb < g.B) ? s.bytes[seq_offset(s, e, i, xb)] : 0;
 
   for (int t = 0; t <= g.T && ok; ++t) {
-    // embedding part of the operand of timestep t: rows [vbar (Bp) | dv (Bp)]
-    if (t < g.T) {
-      for (int c = tid; c < 2 * g.Bp * (g.Ek / 8); c += kResThreads) {
-        const int row = c / (g.Ek / 8), k0 = 8 * (c % (g.Ek / 8));
-        const bool delta = row >= g.Bp;
-        const int b = delta ? row - g.Bp : row;
-        __align__(16) __half v[8];
-        if (b < g.B) {
-          const int y = s.bytes[seq_offset(s, e, i, b) + t];
-          const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
-          const int kmax = min(8, g.E - k0);
-          ProbeBits zb = {0u, 0u};
-          if (delta && do_z && kmax > 0) zb = probe_bits(pk, p0, s.sparse);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float x = 0.f;
-            if (j < kmax)
-              x = delta ? eps_z((zb.neg >> j) & 1u, (zb.act >> j) & 1u, eps) : th[p0 + j];
-            v[j] = __float2half_rn(x);
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) v[j] = __float2half_rn(0.f);
-        }
-        *reinterpret_cast<uint4*>(smem + g.op + kmajor_offset(row, k0, g.K)) =
-            *reinterpret_cast<const uint4*>(v);
+    // embedding part of the operand of timestep t: rows [vbar (Bp) | dv (Bp)],
+    // 16-byte chunks of the Emb / eps z tables; the next byte is fetched
+    // while this timestep runs
+    if (t < g.T && xc >= 0) {
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (xb < g.B) {
+        const uint4* tab = reinterpret_cast<const uint4*>(smem + (x_delta ? g.dx : g.emb));
+        v = tab[ynext * (g.Ek / 8) + xk0 / 8];
       }
+      *reinterpret_cast<uint4*>(smem + g.op + kmajor_offset(xrow, xk0, g.K)) = v;
+      if (xb < g.B && t + 1 < g.T) ynext = s.bytes[seq_offset(s, e, i, xb) + t + 1];
     }
     fence_async_smem();
     tc_fence_before();
@@ -269,6 +285,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
                        bdesc, idesc, k16 > 0 ? 1u : 0u);
           }
         }
+        mma_commit(head_bar);
       }
       if (t < g.T) {  // gate of t
         for (int m = 0; m < g.MTg; ++m) {
@@ -282,22 +299,25 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
                        bdesc, idesc, k16 > 0 ? 1u : 0u);
           }
         }
+        mma_commit(gate_bar);
       }
-      mma_commit(mma_bar);
     }
     __syncwarp();
-    bool got = mbar_wait(mma_bar, (uint32_t)t & 1u);
-    if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
-    // one decision for the whole CTA: a timed-out wait ends the recurrence
-    // for every thread at the same barrier
-    ok = __syncthreads_and(got) != 0;
-    tc_fence_after();
 
+    if (t >= 1) {
+      // the head MMAs of t - 1 were issued first: their epilogue overlaps the
+      // gate MMAs of t.  One decision for the whole CTA: a timed-out wait
+      // ends the recurrence for every thread at the same barrier.
+      const bool got = mbar_wait(head_bar, (uint32_t)(t - 1) & 1u);
+      if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
+      ok = __syncthreads_and(got) != 0;
+      tc_fence_after();
+    }
     if (t >= 1 && ok) {
       // ---- head epilogue of t - 1
       const uint32_t tq = tmem + hcol0 + (uint32_t)half * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
       const uint32_t tq2 = tq + (16u << 16);
-      for (int b0 = 0; b0 < g.Bp; b0 += 4) {
+      for (int b0 = 4 * sp; b0 < g.Bp; b0 += 8) {
         uint32_t wv[4], wd[4], zv[4], zd[4];
         const uint32_t cw = (uint32_t)b0;
         tmem_ld_16x128b(tq + cw, wv[0], wv[1]);
@@ -368,6 +388,12 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       }
     }
 
+    if (t < g.T && ok) {
+      const bool got = mbar_wait(gate_bar, (uint32_t)t & 1u);
+      if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
+      ok = __syncthreads_and(got) != 0;
+      tc_fence_after();
+    }
     if (t < g.T && ok && tile < g.MTg) {
       // ---- gate epilogue of t: cells in registers, h of t into the operand
       const uint32_t tq = tmem + gcol0 + (uint32_t)tile * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
@@ -376,6 +402,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       for (int c = 0; c < kResMaxBp / 8; ++c) {
         const int b0 = 8 * c;
         if (b0 >= g.Bp) break;
+        if ((c & 1) != sp) continue;
         uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -457,7 +484,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
 bool res_supported(const Layout& lay, int B) {
   if (B < 1 || B > kResMaxBp || lay.H > 64) return false;
   const ResGeom g = make_res_geom(lay, B, 1);
-  return g.bytes <= kResMaxSmem;
+  // one thread gathers each 8-column chunk of the embedding operand
+  return g.bytes <= kResMaxSmem && 2 * g.Bp * (g.Ek / 8) <= kResThreads;
 }
 
 cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, float* coef_out,
