@@ -32,8 +32,10 @@ using namespace tc;
 
 namespace {
 
-constexpr int kResThreads = 512;  // 16 warps: (two M tiles x four TMEM lane quarters) x two
-                                  // halves of the sequences
+constexpr int kResEpiWarps = 16;  // (two M tiles x four TMEM lane quarters) x two halves
+                                   // of the sequences
+constexpr int kResMmaWarp = kResEpiWarps;  // issues the MMAs and takes no epilogue work
+constexpr int kResThreads = (kResEpiWarps + 1) * 32;
 constexpr int kResMaxBp = 32;
 constexpr size_t kResMaxSmem = 220 * 1024;
 constexpr uint32_t kLboRes = 128;  // bytes between core matrices along K
@@ -242,9 +244,22 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t gcol0 = 0, hcol0 = (uint32_t)g.MTg * 4 * g.Bp;
+  // MMA descriptors as 32-bit words: the low word holds the start address in
+  // 16-byte units, so a step along K (256 bytes) or to the next tile is an
+  // addition; gate tiles and the operand share their high word (SBO = 16 K)
+  const uint32_t n2 = (uint32_t)(2 * g.Bp);
+  const uint32_t idesc = idesc_f16_f32(128, 2 * g.Bp);
+  const uint64_t dg = smem_desc(smem_u32(smem + g.wg), kLboRes, (uint32_t)g.K * 16);
+  const uint64_t dh = smem_desc(smem_u32(smem + g.wo), kLboRes, (uint32_t)g.Hk * 16);
+  const uint32_t ghi = (uint32_t)(dg >> 32), wg_lo = (uint32_t)dg;
+  const uint32_t hhi = (uint32_t)(dh >> 32), wo_lo = (uint32_t)dh;
+  const uint32_t zg_lo = wg_lo + ((g.zg - g.wg) >> 4), op_lo = wg_lo + ((g.op - g.wg) >> 4);
+  const uint32_t oph_lo = op_lo + (uint32_t)g.Ek;  // the h part: Ek / 8 core matrices further
+  const uint32_t zo_lo = wo_lo + ((g.zo - g.wo) >> 4);
+  const uint32_t gstep = 16u * g.K, hstep = 16u * g.Hk;  // one 128-row tile, in 16-byte units
   bool ok = true;
   // the operand chunk this thread gathers every timestep (one row, 8 columns)
-  const int xc = tid < 2 * g.Bp * (g.Ek / 8) ? tid : -1;
+  const int xc = (warp < kResEpiWarps && tid < 2 * g.Bp * (g.Ek / 8)) ? tid : -1;
   const int xrow = xc / (g.Ek / 8), xk0 = 8 * (xc % (g.Ek / 8));
   const bool x_delta = xrow >= g.Bp;
   const int xb = x_delta ? xrow - g.Bp : xrow;
@@ -266,37 +281,30 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
     fence_async_smem();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0) {
+    if (warp == kResMmaWarp && lane == 0) {
       tc_fence_after();
-      const uint32_t n2 = (uint32_t)(2 * g.Bp);
-      const uint32_t idesc = idesc_f16_f32(128, 2 * g.Bp);
-      const uint32_t sbase = smem_u32(smem);
-      const uint32_t gsbo = (uint32_t)g.K * 16, hsbo = (uint32_t)g.Hk * 16;
-      if (t >= 1) {  // head of t - 1: h part of the operand
+      if (t >= 1) {  // head of t - 1: the h part of the operand
+#pragma unroll 1
         for (int h = 0; h < 2; ++h) {
           const uint32_t d = tmem + hcol0 + (uint32_t)h * 2 * n2;
+          const uint32_t wlo = wo_lo + (uint32_t)h * hstep, zlo = zo_lo + (uint32_t)h * hstep;
           for (int k16 = 0; k16 < g.Hk / 16; ++k16) {
-            const uint32_t ko = (uint32_t)k16 * 256;
-            const uint64_t bdesc =
-                smem_desc(sbase + g.op + (uint32_t)(g.Ek / 8) * 128 + ko, kLboRes, gsbo);
-            mma_f16_ss(d, smem_desc(sbase + g.wo + h * (128u * g.Hk * 2) + ko, kLboRes, hsbo),
-                       bdesc, idesc, k16 > 0 ? 1u : 0u);
-            mma_f16_ss(d + n2, smem_desc(sbase + g.zo + h * (128u * g.Hk * 2) + ko, kLboRes, hsbo),
-                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+            const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
+            mma_f16_ss_lohi(d, wlo + ko, hhi, oph_lo + ko, ghi, idesc, acc_flag);
+            mma_f16_ss_lohi(d + n2, zlo + ko, hhi, oph_lo + ko, ghi, idesc, acc_flag);
           }
         }
         mma_commit(head_bar);
       }
       if (t < g.T) {  // gate of t
+#pragma unroll 1
         for (int m = 0; m < g.MTg; ++m) {
           const uint32_t d = tmem + gcol0 + (uint32_t)m * 2 * n2;
+          const uint32_t wlo = wg_lo + (uint32_t)m * gstep, zlo = zg_lo + (uint32_t)m * gstep;
           for (int k16 = 0; k16 < g.K / 16; ++k16) {
-            const uint32_t ko = (uint32_t)k16 * 256;
-            const uint64_t bdesc = smem_desc(sbase + g.op + ko, kLboRes, gsbo);
-            mma_f16_ss(d, smem_desc(sbase + g.wg + m * (128u * g.K * 2) + ko, kLboRes, gsbo),
-                       bdesc, idesc, k16 > 0 ? 1u : 0u);
-            mma_f16_ss(d + n2, smem_desc(sbase + g.zg + m * (128u * g.K * 2) + ko, kLboRes, gsbo),
-                       bdesc, idesc, k16 > 0 ? 1u : 0u);
+            const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
+            mma_f16_ss_lohi(d, wlo + ko, ghi, op_lo + ko, ghi, idesc, acc_flag);
+            mma_f16_ss_lohi(d + n2, zlo + ko, ghi, op_lo + ko, ghi, idesc, acc_flag);
           }
         }
         mma_commit(gate_bar);
@@ -304,16 +312,15 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
     }
     __syncwarp();
 
+    // a failed wait marks this thread; the decision is taken for the whole
+    // CTA at the barrier that ends the timestep, so that no wait is followed
+    // by a CTA barrier (the issuing thread's warp would hold every warp back)
+    bool fine = true;
     if (t >= 1) {
-      // the head MMAs of t - 1 were issued first: their epilogue overlaps the
-      // gate MMAs of t.  One decision for the whole CTA: a timed-out wait
-      // ends the recurrence for every thread at the same barrier.
-      const bool got = mbar_wait(head_bar, (uint32_t)(t - 1) & 1u);
-      if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
-      ok = __syncthreads_and(got) != 0;
+      fine = mbar_wait(head_bar, (uint32_t)(t - 1) & 1u) && fine;
       tc_fence_after();
     }
-    if (t >= 1 && ok) {
+    if (t >= 1 && ok && warp < kResEpiWarps) {
       // ---- head epilogue of t - 1
       const uint32_t tq = tmem + hcol0 + (uint32_t)half * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
       const uint32_t tq2 = tq + (16u << 16);
@@ -369,7 +376,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
           }
         }
       }
-      __syncthreads();
+      // the epilogue warps only: the MMA warp may still be issuing the gate
+      asm volatile("bar.sync 1, %0;" ::"n"(kResEpiWarps * 32) : "memory");
       if (tid < g.B) {
         float nll[2];
         for (int sg = 0; sg < 2; ++sg) {
@@ -388,13 +396,11 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       }
     }
 
-    if (t < g.T && ok) {
-      const bool got = mbar_wait(gate_bar, (uint32_t)t & 1u);
-      if (!got && lane == 0) atomicCAS(a.status, 0, kStatusTimeout);
-      ok = __syncthreads_and(got) != 0;
+    if (t < g.T) {
+      fine = mbar_wait(gate_bar, (uint32_t)t & 1u) && fine;
       tc_fence_after();
     }
-    if (t < g.T && ok && tile < g.MTg) {
+    if (t < g.T && ok && warp < kResEpiWarps && tile < g.MTg) {
       // ---- gate epilogue of t: cells in registers, h of t into the operand
       const uint32_t tq = tmem + gcol0 + (uint32_t)tile * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
       const uint32_t tq2 = tq + (16u << 16);
@@ -448,8 +454,9 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
         }
       }
     }
+    if (!fine) atomicCAS(a.status, 0, kStatusTimeout);
     tc_fence_before();
-    __syncthreads();
+    ok = (__syncthreads_and(fine) != 0) && ok;
   }
 
   // ---- losses and coefficient of the pair (fp64 sums, sequences in order)
@@ -485,7 +492,7 @@ bool res_supported(const Layout& lay, int B) {
   if (B < 1 || B > kResMaxBp || lay.H > 64) return false;
   const ResGeom g = make_res_geom(lay, B, 1);
   // one thread gathers each 8-column chunk of the embedding operand
-  return g.bytes <= kResMaxSmem && 2 * g.Bp * (g.Ek / 8) <= kResThreads;
+  return g.bytes <= kResMaxSmem && 2 * g.Bp * (g.Ek / 8) <= kResEpiWarps * 32;
 }
 
 cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, float* coef_out,
