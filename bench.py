@@ -102,13 +102,16 @@ def tokens_per_step(c):
 DTYPE = "f16/f32"
 
 
-def gate_kernel_name(B):
+def gate_kernel_name(B, resident):
+    if resident:
+        return ("res_kernel (tcgen05, the whole recurrence of a probe pair resident in one CTA: "
+                "gate GEMM + cell + head + loss; its time includes the head)")
     if B <= 64:
         return "tc_persistent_kernel<gate> (tcgen05 gate GEMM + fused cell)"
     return "gate_step_kernel (fp32 CUDA-core gate GEMM + cell)"
 
 
-def gate_flops_per_launch(c):
+def gate_flops_per_timestep(c):
     # one launch = one timestep of every (expert, probe, sign) lane:
     # [B, E+H] x [E+H, 4H] per lane, 2 flops per multiply-add
     return c["n_experts"] * c["n_pert"] * 2 * c["batch"] * 8 * c["H"] * (c["E"] + c["H"])
@@ -360,7 +363,12 @@ def our_arm(args):
     gate_ms, gate_n = traced["gate"]
     peaks, peak_src = measured_peaks()
     peak = peaks["bf16_tflops_sustained"]
-    achieved = gate_flops_per_launch(c) / (gate_ms / gate_n / 1e3) / 1e12 if gate_n else None
+    # all gate work of the timed region over the gate kernel's traced time:
+    # K steps x A estimates x T timesteps, whether a launch covers one
+    # timestep (persistent kernel) or all of them (resident kernel)
+    one_launch = traced["head"][1] == 0 and gate_n == K * A  # the resident kernel
+    gate_flops_total = gate_flops_per_timestep(c) * T * K * A
+    achieved = gate_flops_total / (gate_ms / 1e3) / 1e12 if gate_n else None
     tr = TRAFFIC.get(args.config)
     traffic = (tr["bytes_per_launch"]
                if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
@@ -385,11 +393,12 @@ def our_arm(args):
                            "replica(s), no collective",
         },
         "roofline": {
-            "bound": "tensor", "kernel": gate_kernel_name(B),
+            "bound": "tensor", "kernel": gate_kernel_name(B, one_launch),
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": (achieved / peak) if achieved else None, "traffic": traffic,
             "peak_source": f"{peak_src} bf16 dense sustained (MEASURED_PEAKS.json)",
-            "flops_per_launch": gate_flops_per_launch(c), "launches": gate_n,
+            "flops_per_launch": gate_flops_total / gate_n if gate_n else None,
+            "launches": gate_n,
             "kernel_ms_per_launch": gate_ms / gate_n if gate_n else None,
             "share_of_step": gate_ms / ms if ms else None,
         },
