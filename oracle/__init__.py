@@ -35,6 +35,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "soma_oracle.c")
+_SRCS = [_SRC, os.path.join(_HERE, "body_oracle.c")]
 _LIB_PATH = os.path.join(_HERE, "liboracle_soma.so")
 _lock = threading.Lock()
 _lib = None
@@ -43,13 +44,14 @@ V = 256
 
 
 def build(force: bool = False) -> str:
-    """Compile soma_oracle.c into liboracle_soma.so with gcc (-fopenmp)."""
+    """Compile soma_oracle.c and body_oracle.c into liboracle_soma.so with gcc
+    (-fopenmp)."""
     if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB_PATH) >= os.path.getmtime(f) for f in _SRCS)):
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
-           "-fno-fast-math", "-o", tmp, _SRC, "-lm"]
+           "-fno-fast-math", "-o", tmp, *_SRCS, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
@@ -121,6 +123,31 @@ def _load():
         lib.oracle_bptt_grad.argtypes = [c_dp, ctypes.c_int, ctypes.c_int, c_u8p, ctypes.c_int,
                                          ctypes.c_int, c_dp]
         lib.oracle_bptt_grad.restype = ctypes.c_double
+        c_i32p = ctypes.POINTER(ctypes.c_int32)
+        c_i = ctypes.c_int
+        lib.oracle_body_param_count.argtypes = [c_i, c_i]
+        lib.oracle_body_param_count.restype = ctypes.c_int64
+        lib.oracle_body_gain_offset.argtypes = [c_i, c_i]
+        lib.oracle_body_gain_offset.restype = ctypes.c_int64
+        lib.oracle_body_probe.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32,
+                                          ctypes.c_uint32, c_i, c_i, c_i, ctypes.c_int64,
+                                          ctypes.c_int64, ctypes.POINTER(ctypes.c_int8)]
+        lib.oracle_body_probe.restype = c_i
+        lib.oracle_body_loss.argtypes = [c_dp, c_i, c_i, c_dp, c_u8p, c_i, c_i, c_dp, c_i]
+        lib.oracle_body_loss.restype = ctypes.c_double
+        lib.oracle_body_spsa_losses.argtypes = [c_dp, c_i, c_i, c_i, c_i, c_dp, ctypes.c_double,
+                                                c_i, ctypes.c_uint64, ctypes.c_uint64, c_u8p,
+                                                c_i, c_i, c_i32p, c_i, c_dp, c_dp, c_i]
+        lib.oracle_body_spsa_losses.restype = c_i
+        lib.oracle_body_spsa_update.argtypes = [c_dp, c_i, c_i, c_i, c_i, c_i, ctypes.c_double,
+                                                ctypes.c_uint64, ctypes.c_uint64, c_dp, c_dp]
+        lib.oracle_body_spsa_update.restype = c_i
+        lib.oracle_body_adam_update.argtypes = [c_dp, c_dp, c_dp, c_i, c_i, c_i, c_i, c_i,
+                                                ctypes.c_uint64, ctypes.POINTER(ctypes.c_uint64),
+                                                c_i, c_dp, ctypes.c_double, ctypes.c_double,
+                                                ctypes.c_double, ctypes.c_double,
+                                                ctypes.c_double, c_i, c_dp, c_dp, c_dp]
+        lib.oracle_body_adam_update.restype = c_i
         _lib = lib
         return lib
 
@@ -302,3 +329,112 @@ def bptt_grad(theta, E: int, H: int, bytes_):
     m = _load().oracle_bptt_grad(_ptr(th, ctypes.c_double), E, H, _ptr(bx, ctypes.c_uint8), B, T,
                                  _ptr(g, ctypes.c_double))
     return m, g
+
+
+# ---------------------------------------------------------------------------
+# The paper's two-block expert body (body_oracle.c): D pre-norm residual
+# blocks of width d (bias-free LSTM, then a GELU MLP of width 4d), gain-only
+# LayerNorm, and a frozen tied head E [V, d] shared by every expert.
+# Probe kinds: "dense" on every coordinate; "sparse" is the paper's training
+# law (App. E): gains dense, every other coordinate sparse.
+# ---------------------------------------------------------------------------
+
+def body_param_count(d: int, D: int = 2) -> int:
+    return int(_load().oracle_body_param_count(d, D))
+
+
+def body_gain_offset(d: int, D: int = 2) -> int:
+    return int(_load().oracle_body_gain_offset(d, D))
+
+
+def body_probe(seed: int, step: int, expert: int, probe_index: int, d: int, D: int, p0: int,
+               count: int, kind: str = "sparse") -> np.ndarray:
+    """Body probe entries z[p0 : p0+count] (int8)."""
+    z = np.zeros(count, dtype=np.int8)
+    rc = _load().oracle_body_probe(seed, step, expert, probe_index, PROBE_KINDS[kind], d, D, p0,
+                                   count, _ptr(z, ctypes.c_int8))
+    if rc != 0:
+        raise RuntimeError(f"oracle_body_probe failed ({rc})")
+    return z
+
+
+def body_loss(theta, d: int, D: int, head, bytes_, n_threads: int = 0,
+              per_token: bool = False):
+    """Mean next-byte cross entropy of ONE expert body: theta [P], head
+    [V, d], bytes_ [B, T+1].  Returns the mean, or (mean, nll [B, T])."""
+    th = _f64(theta).reshape(-1)
+    hd = _f64(head)
+    assert th.size == body_param_count(d, D) and hd.shape == (V, d)
+    bx = _u8(bytes_)
+    B, T = bx.shape[0], bx.shape[1] - 1
+    nll = np.zeros((B, T), dtype=np.float64) if per_token else None
+    m = _load().oracle_body_loss(_ptr(th, ctypes.c_double), d, D, _ptr(hd, ctypes.c_double),
+                                 _ptr(bx, ctypes.c_uint8), B, T,
+                                 _ptr(nll, ctypes.c_double) if per_token else None, n_threads)
+    return (m, nll) if per_token else m
+
+
+def body_spsa_losses(theta, d: int, D: int, head, eps: float, seed: int, step: int, bytes_,
+                     probes=None, n_pert: int | None = None, kind: str = "sparse",
+                     first_expert: int = 0, n_threads: int = 0):
+    """Antithetic losses and coefficients of the selected probes of N expert
+    bodies: theta [N, P], bytes_ [N, B, T+1].  Returns (L [N, n_sel, 2],
+    coef [N, n_sel])."""
+    th = _f64(theta)
+    N = th.shape[0]
+    hd = _f64(head)
+    bx = _u8(bytes_)
+    assert bx.shape[0] == N and hd.shape == (V, d)
+    B, T = bx.shape[1], bx.shape[2] - 1
+    if probes is None:
+        probes = range(n_pert)
+    sel = np.ascontiguousarray(list(probes), dtype=np.int32)
+    L = np.zeros((N, sel.size, 2), dtype=np.float64)
+    coef = np.zeros((N, sel.size), dtype=np.float64)
+    rc = _load().oracle_body_spsa_losses(_ptr(th, ctypes.c_double), N, first_expert, d, D,
+                                         _ptr(hd, ctypes.c_double), float(eps),
+                                         PROBE_KINDS[kind], seed, step, _ptr(bx, ctypes.c_uint8),
+                                         B, T, _ptr(sel, ctypes.c_int32), sel.size,
+                                         _ptr(L, ctypes.c_double), _ptr(coef, ctypes.c_double),
+                                         n_threads)
+    if rc != 0:
+        raise RuntimeError(f"oracle_body_spsa_losses failed ({rc})")
+    return L, coef
+
+
+def body_spsa_update(theta, d: int, D: int, lr: float, seed: int, step: int, coef,
+                     kind: str = "sparse") -> np.ndarray:
+    """theta - lr (1/n_pert) sum_i coef[e, i] z_{e,i}, fp64 [N, P]."""
+    th = _f64(theta)
+    N = th.shape[0]
+    cf = np.ascontiguousarray(coef, dtype=np.float64)
+    out = np.zeros_like(th)
+    rc = _load().oracle_body_spsa_update(_ptr(th, ctypes.c_double), N, d, D, cf.shape[1],
+                                         PROBE_KINDS[kind], float(lr), seed, step,
+                                         _ptr(cf, ctypes.c_double), _ptr(out, ctypes.c_double))
+    if rc != 0:
+        raise RuntimeError(f"oracle_body_spsa_update failed ({rc})")
+    return out
+
+
+def body_adam_update(theta, m, v, d: int, D: int, seed: int, steps, coef, lr: float,
+                     beta1: float, beta2: float, delta: float, wd: float, t: int,
+                     kind: str = "sparse"):
+    """Eq. localspsa on the body coordinates: (theta', m', v') in fp64."""
+    th, mm, vv = _f64(theta), _f64(m), _f64(v)
+    N = th.shape[0]
+    cf = np.ascontiguousarray(coef, dtype=np.float64)
+    A, n_pert = cf.shape[0], cf.shape[2]
+    st = np.ascontiguousarray(steps, dtype=np.uint64)
+    assert st.size == A and cf.shape[1] == N
+    to, mo, vo = np.zeros_like(th), np.zeros_like(th), np.zeros_like(th)
+    rc = _load().oracle_body_adam_update(_ptr(th, ctypes.c_double), _ptr(mm, ctypes.c_double),
+                                         _ptr(vv, ctypes.c_double), N, d, D, n_pert,
+                                         PROBE_KINDS[kind], seed, _ptr(st, ctypes.c_uint64), A,
+                                         _ptr(cf, ctypes.c_double), float(lr), float(beta1),
+                                         float(beta2), float(delta), float(wd), int(t),
+                                         _ptr(to, ctypes.c_double), _ptr(mo, ctypes.c_double),
+                                         _ptr(vo, ctypes.c_double))
+    if rc != 0:
+        raise RuntimeError(f"oracle_body_adam_update failed ({rc})")
+    return to, mo, vo

@@ -164,3 +164,79 @@ def config_batch(name: str, seed: int = 0, step: int = 0, **overrides) -> np.nda
 def config_params(name: str, seed: int = 0, **overrides) -> np.ndarray:
     c = dict(CONFIGS[name], **overrides)
     return init_params(c["n_experts"], c["E"], c["H"], seed, c["init_std"])
+
+
+# ---------------------------------------------------------------------------
+# The paper's expert body (Sec. "Model size"): D pre-norm residual blocks of
+# width d, a bias-free LSTM and a GELU MLP of width 4d each, gain-only
+# LayerNorm, and one frozen tied head E [V, d] shared by every expert.
+# ---------------------------------------------------------------------------
+
+def body_param_count(d: int, D: int = 2) -> int:
+    """M_body = 16 D d^2 + (2D + 1) d body parameters of one expert."""
+    return 16 * D * d * d + (2 * D + 1) * d
+
+
+def body_offsets(d: int, D: int = 2) -> dict:
+    """Offsets inside one body's flat vector: per block k, W_ih [4d, d],
+    W_hh [4d, d], W_1 [4d, d], W_2 [d, 4d]; then per block the gains ga, gb
+    [d]; then the final gain gf [d]."""
+    q = d * d
+    o = {}
+    for k in range(D):
+        base = 16 * q * k
+        o[f"w_ih{k}"] = base
+        o[f"w_hh{k}"] = base + 4 * q
+        o[f"w1{k}"] = base + 8 * q
+        o[f"w2{k}"] = base + 12 * q
+    g0 = 16 * q * D
+    for k in range(D):
+        o[f"ga{k}"] = g0 + 2 * d * k
+        o[f"gb{k}"] = g0 + 2 * d * k + d
+    o["gf"] = g0 + 2 * d * D
+    o["gains"] = g0
+    o["end"] = o["gf"] + d
+    return o
+
+
+def init_body(n_experts: int, d: int, D: int, seed: int) -> np.ndarray:
+    """fp32 [n_experts, M_body]: W_ih, W_hh, W_1 ~ N(0, 1/sqrt(d)),
+    W_2 ~ N(0, 1/sqrt(4d)), gains 1."""
+    o = body_offsets(d, D)
+    rng = np.random.default_rng([seed & 0xFFFFFFFF, 0x2B0D])
+    th = np.zeros((n_experts, o["end"]), dtype=np.float64)
+    for k in range(D):
+        th[:, o[f"w_ih{k}"]:o[f"w2{k}"]] = rng.standard_normal((n_experts, 12 * d * d)) / np.sqrt(d)
+        th[:, o[f"w2{k}"]:o[f"w2{k}"] + 4 * d * d] = (rng.standard_normal((n_experts, 4 * d * d))
+                                                     / np.sqrt(4 * d))
+    th[:, o["gains"]:] = 1.0
+    return th.astype(np.float32)
+
+
+def init_head(d: int, seed: int) -> np.ndarray:
+    """fp32 [V, d] frozen tied embedding/decode matrix E ~ N(0, 1/sqrt(d)),
+    standing in for the seed run's learned E."""
+    rng = np.random.default_rng([seed & 0xFFFFFFFF, 0x4EAD])
+    return (rng.standard_normal((V, d)) / np.sqrt(d)).astype(np.float32)
+
+
+# The body workloads: the paper's width-32 N = 256 ensemble at the SOMA
+# N=256 batch shape, and its own training batch (B = 64, 1,024-byte windows).
+BODY_CONFIGS = {
+    "body_tiny": dict(n_experts=2, d=32, D=2, n_pert=4, eps=1e-3, lr=1e-3, batch=3, seq_len=20,
+                      order=2),
+    "body_n256": dict(n_experts=256, d=32, D=2, n_pert=64, eps=1e-3, lr=1e-3, batch=16,
+                      seq_len=512, order=2),
+    "body_n256_paper": dict(n_experts=256, d=32, D=2, n_pert=64, eps=1e-3, lr=1e-3, batch=64,
+                            seq_len=1024, order=2),
+}
+
+
+def body_config_batch(name: str, seed: int = 0, step: int = 0, **overrides) -> np.ndarray:
+    c = dict(BODY_CONFIGS[name], **overrides)
+    return expert_batch(c["n_experts"], c["batch"], c["seq_len"], c["order"], seed, step)
+
+
+def body_config_params(name: str, seed: int = 0, **overrides) -> np.ndarray:
+    c = dict(BODY_CONFIGS[name], **overrides)
+    return init_body(c["n_experts"], c["d"], c["D"], seed)
