@@ -498,8 +498,239 @@ def inference_arm(args):
     return 0
 
 
+# ---- the paper's expert body -------------------------------------------------
+
+def body_desc(name, c):
+    from paper_2609_37899_gb300 import inputs
+    P = inputs.body_param_count(c["d"], c["D"])
+    return (f"{name}: {c['n_experts']} expert bodies (D={c['D']} pre-norm blocks of width "
+            f"d={c['d']}: bias-free LSTM + GELU MLP 4d, gain-only LayerNorm; M_body={P:,}; frozen "
+            f"tied head E [256, {c['d']}]), n_pert={c['n_pert']}, eps={c['eps']}, lr={c['lr']}, "
+            f"B={c['batch']} x T={c['seq_len']} bytes per expert, order-{c['order']} Zipf(1.1) "
+            f"Markov clusters")
+
+
+def body_flops_per_token(c):
+    # per block: LSTM gates [2d] x [2d, 4d] and the MLP [d] x [d, 4d] x [4d, d];
+    # the tied decode [d] x [d, 256]; 2 flops per multiply-add
+    d = c["d"]
+    return c["D"] * (2 * 2 * d * 4 * d + 2 * 2 * d * 4 * d) + 2 * d * 256
+
+
+# fp32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flops x 2.07 GHz
+FP32_SIMT_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def body_cpu_baseline(cfg_name, c, n_seqs, kind):
+    import oracle
+    from paper_2609_37899_gb300 import inputs
+    theta = inputs.body_config_params(cfg_name)[:1]
+    head = inputs.init_head(c["d"], 0)
+    bx = inputs.body_config_batch(cfg_name)[:1, :n_seqs]
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    oracle.build()
+    t0 = time.perf_counter()
+    oracle.body_spsa_losses(theta, c["d"], c["D"], head, np.float32(c["eps"]), 0, 0, bx,
+                            probes=[0], kind=kind, n_threads=cores)
+    dt = time.perf_counter() - t0
+    toks = 2 * n_seqs * c["seq_len"]
+    return {"value": toks / dt, "unit": UNIT, "cores": min(cores, n_seqs), "kind": "oracle",
+            "sample": f"expert 0, {kind} probe 0, both signs, {n_seqs} of {c['batch']} sequences x "
+                      f"{c['seq_len']} bytes ({toks} perturbed tokens) in {dt:.2f} s; OpenMP "
+                      f"over sequences, so {min(cores, n_seqs)} of {cores} cores busy"}
+
+
+def body_reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2609_37899_gb300 import inputs
+    c = inputs.BODY_CONFIGS[args.config]
+    n_seqs = min(args.ref_sample_seqs, c["batch"])
+    theta = inputs.body_config_params(args.config)
+    head = inputs.init_head(c["d"], 0)
+    bx = inputs.body_config_batch(args.config)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    oracle.build()
+
+    def one(k):
+        e, i = k % c["n_experts"], k % c["n_pert"]
+        oracle.body_spsa_losses(theta[e:e + 1], c["d"], c["D"], head, np.float32(c["eps"]), 0, 0,
+                                bx[e:e + 1, :n_seqs], probes=[i], first_expert=e,
+                                n_threads=cores)
+
+    for k in range(args.warmup):
+        one(k)
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        one(args.warmup + k)
+    dt = time.perf_counter() - t0
+    toks = 2 * n_seqs * c["seq_len"]
+    value = toks * args.steps / dt
+    sample = (f"per step one probe pair (both signs) of one expert body over {n_seqs} of "
+              f"{c['batch']} sequences x {c['seq_len']} bytes = {toks} perturbed tokens")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": body_desc(args.config, c), "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": min(cores, n_seqs),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+    return 0
+
+
+def body_arm(args):
+    """SPSA steps of N expert bodies: the SGD step (Eq. main-spsa), or with
+    --optimizer adam the paper's step (sparse probes with dense gains, A
+    estimates, Adam: Eq. localspsa)."""
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_37899_gb300 import api, build, inputs
+    if not os.path.exists(api.LIB_PATH):
+        build.build()
+    c = dict(inputs.BODY_CONFIGS[args.config])
+    if args.seq_len:
+        c["seq_len"] = args.seq_len
+    N, d, D, n, B, T = c["n_experts"], c["d"], c["D"], c["n_pert"], c["batch"], c["seq_len"]
+    K, W = args.steps, args.warmup
+    adam = args.optimizer == "adam"
+    A = args.accum if adam else 1
+    kind = (args.probes or "sparse") if adam else (args.probes or "dense")
+    bodies = api.SomaBodies(N, n, B, T, d, D, device=dev)
+    bodies.params.copy_(torch.from_numpy(inputs.init_body(N, d, D, 1000 + rank)))
+    bodies.head.copy_(torch.from_numpy(inputs.init_head(d, 0)))
+    host = [[torch.from_numpy(inputs.body_config_batch(args.config, seed=rank, step=A * s + a,
+                                                       seq_len=T)).pin_memory()
+             for a in range(A)] for s in range(W + K)]
+    resident = [[h.to(dev) for h in hs] for hs in host]
+
+    def do_step(batches, s):
+        if not adam:
+            return bodies.step(batches[0], c["eps"], c["lr"], 0, s, kind=kind)[0]
+        return bodies.adam_step(batches, c["eps"], 0, [A * s + a for a in range(A)], t=s + 1,
+                                lr=c["lr"], kind=kind)[0]
+
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for s in range(W):
+        do_step(resident[s], s)
+    barrier()
+    api.trace_enable(True)
+    api.trace_read(reset=True)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        start.record(stream)
+        for s in range(K):
+            flush.fill_(s & 0xFF)
+            do_step(resident[W + s], W + s)
+        stop.record(stream)
+        barrier()
+    api.trace_enable(False)
+    traced = api.trace_read(reset=True)
+    ms = start.elapsed_time(stop)
+    status = api.get_status()
+    losses_host = torch.empty(A, N, n, 2, dtype=torch.float32).pin_memory()
+    dev_bytes = [torch.empty_like(r) for r in resident[0]]
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(K):
+        flush.fill_(s & 0xFF)
+        for a in range(A):
+            dev_bytes[a].copy_(host[W + s][a], non_blocking=True)
+        losses = do_step(dev_bytes, W + K + s)
+        losses_host.copy_(losses.reshape(losses_host.shape), non_blocking=True)
+    e1.record(stream)
+    barrier()
+    ms_e2e = e0.elapsed_time(e1)
+    if dist is not None:
+        t = torch.tensor([ms, ms_e2e], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, ms_e2e = float(t[0]), float(t[1])
+    if rank != 0:
+        dist.destroy_process_group()
+        return 0
+    tok = tokens_per_step(c) * A * world
+    value = tok * K / (ms / 1e3)
+    sweep_ms, sweep_n = traced["gate"]
+    flops = body_flops_per_token(c) * tokens_per_step(c) * A * K
+    achieved = flops / (sweep_ms / 1e3) / 1e12 if sweep_n else None
+    peaks, peak_src = measured_peaks()
+    tensor_peak = peaks["bf16_tflops_sustained"]
+    tr = TRAFFIC.get(args.config)
+    traffic = (tr["bytes_per_launch"]
+               if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "steps_per_s": K / (ms / 1e3),
+        "config": {
+            "workload": body_desc(args.config, c),
+            "optimizer": ("SGD (Eq. main-spsa), " + kind + " probes" if not adam else
+                          f"Adam with coupled decay, {kind} probes (gains dense), {A} "
+                          "accumulation batch(es) per update (Eq. localspsa)"),
+            "tokens_per_step_per_gpu": tokens_per_step(c) * A,
+            "seq_len": T,
+            "l2": "flushed between timed steps (a 256 MiB buffer is written before each "
+                  "step, inside the timed region)",
+            "parallelism": f"every (expert, probe, sign) in one launch; {world} independent "
+                           "replica(s), no collective",
+        },
+        "roofline": {
+            "bound": "alu", "kernel": "body_sweep_kernel (fp32 CUDA cores, one CTA per sign of "
+                                      "a probe pair, whole recurrence resident)",
+            "achieved": achieved, "peak": FP32_SIMT_TFLOPS, "unit": "TFLOP/s",
+            "frac": (achieved / FP32_SIMT_TFLOPS) if achieved else None, "traffic": traffic,
+            "peak_source": "fp32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flops x "
+                           "2.07 GHz (the kernel issues fp32 FMAs, not tensor-core MMAs)",
+            "frac_of_tensor_peak": (achieved / tensor_peak) if achieved else None,
+            "flops_per_token": body_flops_per_token(c),
+            "launches": sweep_n,
+            "kernel_ms_per_launch": sweep_ms / sweep_n if sweep_n else None,
+            "share_of_step": sweep_ms / ms if ms else None,
+        },
+        "kernel_ms": {k: v[0] / K for k, v in traced.items()},
+        "e2e": {"value": tok * K / (ms_e2e / 1e3), "unit": UNIT,
+                "h2d_bytes_per_step": int(sum(r.numel() for r in resident[0])),
+                "d2h_bytes_per_step": int(A * N * n * 2 * 4)},
+        "gpu_launches": sum(v[1] for v in traced.values()),
+        "clocks": clk.summary(),
+        "status": api.STATUS_NAMES.get(status, status),
+    }
+    if not args.no_cpu_baseline and world == 1:
+        line["cpu_baseline"] = body_cpu_baseline(args.config, c, min(args.cpu_sample_seqs, B),
+                                                 kind)
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     args = parse()
+    from paper_2609_37899_gb300 import inputs
+    if args.config in inputs.BODY_CONFIGS:
+        return body_reference_arm(args) if args.impl == "reference" else body_arm(args)
     if args.impl == "reference":
         return reference_arm(args)
     if args.inference:

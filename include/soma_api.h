@@ -289,6 +289,77 @@ int soma_spsa_step_static(float* params, int n_experts, soma_dims d, int n_pert,
                           int batch, int seq_len, float* losses_out, float* coef_out,
                           void* stream);
 
+/* ---- The paper's expert body (Sec. "Model size"; App. E) ---------------
+ * The width-32 ensembles' expert: D pre-norm residual blocks of width d,
+ *   u = LN(x) ga_k;  LSTM_k (bias-free, gates i, f, g, o; state reset per
+ *   sequence) on u;  x += h_k;  v = LN(x) gb_k;  x += W_2^k GELU(W_1^k v)
+ * (bias-free MLP of width 4d, exact erf GELU), starting from x = E[byte_t],
+ * then y = LN(x) gf and logits = E y.  LN(x) = (x - mean) / sqrt(var + 1e-5)
+ * with var the mean squared deviation.  E [256][d] is the frozen tied head:
+ * shared by every expert, never perturbed.
+ * Body parameters of one expert, M_body = 16 D d^2 + (2D + 1) d floats:
+ *   per block k: W_ih [4d][d], W_hh [4d][d], W_1 [4d][d], W_2 [d][4d];
+ *   then ga_0, gb_0, ..., ga_{D-1}, gb_{D-1}, gf [d] each.
+ * Probes (App. E): SOMA_PROBE_DENSE is the dense sign on every coordinate.
+ * SOMA_PROBE_SPARSE is the paper's training law: every gain takes the dense
+ * sign, every weight the sparse probe (same Philox stream and bit map as
+ * above, keyed by the flat body coordinate).
+ * Supported: vocab 256, width 32, blocks 1 or 2; else SOMA_ERR_UNSUPPORTED.
+ * The forward runs on CUDA cores in fp32 (losses summed in fp64); one CTA
+ * runs one sign of one (expert, probe) pair over up to 16 sequences. */
+typedef struct soma_body_dims {
+  int32_t vocab;  /* must be 256 */
+  int32_t width;  /* d = d_t = d_E */
+  int32_t blocks; /* D */
+} soma_body_dims;
+
+/* M_body, or -1 for unsupported dims. */
+int64_t soma_body_param_count(soma_body_dims d);
+
+/* Workspace of soma_body_spsa_step / _estimate / _eval_loss (0 for invalid
+ * sizes). */
+size_t soma_body_workspace_bytes(soma_body_dims d, int n_experts, int n_pert, int batch,
+                                 int seq_len);
+
+/* Losses and coefficients of one batch; params are not changed.
+ *   params      device fp32 [n_experts][M_body]
+ *   head        device fp32 [256][d], the frozen tied matrix E
+ *   byte_batch  device uint8 [n_experts][batch][seq_len + 1], shared by every
+ *               probe and both signs of an expert
+ *   losses_out  device fp32 [n_experts][n_pert][2] (L+, L-) or NULL
+ *   coef_out    device fp32 [n_experts][n_pert]: (L+ - L-) / (2 eps)
+ * eps == 0 gives L+ == L- == L(theta) and coefficients 0. */
+int soma_body_spsa_estimate(const float* params, int n_experts, soma_body_dims d,
+                            const float* head, int n_pert, int probe_kind, float eps,
+                            uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
+                            int seq_len, float* losses_out, float* coef_out, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+/* The estimate, then theta <- theta - lr (1/n_pert) sum_i c_i z_i with the
+ * same probes (Eq. main-spsa); coef_out may be NULL. */
+int soma_body_spsa_step(float* params, int n_experts, soma_body_dims d, const float* head,
+                        int n_pert, int probe_kind, float eps, float lr, uint64_t seed,
+                        uint64_t step, const uint8_t* byte_batch, int batch, int seq_len,
+                        float* losses_out, float* coef_out, void* workspace,
+                        size_t workspace_bytes, void* stream);
+
+/* loss_out device fp32 [n_experts] = L(theta_e) on its batch. */
+int soma_body_eval_loss(const float* params, int n_experts, soma_body_dims d, const float* head,
+                        const uint8_t* byte_batch, int batch, int seq_len, float* loss_out,
+                        void* workspace, size_t workspace_bytes, void* stream);
+
+/* Eq. localspsa on the body coordinates: as soma_adam_update, with the
+ * body's probe law. */
+int soma_body_adam_update(float* params, float* m, float* v, int n_experts, soma_body_dims d,
+                          int n_pert, int probe_kind, uint64_t seed, const uint64_t* steps,
+                          int n_acc, const float* coef, soma_adam_config cfg, void* stream);
+
+/* z_out device int8 [count]: body probe coordinates p0 .. p0 + count - 1
+ * (p0 + count <= 2^30). */
+int soma_debug_body_probe(uint64_t seed, uint64_t step, int expert, int pert, soma_body_dims d,
+                          int probe_kind, int64_t p0, int64_t count, int8_t* z_out,
+                          void* stream);
+
 #ifdef __cplusplus
 }
 #endif

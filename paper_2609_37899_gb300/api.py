@@ -39,6 +39,10 @@ class soma_dims(ctypes.Structure):
 TRACE_KINDS = ("gate", "head", "reduce", "update", "prep")
 
 
+class soma_body_dims(ctypes.Structure):
+    _fields_ = [("vocab", ctypes.c_int32), ("width", ctypes.c_int32), ("blocks", ctypes.c_int32)]
+
+
 class soma_adam_config(ctypes.Structure):
     _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
                 ("delta", ctypes.c_float), ("weight_decay", ctypes.c_float),
@@ -103,6 +107,18 @@ def lib():
         _sig(L, "soma_spsa_estimate_opts", i32, [vp, i32, soma_dims, i32,
                                                  ctypes.POINTER(soma_estimate_options), f32, u64,
                                                  u64, vp, i32, i32, vp, vp, vp, sz, vp])
+        bd = soma_body_dims
+        _sig(L, "soma_body_param_count", i64, [bd])
+        _sig(L, "soma_body_workspace_bytes", sz, [bd, i32, i32, i32, i32])
+        _sig(L, "soma_body_spsa_estimate", i32, [vp, i32, bd, vp, i32, i32, f32, u64, u64, vp,
+                                                 i32, i32, vp, vp, vp, sz, vp])
+        _sig(L, "soma_body_spsa_step", i32, [vp, i32, bd, vp, i32, i32, f32, f32, u64, u64, vp,
+                                             i32, i32, vp, vp, vp, sz, vp])
+        _sig(L, "soma_body_eval_loss", i32, [vp, i32, bd, vp, vp, i32, i32, vp, vp, sz, vp])
+        _sig(L, "soma_body_adam_update", i32, [vp, vp, vp, i32, bd, i32, i32, u64,
+                                               ctypes.POINTER(ctypes.c_uint64), i32, vp,
+                                               soma_adam_config, vp])
+        _sig(L, "soma_debug_body_probe", i32, [u64, u64, i32, i32, bd, i32, i64, i64, vp, vp])
         _lib = L
         return L
 
@@ -368,3 +384,144 @@ class SomaExperts:
         adam_update(self.params, self.m, self.v, self.E, self.H, kind, seed, steps, self.coef_acc,
                     lr, beta1, beta2, delta, weight_decay, t, stream)
         return self.losses_acc, self.coef_acc
+
+
+# ---------------------------------------------------------------------------
+# The paper's expert body (Sec. "Model size"): D pre-norm residual blocks of
+# width d (bias-free LSTM, GELU MLP of width 4d), gain-only LayerNorm, and a
+# frozen tied head E [256, d] shared by every expert.
+# ---------------------------------------------------------------------------
+
+def body_dims(d: int = 32, D: int = 2) -> soma_body_dims:
+    return soma_body_dims(V, d, D)
+
+
+def body_param_count(d: int = 32, D: int = 2) -> int:
+    return int(lib().soma_body_param_count(body_dims(d, D)))
+
+
+def body_workspace_bytes(d: int, D: int, n_experts: int, n_pert: int, batch: int,
+                         seq_len: int) -> int:
+    return int(lib().soma_body_workspace_bytes(body_dims(d, D), n_experts, n_pert, batch,
+                                               seq_len))
+
+
+def body_alloc_workspace(d, D, n_experts, n_pert, batch, seq_len, device="cuda") -> torch.Tensor:
+    n = body_workspace_bytes(d, D, n_experts, n_pert, batch, seq_len)
+    if n == 0:
+        raise ValueError("invalid sizes for the workspace")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def body_spsa_estimate(params: torch.Tensor, head: torch.Tensor, byte_batch: torch.Tensor,
+                       d: int, D: int, n_pert: int, kind: str, eps: float, seed: int, step: int,
+                       losses: torch.Tensor | None, coef: torch.Tensor, workspace: torch.Tensor,
+                       stream=None):
+    """Losses [N, n_pert, 2] and coefficients [N, n_pert] of the body;
+    params [N, M_body] are read only, head [256, d], byte_batch [N, B, T+1]."""
+    N, B, T1 = byte_batch.shape
+    P = body_param_count(d, D)
+    _check(lib().soma_body_spsa_estimate(
+        _dev(params, torch.float32, "params", N * P), N, body_dims(d, D),
+        _dev(head, torch.float32, "head", V * d), n_pert, PROBE_KINDS[kind], eps, seed, step,
+        _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
+        _dev(losses, torch.float32, "losses", N * n_pert * 2) if losses is not None else None,
+        _dev(coef, torch.float32, "coef", N * n_pert),
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_body_spsa_estimate")
+
+
+def body_spsa_step(params: torch.Tensor, head: torch.Tensor, byte_batch: torch.Tensor, d: int,
+                   D: int, n_pert: int, kind: str, eps: float, lr: float, seed: int, step: int,
+                   losses: torch.Tensor | None, coef: torch.Tensor | None,
+                   workspace: torch.Tensor, stream=None):
+    """The body's SPSA step: the estimate, then theta -= lr (1/n) sum_i c_i z_i."""
+    N, B, T1 = byte_batch.shape
+    P = body_param_count(d, D)
+    _check(lib().soma_body_spsa_step(
+        _dev(params, torch.float32, "params", N * P), N, body_dims(d, D),
+        _dev(head, torch.float32, "head", V * d), n_pert, PROBE_KINDS[kind], eps, lr, seed, step,
+        _dev(byte_batch, torch.uint8, "byte_batch"), B, T1 - 1,
+        _dev(losses, torch.float32, "losses", N * n_pert * 2) if losses is not None else None,
+        _dev(coef, torch.float32, "coef", N * n_pert) if coef is not None else None,
+        _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)),
+        "soma_body_spsa_step")
+
+
+def body_eval_loss(params: torch.Tensor, head: torch.Tensor, byte_batch: torch.Tensor, d: int,
+                   D: int, workspace: torch.Tensor, stream=None) -> torch.Tensor:
+    N, B, T1 = byte_batch.shape
+    out = torch.empty(N, dtype=torch.float32, device=params.device)
+    _check(lib().soma_body_eval_loss(
+        _dev(params, torch.float32, "params", N * body_param_count(d, D)), N, body_dims(d, D),
+        _dev(head, torch.float32, "head", V * d), _dev(byte_batch, torch.uint8, "byte_batch"),
+        B, T1 - 1, _dev(out, torch.float32, "loss"), _dev(workspace, torch.uint8, "workspace"),
+        workspace.numel(), _stream(stream)), "soma_body_eval_loss")
+    return out
+
+
+def body_adam_update(params: torch.Tensor, m: torch.Tensor, v: torch.Tensor, d: int, D: int,
+                     kind: str, seed: int, steps, coef: torch.Tensor, lr: float, beta1: float,
+                     beta2: float, delta: float, weight_decay: float, t: int, stream=None):
+    """Eq. localspsa on the body; coef [A, N, n_pert], steps: A host ints."""
+    A, N, n_pert = coef.shape
+    P = body_param_count(d, D)
+    st = (ctypes.c_uint64 * A)(*[int(x) for x in steps])
+    cfg = soma_adam_config(lr, beta1, beta2, delta, weight_decay, t)
+    _check(lib().soma_body_adam_update(
+        _dev(params, torch.float32, "params", N * P), _dev(m, torch.float32, "m", N * P),
+        _dev(v, torch.float32, "v", N * P), N, body_dims(d, D), n_pert, PROBE_KINDS[kind], seed,
+        st, A, _dev(coef, torch.float32, "coef", A * N * n_pert), cfg, _stream(stream)),
+        "soma_body_adam_update")
+
+
+def debug_body_probe(seed: int, step: int, expert: int, probe: int, d: int, D: int, kind: str,
+                     p0: int, count: int, stream=None) -> torch.Tensor:
+    z = torch.zeros(count, dtype=torch.int8, device="cuda")
+    _check(lib().soma_debug_body_probe(seed, step, expert, probe, body_dims(d, D),
+                                       PROBE_KINDS[kind], p0, count,
+                                       _dev(z, torch.int8, "z"), _stream(stream)),
+           "soma_debug_body_probe")
+    return z
+
+
+class SomaBodies:
+    """N expert bodies of the paper's architecture with their shared frozen
+    head, parameters, workspace and Adam moments resident on the device."""
+
+    def __init__(self, n_experts: int, n_pert: int, batch: int, seq_len: int, d: int = 32,
+                 D: int = 2, device: str = "cuda"):
+        self.N, self.d, self.D, self.n_pert = n_experts, d, D, n_pert
+        self.P = body_param_count(d, D)
+        if self.P < 0:
+            raise ValueError("unsupported body dims")
+        self.params = torch.zeros(n_experts, self.P, dtype=torch.float32, device=device)
+        self.head = torch.zeros(V, d, dtype=torch.float32, device=device)
+        self.m = torch.zeros_like(self.params)
+        self.v = torch.zeros_like(self.params)
+        self.workspace = body_alloc_workspace(d, D, n_experts, n_pert, batch, seq_len, device)
+        self.losses = torch.empty(n_experts, n_pert, 2, dtype=torch.float32, device=device)
+        self.coef = torch.empty(n_experts, n_pert, dtype=torch.float32, device=device)
+
+    def step(self, byte_batch, eps, lr, seed, step, kind="sparse", stream=None):
+        body_spsa_step(self.params, self.head, byte_batch, self.d, self.D, self.n_pert, kind, eps,
+                       lr, seed, step, self.losses, self.coef, self.workspace, stream)
+        return self.losses, self.coef
+
+    def eval(self, byte_batch, stream=None):
+        return body_eval_loss(self.params, self.head, byte_batch, self.d, self.D, self.workspace,
+                              stream)
+
+    def adam_step(self, byte_batches, eps, seed, steps, t, lr, beta1=0.9, beta2=0.999,
+                  delta=1e-8, weight_decay=1e-4, kind="sparse", stream=None):
+        """Eq. localspsa: one estimate per accumulation batch, then Adam."""
+        A = len(byte_batches)
+        coef = torch.empty(A, self.N, self.n_pert, dtype=torch.float32, device=self.params.device)
+        losses = torch.empty(A, self.N, self.n_pert, 2, dtype=torch.float32,
+                             device=self.params.device)
+        for a, bx in enumerate(byte_batches):
+            body_spsa_estimate(self.params, self.head, bx, self.d, self.D, self.n_pert, kind, eps,
+                               seed, steps[a], losses[a], coef[a], self.workspace, stream)
+        body_adam_update(self.params, self.m, self.v, self.d, self.D, kind, seed, steps, coef, lr,
+                         beta1, beta2, delta, weight_decay, t, stream)
+        return losses, coef

@@ -8,6 +8,7 @@
 #include <vector>
 
 #include "soma_api.h"
+#include "body_device.cuh"
 #include "soma_launch.h"
 
 using namespace soma;
@@ -531,3 +532,160 @@ int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint
     e = launch_mixture(nll, route, slot, R, k, seq_len, t0, m.b_max, nll_out, st);
   return cuda_status(e);
 }
+
+// ---- The paper's expert body (body.cu) ------------------------------------
+
+namespace {
+
+bool body_dims_ok(const soma_body_dims& d) {
+  return d.vocab == kVocab && d.width == kBodyWidth && d.blocks >= 1 &&
+         d.blocks <= kBodyMaxBlocks;
+}
+
+// fp64 NLL sums [N * n * n_sign][chunks], then the coefficients [N][n].
+struct BodyWs {
+  size_t partial, coef, total;
+};
+
+BodyWs plan_body(int n_experts, int n_pert, int n_sign, int B) {
+  BodyWs w;
+  const int chunks = (B + body_rows_per_cta() - 1) / body_rows_per_cta();
+  w.partial = round_up((size_t)n_experts * n_pert * n_sign * chunks * sizeof(double));
+  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
+  w.total = w.partial + w.coef;
+  return w;
+}
+
+bool body_sizes_ok(int n_experts, int n_pert, int batch, int seq_len) {
+  if (!sizes_ok(n_experts, n_pert, batch, seq_len)) return false;
+  return (batch + body_rows_per_cta() - 1) / body_rows_per_cta() <= 65535;
+}
+
+int body_forward(float* params, int n_experts, soma_body_dims d, const float* head, int n_pert,
+                 int probe_kind, float eps, float lr, bool update, uint64_t seed, uint64_t step,
+                 const uint8_t* byte_batch, int batch, int seq_len, float* losses_out,
+                 float* coef_out, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!body_dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !head || !byte_batch || !aligned16(params) || !aligned16(head) ||
+      !body_sizes_ok(n_experts, n_pert, batch, seq_len) || !(eps >= 0.f) ||
+      !std::isfinite(eps) || !std::isfinite(lr) ||
+      (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE) ||
+      (!update && !coef_out))
+    return SOMA_ERR_INVALID_ARG;
+  const BodyWs w = plan_body(n_experts, n_pert, 2, batch);
+  if (!workspace || !aligned16(workspace) || workspace_bytes < w.total) return SOMA_ERR_WORKSPACE;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+  double* partial = static_cast<double*>(workspace);
+  float* coef_ws = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + w.partial);
+  cudaError_t e = launch_body_sweep(params, head, byte_batch, n_experts, d.blocks, n_pert, 2,
+                                    batch, seq_len, eps, probe_kind, seed, step, partial, st);
+  if (e == cudaSuccess)
+    e = launch_body_reduce(partial, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
+                           coef_out, coef_ws, status, st);
+  // eps == 0 or lr == 0 leaves theta bit-identical: no update launch
+  if (update && e == cudaSuccess && eps != 0.f && lr != 0.f)
+    e = launch_body_sgd(params, n_experts, d.blocks, n_pert, probe_kind, lr, seed, step, coef_ws,
+                        st);
+  return cuda_status(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+int64_t soma_body_param_count(soma_body_dims d) {
+  if (!body_dims_ok(d)) return -1;
+  return body_param_count(d.width, d.blocks);
+}
+
+size_t soma_body_workspace_bytes(soma_body_dims d, int n_experts, int n_pert, int batch,
+                                 int seq_len) {
+  if (!body_dims_ok(d) || !body_sizes_ok(n_experts, n_pert, batch, seq_len)) return 0;
+  return plan_body(n_experts, n_pert, 2, batch).total;  // >= the eval's
+}
+
+int soma_body_spsa_estimate(const float* params, int n_experts, soma_body_dims d,
+                            const float* head, int n_pert, int probe_kind, float eps,
+                            uint64_t seed, uint64_t step, const uint8_t* byte_batch, int batch,
+                            int seq_len, float* losses_out, float* coef_out, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  // the sweep only reads params
+  return body_forward(const_cast<float*>(params), n_experts, d, head, n_pert, probe_kind, eps,
+                      0.f, false, seed, step, byte_batch, batch, seq_len, losses_out, coef_out,
+                      workspace, workspace_bytes, stream);
+}
+
+int soma_body_spsa_step(float* params, int n_experts, soma_body_dims d, const float* head,
+                        int n_pert, int probe_kind, float eps, float lr, uint64_t seed,
+                        uint64_t step, const uint8_t* byte_batch, int batch, int seq_len,
+                        float* losses_out, float* coef_out, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+  return body_forward(params, n_experts, d, head, n_pert, probe_kind, eps, lr, true, seed, step,
+                      byte_batch, batch, seq_len, losses_out, coef_out, workspace,
+                      workspace_bytes, stream);
+}
+
+int soma_body_eval_loss(const float* params, int n_experts, soma_body_dims d, const float* head,
+                        const uint8_t* byte_batch, int batch, int seq_len, float* loss_out,
+                        void* workspace, size_t workspace_bytes, void* stream) {
+  if (!body_dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !head || !byte_batch || !loss_out || !aligned16(params) || !aligned16(head) ||
+      !body_sizes_ok(n_experts, 1, batch, seq_len))
+    return SOMA_ERR_INVALID_ARG;
+  const BodyWs w = plan_body(n_experts, 1, 1, batch);
+  if (!workspace || !aligned16(workspace) || workspace_bytes < w.total) return SOMA_ERR_WORKSPACE;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)stream;
+  double* partial = static_cast<double*>(workspace);
+  cudaError_t e = launch_body_sweep(params, head, byte_batch, n_experts, d.blocks, 1, 1, batch,
+                                    seq_len, 0.f, 0, 0, 0, partial, st);
+  if (e == cudaSuccess)
+    e = launch_body_reduce(partial, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
+                           nullptr, status, st);
+  return cuda_status(e);
+}
+
+int soma_body_adam_update(float* params, float* m, float* v, int n_experts, soma_body_dims d,
+                          int n_pert, int probe_kind, uint64_t seed, const uint64_t* steps,
+                          int n_acc, const float* coef, soma_adam_config cfg, void* stream) {
+  if (!body_dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!params || !m || !v || !coef || !steps || !aligned16(params) || !aligned16(m) ||
+      !aligned16(v) || n_experts < 1 || n_pert < 1 || n_pert > kMaxPert || n_acc < 1 ||
+      n_acc > SOMA_MAX_ACCUM || (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE))
+    return SOMA_ERR_INVALID_ARG;
+  if (!std::isfinite(cfg.lr) || !(cfg.beta1 >= 0.f && cfg.beta1 < 1.f) ||
+      !(cfg.beta2 >= 0.f && cfg.beta2 < 1.f) || !(cfg.delta > 0.f) || !std::isfinite(cfg.delta) ||
+      !(cfg.weight_decay >= 0.f) || !std::isfinite(cfg.weight_decay) || cfg.t < 1)
+    return SOMA_ERR_INVALID_ARG;
+  AdamSteps st;
+  st.n_acc = n_acc;
+  for (int a = 0; a < n_acc; ++a) st.step[a] = steps[a];
+  AdamArgs h;
+  h.lr = cfg.lr;
+  h.b1 = cfg.beta1;
+  h.b2 = cfg.beta2;
+  h.delta = cfg.delta;
+  h.wd = cfg.weight_decay;
+  h.inv_bc1 = (float)(1.0 / (1.0 - std::pow((double)cfg.beta1, (double)cfg.t)));
+  h.inv_bc2 = (float)(1.0 / (1.0 - std::pow((double)cfg.beta2, (double)cfg.t)));
+  return cuda_status(launch_body_adam(params, m, v, n_experts, d.blocks, n_pert, probe_kind, seed,
+                                      st, coef, h, (cudaStream_t)stream));
+}
+
+int soma_debug_body_probe(uint64_t seed, uint64_t step, int expert, int pert, soma_body_dims d,
+                          int probe_kind, int64_t p0, int64_t count, int8_t* z_out,
+                          void* stream) {
+  if (!body_dims_ok(d)) return SOMA_ERR_UNSUPPORTED;
+  if (!z_out || count < 0 || p0 < 0 || expert < 0 || pert < 0 ||
+      (probe_kind != SOMA_PROBE_DENSE && probe_kind != SOMA_PROBE_SPARSE) ||
+      p0 + count > ((int64_t)1 << 30))
+    return SOMA_ERR_INVALID_ARG;
+  if (count == 0) return SOMA_OK;
+  return cuda_status(launch_debug_body_probe(seed, step, expert, pert, d.blocks, probe_kind, p0,
+                                             count, z_out, (cudaStream_t)stream));
+}
+
+}  // extern "C"

@@ -110,4 +110,25 @@ cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& 
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                                const float* coef, const AdamArgs& h, cudaStream_t stream);
 
+// The paper's expert body (body.cu): width kBodyWidth, 1 <= blocks <=
+// kBodyMaxBlocks.  partial [N * n * n_sign][ceil(B / 16)] fp64 NLL sums.
+size_t body_smem_bytes();
+int body_rows_per_cta();
+cudaError_t launch_body_sweep(const float* params, const float* head, const uint8_t* bytes,
+                              int n_experts, int blocks, int n_pert, int n_sign, int B, int T,
+                              float eps, int sparse, uint64_t seed, uint64_t step,
+                              double* partial, cudaStream_t stream);
+cudaError_t launch_body_reduce(const double* partial, int pairs, int n_sign, int B, int T,
+                               float eps, float* losses_out, float* coef_out, float* coef_ws,
+                               int* status, cudaStream_t stream);
+cudaError_t launch_body_sgd(float* params, int n_experts, int blocks, int n_pert, int sparse,
+                            float lr, uint64_t seed, uint64_t step, const float* coef,
+                            cudaStream_t stream);
+cudaError_t launch_body_adam(float* params, float* m, float* v, int n_experts, int blocks,
+                             int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
+                             const float* coef, const AdamArgs& h, cudaStream_t stream);
+cudaError_t launch_debug_body_probe(uint64_t seed, uint64_t step, int expert, int pert, int blocks,
+                                    int sparse, int64_t p0, int64_t count, int8_t* z,
+                                    cudaStream_t stream);
+
 }  // namespace soma

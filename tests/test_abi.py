@@ -31,7 +31,10 @@ def test_header_declares_the_entry_points():
                      "soma_status_string", "soma_spsa_update", "soma_debug_philox",
                      "soma_debug_rademacher", "soma_spsa_estimate", "soma_adam_update",
                      "soma_debug_probe", "soma_spsa_estimate_opts", "soma_mixture_nll",
-                     "soma_mixture_workspace_bytes"]:
+                     "soma_mixture_workspace_bytes", "soma_body_param_count",
+                     "soma_body_workspace_bytes", "soma_body_spsa_estimate",
+                     "soma_body_spsa_step", "soma_body_eval_loss", "soma_body_adam_update",
+                     "soma_debug_body_probe"]:
         assert required in names
 
 
@@ -127,3 +130,41 @@ def test_host_validation_rejects_before_launch(soma):
                               None) == 1  # t0 = seq_len
     assert L.soma_mixture_nll(fake, 2, d, fake, 1, 8, good, 17, 0, fake, fake, 1 << 20,
                               None) == 1  # k > 16
+
+
+def test_body_sizes_and_validation(soma):
+    """The expert body's entry points: sizes and host-side rejection (no launch)."""
+    L = soma.lib()
+    assert soma.body_param_count(32, 2) == 32 * 32 * 32 + 5 * 32 == 32_928
+    assert soma.body_param_count(32, 1) == 16 * 32 * 32 + 3 * 32
+    for bad in ((16, 2), (32, 3), (32, 0)):
+        assert soma.body_param_count(*bad) == -1
+    assert L.soma_body_param_count(soma.soma_body_dims(255, 32, 2)) == -1
+    w = soma.body_workspace_bytes(32, 2, 256, 64, 16, 512)
+    assert w >= 256 * 64 * 2 * 8 + 256 * 64 * 4
+    assert soma.body_workspace_bytes(32, 2, 256, 64, 17, 512) > w  # a second chunk
+    assert soma.body_workspace_bytes(32, 2, 0, 64, 16, 512) == 0
+    d = soma.body_dims(32, 2)
+    fake = ctypes.c_void_p(0x10000)
+    ws = 1 << 20
+    # unsupported dims, bad kind, negative eps, missing coefficients, workspace
+    assert L.soma_body_spsa_step(fake, 1, soma.soma_body_dims(256, 16, 2), fake, 4, 1, 1e-3,
+                                 1e-3, 0, 0, fake, 4, 8, fake, fake, fake, ws, None) == 2
+    assert L.soma_body_spsa_step(fake, 1, d, fake, 4, 2, 1e-3, 1e-3, 0, 0, fake, 4, 8, fake,
+                                 fake, fake, ws, None) == 1
+    assert L.soma_body_spsa_step(fake, 1, d, fake, 4, 1, -1e-3, 1e-3, 0, 0, fake, 4, 8, fake,
+                                 fake, fake, ws, None) == 1
+    assert L.soma_body_spsa_step(fake, 1, d, None, 4, 1, 1e-3, 1e-3, 0, 0, fake, 4, 8, fake,
+                                 fake, fake, ws, None) == 1  # no head
+    assert L.soma_body_spsa_estimate(fake, 1, d, fake, 4, 1, 1e-3, 0, 0, fake, 4, 8, fake, None,
+                                     fake, ws, None) == 1
+    assert L.soma_body_spsa_step(fake, 1, d, fake, 4, 1, 1e-3, 1e-3, 0, 0, fake, 4, 8, fake,
+                                 fake, fake, 16, None) == 3
+    assert L.soma_body_eval_loss(fake, 1, d, fake, fake, 4, 8, fake, fake, 16, None) == 3
+    assert L.soma_body_eval_loss(fake, 1, d, fake, fake, 0, 8, fake, fake, ws, None) == 1
+    cfg = soma.soma_adam_config(1e-3, 0.9, 0.999, 1e-8, 1e-4, 0)  # t = 0
+    steps = (ctypes.c_uint64 * 1)(0)
+    assert L.soma_body_adam_update(fake, fake, fake, 1, d, 4, 1, 0, steps, 1, fake, cfg,
+                                   None) == 1
+    assert L.soma_debug_body_probe(0, 0, 0, 0, d, 1, -1, 4, fake, None) == 1
+    assert L.soma_debug_body_probe(0, 0, 0, 0, d, 1, 1 << 30, 4, fake, None) == 1
