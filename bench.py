@@ -117,6 +117,24 @@ def gate_flops_per_timestep(c):
     return c["n_experts"] * c["n_pert"] * 2 * c["batch"] * 8 * c["H"] * (c["E"] + c["H"])
 
 
+def shard_seeds(rank):
+    """Seeds of rank `rank`'s shard.  The parameter init, the data and the
+    probe streams all differ between ranks, so N ranks step N disjoint sets of
+    experts with no data-path collective (weak scaling)."""
+    return {"init": 1000 + rank, "data": rank, "probe": rank}
+
+
+def max_over_ranks(dist, values, device=None):
+    """Timings reduced with MAX over the ranks: the slowest rank sets the
+    job's time.  The identity without a process group."""
+    if dist is None:
+        return [float(v) for v in values]
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -276,8 +294,9 @@ def our_arm(args):
     kind = (args.probes or "sparse") if adam else "dense"
     if not 1 <= A <= api.MAX_ACCUM:
         raise SystemExit(f"--accum must be in 1..{api.MAX_ACCUM}")
+    seeds = shard_seeds(rank)
     experts = api.SomaExperts(N, E, H, n, B, T, device=dev)
-    experts.init(seed=1000 + rank, std=c["init_std"] or 0.0)
+    experts.init(seed=seeds["init"], std=c["init_std"] or 0.0)
     # every step gets its own A batches: (W + K) A host batches, pinned, and
     # their HBM-resident copies for the device-timed run
     per_probe = adam and args.batch_per_probe
@@ -285,11 +304,12 @@ def our_arm(args):
 
     def host_batch(k):
         if not per_probe:
-            return torch.from_numpy(inputs.config_batch(args.config, seed=rank, step=k,
+            return torch.from_numpy(inputs.config_batch(args.config, seed=seeds["data"], step=k,
                                                         seq_len=c["seq_len"])).pin_memory()
         # [N, n, B, T+1]: probe i of batch k draws its own sequences
         return torch.from_numpy(np.stack(
-            [inputs.config_batch(args.config, seed=rank, step=k * n + i, seq_len=c["seq_len"])
+            [inputs.config_batch(args.config, seed=seeds["data"], step=k * n + i,
+                                 seq_len=c["seq_len"])
              for i in range(n)], axis=1)).pin_memory()
 
     host = [[host_batch(A * s + a) for a in range(A)] for s in range(W + K)]
@@ -299,8 +319,9 @@ def our_arm(args):
         """One step: the SGD step, or A estimates plus the Adam update t = s + 1
         (App. E hyper-parameters: beta 0.9 / 0.999, delta 1e-8, decay 1e-4)."""
         if not adam:
-            return experts.step(batches[0], c["eps"], c["lr"], 0, s)[0]
-        losses, _ = experts.adam_step(batches, c["eps"], 0, [A * s + a for a in range(A)],
+            return experts.step(batches[0], c["eps"], c["lr"], seeds["probe"], s)[0]
+        losses, _ = experts.adam_step(batches, c["eps"], seeds["probe"],
+                                      [A * s + a for a in range(A)],
                                       t=s + 1, lr=c["lr"], kind=kind,
                                       batch_per_probe=per_probe, summed_loss=summed)
         return losses
@@ -350,10 +371,7 @@ def our_arm(args):
     barrier()
     ms_e2e = e0.elapsed_time(e1)
 
-    if dist is not None:
-        t = torch.tensor([ms, ms_e2e], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, ms_e2e = float(t[0]), float(t[1])
+    ms, ms_e2e = max_over_ranks(dist, [ms, ms_e2e], dev)
     if rank != 0:
         dist.destroy_process_group()
         return 0
@@ -608,19 +626,20 @@ def body_arm(args):
     adam = args.optimizer == "adam"
     A = args.accum if adam else 1
     kind = (args.probes or "sparse") if adam else (args.probes or "dense")
+    seeds = shard_seeds(rank)
     bodies = api.SomaBodies(N, n, B, T, d, D, device=dev)
-    bodies.params.copy_(torch.from_numpy(inputs.init_body(N, d, D, 1000 + rank)))
+    bodies.params.copy_(torch.from_numpy(inputs.init_body(N, d, D, seeds["init"])))
     bodies.head.copy_(torch.from_numpy(inputs.init_head(d, 0)))
-    host = [[torch.from_numpy(inputs.body_config_batch(args.config, seed=rank, step=A * s + a,
-                                                       seq_len=T)).pin_memory()
+    host = [[torch.from_numpy(inputs.body_config_batch(args.config, seed=seeds["data"],
+                                                       step=A * s + a, seq_len=T)).pin_memory()
              for a in range(A)] for s in range(W + K)]
     resident = [[h.to(dev) for h in hs] for hs in host]
 
     def do_step(batches, s):
         if not adam:
-            return bodies.step(batches[0], c["eps"], c["lr"], 0, s, kind=kind)[0]
-        return bodies.adam_step(batches, c["eps"], 0, [A * s + a for a in range(A)], t=s + 1,
-                                lr=c["lr"], kind=kind)[0]
+            return bodies.step(batches[0], c["eps"], c["lr"], seeds["probe"], s, kind=kind)[0]
+        return bodies.adam_step(batches, c["eps"], seeds["probe"], [A * s + a for a in range(A)],
+                                t=s + 1, lr=c["lr"], kind=kind)[0]
 
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
@@ -662,10 +681,7 @@ def body_arm(args):
     e1.record(stream)
     barrier()
     ms_e2e = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([ms, ms_e2e], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, ms_e2e = float(t[0]), float(t[1])
+    ms, ms_e2e = max_over_ranks(dist, [ms, ms_e2e], dev)
     if rank != 0:
         dist.destroy_process_group()
         return 0
