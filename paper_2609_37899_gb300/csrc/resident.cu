@@ -7,18 +7,22 @@
 // The gate weights W = [W_ih | W_hh], the head weights W_out and the probe
 // tiles Z of this pair are converted to fp16 tiles in shared memory once,
 // and the probes are therefore drawn once per step, not once per timestep.
-// The operand [vbar | dv] (rows) x [x | h] (K) also lives in shared memory:
-// the gate epilogue writes h of timestep t straight into it, where the head
-// of t and the gate of t + 1 read it.  Cell states stay in registers, and
-// the losses are summed in the CTA.  Per timestep:
-//   MMAs   head(t - 1) and gate(t) (one thread), one commit;
-//   head epilogue of t - 1: max / sum-exp per (sequence, sign) over both
-//          vocabulary halves, target logit, NLL summed in fp64;
-//   gate epilogue of t: gates and cells, h of t into the operand;
-//   the embedding part of the operand of t + 1.
+// The operand [vbar | dv] (rows) x [x | h] (K) also lives in shared memory,
+// in two buffers: buffer t % 2 holds [x_t | h_{t-1}].  Cell states stay in
+// registers, and the losses are summed in the CTA.  Per timestep t, after
+// the barrier that publishes buffer t % 2:
+//   MMA warp   gate(t) (commit), then head(t - 1) into head accumulator
+//              (t - 1) % 2 (its own commit barrier), both reading buffer t % 2;
+//   epilogues  head epilogue of t - 1 (max / sum-exp per (sequence, sign)
+//              over both vocabulary halves, target logit, NLL summed in fp64)
+//              while the gate MMAs of t run; then the gate epilogue of t
+//              (gates and cells), which writes h_t and the embedding of
+//              t + 1 into buffer (t + 1) % 2; then the barrier.
+// The head epilogue, the longest phase, thus overlaps the next gate MMAs,
+// and the serial chain of a timestep is gate MMAs -> gate epilogue.
 // The shape limits (H <= 64, B <= 32, 2 Bp Ek / 8 <= 256 operand chunks, the
-// tiles within shared memory) are
-// checked by res_supported(); larger experts use the persistent kernel.
+// tiles within shared memory, (MT + 4) 4 Bp <= 512 TMEM columns) are checked
+// by res_supported(); other experts use the persistent kernel.
 #include <cuda_fp16.h>
 
 #include "soma_api.h"
@@ -44,7 +48,7 @@ __device__ __forceinline__ float sigm_res(float x) { return __fdividef(1.0f, 1.0
 
 struct ResGeom {
   int E, H, Ek, Hk, K, MTg, Bp, B, T;
-  uint32_t wg, zg, wo, zo, op, emb, dx, red, ylog, acc, ctl, bytes;  // shared-memory offsets
+  uint32_t wg, zg, wo, zo, op, opsz, emb, dx, red, ylog, acc, ctl, bytes;  // shared-memory offsets
   uint32_t tmem_cols;
 };
 
@@ -67,7 +71,8 @@ ResGeom make_res_geom(const Layout& lay, int B, int T) {
   r.zg = o; o = res_align(o + r.MTg * gate_tile);
   r.wo = o; o = res_align(o + 2 * head_tile);
   r.zo = o; o = res_align(o + 2 * head_tile);
-  r.op = o; o = res_align(o + 2u * r.Bp * r.K * 2);
+  r.opsz = 2u * r.Bp * r.K * 2;  // one operand buffer [vbar | dv] x K, fp16
+  r.op = o; o = res_align(o + 2u * r.opsz);
   r.emb = o; o += 256u * r.Ek * 2;   // fp16 Emb rows [V][Ek]
   r.dx = o; o += 256u * r.Ek * 2;    // fp16 eps z of the Emb rows
   r.red = o; o += 2u * 4 * 2 * r.Bp * sizeof(float2);  // [half][quarter][sign][Bp]
@@ -77,7 +82,8 @@ ResGeom make_res_geom(const Layout& lay, int B, int T) {
   o = (o + 7u) & ~7u;
   r.ctl = o; o += 64;
   r.bytes = o + 1024;  // alignment slack of the dynamic shared-memory base
-  const uint32_t cols = (uint32_t)(r.MTg + 2) * 4 * r.Bp;
+  // gate accumulators, then two head accumulators (4 Bp columns per tile)
+  const uint32_t cols = (uint32_t)(r.MTg + 4) * 4 * r.Bp;
   r.tmem_cols = 32;
   while (r.tmem_cols < cols) r.tmem_cols <<= 1;
   return r;
@@ -113,8 +119,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
   uint64_t* gate_bar = reinterpret_cast<uint64_t*>(smem + g.ctl);
-  uint64_t* head_bar = reinterpret_cast<uint64_t*>(smem + g.ctl + 8);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 16);
+  uint64_t* head_bar = reinterpret_cast<uint64_t*>(smem + g.ctl + 8);  // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 24);
   float2* red = reinterpret_cast<float2*>(smem + g.red);
   float* ylog = reinterpret_cast<float*>(smem + g.ylog);
   double* acc = reinterpret_cast<double*>(smem + g.acc);
@@ -122,6 +128,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   if (tid == 0) {
     mbar_init(gate_bar, 1);
     mbar_init(head_bar, 1);
+    mbar_init(head_bar + 1, 1);
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(tmem_slot, g.tmem_cols);
@@ -176,7 +183,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
     *reinterpret_cast<uint4*>(smem + g.wo + off) = *reinterpret_cast<const uint4*>(w);
     *reinterpret_cast<uint4*>(smem + g.zo + off) = *reinterpret_cast<const uint4*>(z);
   }
-  for (int c = tid; c < 2 * g.Bp * g.K / 8; c += kResThreads)
+  for (int c = tid; c < 2 * (2 * g.Bp * g.K / 8); c += kResThreads)
     reinterpret_cast<uint4*>(smem + g.op)[c] = make_uint4(0u, 0u, 0u, 0u);
   // the embedding table and its eps z, so that the operand of a timestep is
   // gathered from shared memory
@@ -254,7 +261,6 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const uint32_t ghi = (uint32_t)(dg >> 32), wg_lo = (uint32_t)dg;
   const uint32_t hhi = (uint32_t)(dh >> 32), wo_lo = (uint32_t)dh;
   const uint32_t zg_lo = wg_lo + ((g.zg - g.wg) >> 4), op_lo = wg_lo + ((g.op - g.wg) >> 4);
-  const uint32_t oph_lo = op_lo + (uint32_t)g.Ek;  // the h part: Ek / 8 core matrices further
   const uint32_t zo_lo = wo_lo + ((g.zo - g.wo) >> 4);
   const uint32_t gstep = 16u * g.K, hstep = 16u * g.Hk;  // one 128-row tile, in 16-byte units
   bool ok = true;
@@ -263,66 +269,141 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const int xrow = xc / (g.Ek / 8), xk0 = 8 * (xc % (g.Ek / 8));
   const bool x_delta = xrow >= g.Bp;
   const int xb = x_delta ? xrow - g.Bp : xrow;
-  int ynext = (xc >= 0 && xb < g.B) ? s.bytes[seq_offset(s, e, i, xb)] : 0;
+  const uint4* xtab = reinterpret_cast<const uint4*>(smem + (x_delta ? g.dx : g.emb));
+  // the embedding part of operand buffer 0 (x_0; h_{-1} = 0): rows
+  // [vbar (Bp) | dv (Bp)], 16-byte chunks of the Emb / eps z tables
+  int ynext = 0;
+  if (xc >= 0 && xb < g.B) {
+    const int y0 = s.bytes[seq_offset(s, e, i, xb)];
+    *reinterpret_cast<uint4*>(smem + g.op + kmajor_offset(xrow, xk0, g.K)) =
+        xtab[y0 * (g.Ek / 8) + xk0 / 8];
+    if (g.T > 1) ynext = s.bytes[seq_offset(s, e, i, xb) + 1];
+  }
+  fence_async_smem();
+  tc_fence_before();
+  __syncthreads();
 
+  // A failed wait marks this thread; the decision is taken for the whole CTA
+  // at the barrier that ends the timestep.  Every warp reaches every barrier
+  // whatever its waits returned (a wait that times out returns false).
+  bool fine = true;
   for (int t = 0; t <= g.T && ok; ++t) {
-    // embedding part of the operand of timestep t: rows [vbar (Bp) | dv (Bp)],
-    // 16-byte chunks of the Emb / eps z tables; the next byte is fetched
-    // while this timestep runs
-    if (t < g.T && xc >= 0) {
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (xb < g.B) {
-        const uint4* tab = reinterpret_cast<const uint4*>(smem + (x_delta ? g.dx : g.emb));
-        v = tab[ynext * (g.Ek / 8) + xk0 / 8];
+    const uint32_t cur = (uint32_t)(t & 1), nxt = cur ^ 1u;
+    if (warp == kResMmaWarp) {
+      if (lane == 0) {
+        tc_fence_after();
+        const uint32_t ob = op_lo + cur * (g.opsz >> 4);  // operand buffer t % 2
+        if (t < g.T) {  // gate of t: [x_t | h_{t-1}]
+#pragma unroll 1
+          for (int m = 0; m < g.MTg; ++m) {
+            const uint32_t d = tmem + gcol0 + (uint32_t)m * 2 * n2;
+            const uint32_t wlo = wg_lo + (uint32_t)m * gstep, zlo = zg_lo + (uint32_t)m * gstep;
+            for (int k16 = 0; k16 < g.K / 16; ++k16) {
+              const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
+              mma_f16_ss_lohi(d, wlo + ko, ghi, ob + ko, ghi, idesc, acc_flag);
+              mma_f16_ss_lohi(d + n2, zlo + ko, ghi, ob + ko, ghi, idesc, acc_flag);
+            }
+          }
+          mma_commit(gate_bar);
+        }
+        if (t >= 1) {  // head of t - 1: the h part, h_{t-1}, into accumulator (t - 1) % 2
+          const uint32_t hb = (uint32_t)((t - 1) & 1);
+          const uint32_t obh = ob + (uint32_t)g.Ek;  // Ek / 8 core matrices further
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t d = tmem + hcol0 + hb * 4 * n2 + (uint32_t)h * 2 * n2;
+            const uint32_t wlo = wo_lo + (uint32_t)h * hstep, zlo = zo_lo + (uint32_t)h * hstep;
+            for (int k16 = 0; k16 < g.Hk / 16; ++k16) {
+              const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
+              mma_f16_ss_lohi(d, wlo + ko, hhi, obh + ko, ghi, idesc, acc_flag);
+              mma_f16_ss_lohi(d + n2, zlo + ko, hhi, obh + ko, ghi, idesc, acc_flag);
+            }
+          }
+          mma_commit(head_bar + hb);
+        }
       }
-      *reinterpret_cast<uint4*>(smem + g.op + kmajor_offset(xrow, xk0, g.K)) = v;
-      if (xb < g.B && t + 1 < g.T) ynext = s.bytes[seq_offset(s, e, i, xb) + t + 1];
+      __syncwarp();
     }
+
+    if (t < g.T && warp < kResEpiWarps) {
+      fine = mbar_wait(gate_bar, (uint32_t)t & 1u) && fine;
+      tc_fence_after();
+      if (tile < g.MTg) {
+        const uint32_t tq = tmem + gcol0 + (uint32_t)tile * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
+        const uint32_t tq2 = tq + (16u << 16);
+#pragma unroll
+        for (int c = 0; c < kResMaxBp / 8; ++c) {
+          const int b0 = 8 * c;
+          if (b0 >= g.Bp) break;
+          if ((c & 1) != sp) continue;
+          uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t cw = (uint32_t)(b0 + 4 * h);
+            tmem_ld_16x128b(tq + cw, wv[h][0], wv[h][1]);
+            tmem_ld_16x128b(tq2 + cw, wv[h][2], wv[h][3]);
+            tmem_ld_16x128b(tq + cw + g.Bp, wd[h][0], wd[h][1]);
+            tmem_ld_16x128b(tq2 + cw + g.Bp, wd[h][2], wd[h][3]);
+            tmem_ld_16x128b(tq + 2 * g.Bp + cw, zv[h][0], zv[h][1]);
+            tmem_ld_16x128b(tq2 + 2 * g.Bp + cw, zv[h][2], zv[h][3]);
+            tmem_ld_16x128b(tq + 3 * g.Bp + cw, zd[h][0], zd[h][1]);
+            tmem_ld_16x128b(tq2 + 3 * g.Bp + cw, zd[h][2], zd[h][3]);
+          }
+          tmem_wait_ld();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            float actp[4], actm[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float C = fmaf(eps, __uint_as_float(zd[h][k]), __uint_as_float(wv[h][k])) + bias[k];
+              const float D = fmaf(eps, __uint_as_float(zv[h][k]), __uint_as_float(wd[h][k])) + dbias[k];
+              if (k == 2) {
+                actp[k] = fmaf(sigm_res(2.f * (C + D)), 2.f, -1.f);
+                actm[k] = fmaf(sigm_res(2.f * (C - D)), 2.f, -1.f);
+              } else {
+                actp[k] = sigm_res(C + D);
+                actm[k] = sigm_res(C - D);
+              }
+            }
+            const float cp = fmaf(actp[1], cst[c][h][0], actp[0] * actp[2]);
+            const float cm = fmaf(actm[1], cst[c][h][1], actm[0] * actm[2]);
+            cst[c][h][0] = cp;
+            cst[c][h][1] = cm;
+            const float hp = actp[3] * fmaf(sigm_res(2.f * cp), 2.f, -1.f);
+            const float hm = actm[3] * fmaf(sigm_res(2.f * cm), 2.f, -1.f);
+            const int b = b0 + 4 * h + bq;
+            if (unit_ok && b < g.B) {
+              *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(b, g.Ek + U, g.K)) =
+                  __float2half_rn(0.5f * (hp + hm));
+              *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(g.Bp + b, g.Ek + U, g.K)) =
+                  __float2half_rn(0.5f * (hp - hm));
+            }
+          }
+        }
+      }
+      // the embedding part of buffer (t + 1) % 2
+      if (t + 1 < g.T && xc >= 0) {
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (xb < g.B) v = xtab[ynext * (g.Ek / 8) + xk0 / 8];
+        *reinterpret_cast<uint4*>(smem + g.op + nxt * g.opsz + kmajor_offset(xrow, xk0, g.K)) = v;
+        if (xb < g.B && t + 2 < g.T) ynext = s.bytes[seq_offset(s, e, i, xb) + t + 2];
+      }
+    }
+    if (!fine) atomicCAS(a.status, 0, kStatusTimeout);
     fence_async_smem();
     tc_fence_before();
-    __syncthreads();
-    if (warp == kResMmaWarp && lane == 0) {
+    ok = (__syncthreads_and(fine) != 0) && ok;
+    fine = true;
+    // after the barrier: the head epilogue of t - 1 runs while the MMA warp
+    // issues the gate of t + 1
+    if (t >= 1 && warp < kResEpiWarps) {
+      // head(t - 1) is the ((t - 1) / 2)-th commit to its barrier
+      const uint32_t hb = (uint32_t)((t - 1) & 1);
+      fine = mbar_wait(head_bar + hb, (uint32_t)((t - 1) >> 1) & 1u) && fine;
       tc_fence_after();
-      if (t >= 1) {  // head of t - 1: the h part of the operand
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const uint32_t d = tmem + hcol0 + (uint32_t)h * 2 * n2;
-          const uint32_t wlo = wo_lo + (uint32_t)h * hstep, zlo = zo_lo + (uint32_t)h * hstep;
-          for (int k16 = 0; k16 < g.Hk / 16; ++k16) {
-            const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
-            mma_f16_ss_lohi(d, wlo + ko, hhi, oph_lo + ko, ghi, idesc, acc_flag);
-            mma_f16_ss_lohi(d + n2, zlo + ko, hhi, oph_lo + ko, ghi, idesc, acc_flag);
-          }
-        }
-        mma_commit(head_bar);
-      }
-      if (t < g.T) {  // gate of t
-#pragma unroll 1
-        for (int m = 0; m < g.MTg; ++m) {
-          const uint32_t d = tmem + gcol0 + (uint32_t)m * 2 * n2;
-          const uint32_t wlo = wg_lo + (uint32_t)m * gstep, zlo = zg_lo + (uint32_t)m * gstep;
-          for (int k16 = 0; k16 < g.K / 16; ++k16) {
-            const uint32_t ko = (uint32_t)k16 * 16, acc_flag = k16 > 0 ? 1u : 0u;
-            mma_f16_ss_lohi(d, wlo + ko, ghi, op_lo + ko, ghi, idesc, acc_flag);
-            mma_f16_ss_lohi(d + n2, zlo + ko, ghi, op_lo + ko, ghi, idesc, acc_flag);
-          }
-        }
-        mma_commit(gate_bar);
-      }
-    }
-    __syncwarp();
-
-    // a failed wait marks this thread; the decision is taken for the whole
-    // CTA at the barrier that ends the timestep, so that no wait is followed
-    // by a CTA barrier (the issuing thread's warp would hold every warp back)
-    bool fine = true;
-    if (t >= 1) {
-      fine = mbar_wait(head_bar, (uint32_t)(t - 1) & 1u) && fine;
-      tc_fence_after();
-    }
-    if (t >= 1 && ok && warp < kResEpiWarps) {
       // ---- head epilogue of t - 1
-      const uint32_t tq = tmem + hcol0 + (uint32_t)half * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
+      const uint32_t tq = tmem + hcol0 + hb * 8u * g.Bp + (uint32_t)half * 4 * g.Bp +
+                         ((uint32_t)(32 * q4) << 16);
       const uint32_t tq2 = tq + (16u << 16);
       for (int b0 = 4 * sp; b0 < g.Bp; b0 += 8) {
         uint32_t wv[4], wd[4], zv[4], zd[4];
@@ -376,7 +457,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
           }
         }
       }
-      // the epilogue warps only: the MMA warp may still be issuing the gate
+      // the epilogue warps only: the MMA warp is issuing the gate of t
       asm volatile("bar.sync 1, %0;" ::"n"(kResEpiWarps * 32) : "memory");
       if (tid < g.B) {
         float nll[2];
@@ -396,68 +477,10 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       }
     }
 
-    if (t < g.T) {
-      fine = mbar_wait(gate_bar, (uint32_t)t & 1u) && fine;
-      tc_fence_after();
-    }
-    if (t < g.T && ok && warp < kResEpiWarps && tile < g.MTg) {
-      // ---- gate epilogue of t: cells in registers, h of t into the operand
-      const uint32_t tq = tmem + gcol0 + (uint32_t)tile * 4 * g.Bp + ((uint32_t)(32 * q4) << 16);
-      const uint32_t tq2 = tq + (16u << 16);
-#pragma unroll
-      for (int c = 0; c < kResMaxBp / 8; ++c) {
-        const int b0 = 8 * c;
-        if (b0 >= g.Bp) break;
-        if ((c & 1) != sp) continue;
-        uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const uint32_t cw = (uint32_t)(b0 + 4 * h);
-          tmem_ld_16x128b(tq + cw, wv[h][0], wv[h][1]);
-          tmem_ld_16x128b(tq2 + cw, wv[h][2], wv[h][3]);
-          tmem_ld_16x128b(tq + cw + g.Bp, wd[h][0], wd[h][1]);
-          tmem_ld_16x128b(tq2 + cw + g.Bp, wd[h][2], wd[h][3]);
-          tmem_ld_16x128b(tq + 2 * g.Bp + cw, zv[h][0], zv[h][1]);
-          tmem_ld_16x128b(tq2 + 2 * g.Bp + cw, zv[h][2], zv[h][3]);
-          tmem_ld_16x128b(tq + 3 * g.Bp + cw, zd[h][0], zd[h][1]);
-          tmem_ld_16x128b(tq2 + 3 * g.Bp + cw, zd[h][2], zd[h][3]);
-        }
-        tmem_wait_ld();
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          float actp[4], actm[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const float C = fmaf(eps, __uint_as_float(zd[h][k]), __uint_as_float(wv[h][k])) + bias[k];
-            const float D = fmaf(eps, __uint_as_float(zv[h][k]), __uint_as_float(wd[h][k])) + dbias[k];
-            if (k == 2) {
-              actp[k] = fmaf(sigm_res(2.f * (C + D)), 2.f, -1.f);
-              actm[k] = fmaf(sigm_res(2.f * (C - D)), 2.f, -1.f);
-            } else {
-              actp[k] = sigm_res(C + D);
-              actm[k] = sigm_res(C - D);
-            }
-          }
-          const float cp = fmaf(actp[1], cst[c][h][0], actp[0] * actp[2]);
-          const float cm = fmaf(actm[1], cst[c][h][1], actm[0] * actm[2]);
-          cst[c][h][0] = cp;
-          cst[c][h][1] = cm;
-          const float hp = actp[3] * fmaf(sigm_res(2.f * cp), 2.f, -1.f);
-          const float hm = actm[3] * fmaf(sigm_res(2.f * cm), 2.f, -1.f);
-          const int b = b0 + 4 * h + bq;
-          if (unit_ok && b < g.B) {
-            *reinterpret_cast<__half*>(smem + g.op + kmajor_offset(b, g.Ek + U, g.K)) =
-                __float2half_rn(0.5f * (hp + hm));
-            *reinterpret_cast<__half*>(smem + g.op + kmajor_offset(g.Bp + b, g.Ek + U, g.K)) =
-                __float2half_rn(0.5f * (hp - hm));
-          }
-        }
-      }
-    }
-    if (!fine) atomicCAS(a.status, 0, kStatusTimeout);
-    tc_fence_before();
-    ok = (__syncthreads_and(fine) != 0) && ok;
   }
+  if (!fine) atomicCAS(a.status, 0, kStatusTimeout);
+  tc_fence_before();
+  ok = (__syncthreads_and(fine) != 0) && ok;
 
   // ---- losses and coefficient of the pair (fp64 sums, sequences in order)
   if (tid == 0) {
@@ -492,7 +515,9 @@ bool res_supported(const Layout& lay, int B) {
   if (B < 1 || B > kResMaxBp || lay.H > 64) return false;
   const ResGeom g = make_res_geom(lay, B, 1);
   // one thread gathers each 8-column chunk of the embedding operand
-  return g.bytes <= kResMaxSmem && 2 * g.Bp * (g.Ek / 8) <= kResEpiWarps * 32;
+  // and the gate plus two head accumulators fit the 512 TMEM columns
+  return g.bytes <= kResMaxSmem && 2 * g.Bp * (g.Ek / 8) <= kResEpiWarps * 32 &&
+         (g.MTg + 4) * 4 * g.Bp <= 512;
 }
 
 cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, float* coef_out,
