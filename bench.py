@@ -47,6 +47,15 @@ TRAFFIC = {
     "soma_n2": {"bytes_per_launch": 64.078848e6 + 5.233920e6,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
                 "source_hash": "58cd4ba846f2a849"},
+    # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
+    "soma_n256": {"bytes_per_launch": 39.559168e6 + 2304,
+                  "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
+                  "source_hash": "dcb065c9f93e4ce8"},
+    # profiles/body_tc_kernel_body_n256.md: one full-size launch (T=512)
+    "body_n256": {"bytes_per_launch": 36.064512e6,
+                  "files": ["body_tc.cu", "body_device.cuh", "tc_primitives.cuh",
+                            "soma_device.cuh"],
+                  "source_hash": "b42810e86a76a58b"},
 }
 
 
@@ -535,10 +544,6 @@ def body_flops_per_token(c):
     return c["D"] * (2 * 2 * d * 4 * d + 2 * 2 * d * 4 * d) + 2 * d * 256
 
 
-# fp32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flops x 2.07 GHz
-FP32_SIMT_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
-
-
 def body_cpu_baseline(cfg_name, c, n_seqs, kind):
     import oracle
     from paper_2609_37899_gb300 import inputs
@@ -698,7 +703,7 @@ def body_arm(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": W, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "vs_baseline": None, "dtype": DTYPE, "data": "synthetic",
         "steps_per_s": K / (ms / 1e3),
         "config": {
             "workload": body_desc(args.config, c),
@@ -713,13 +718,12 @@ def body_arm(args):
                            "replica(s), no collective",
         },
         "roofline": {
-            "bound": "alu", "kernel": "body_sweep_kernel (fp32 CUDA cores, one CTA per sign of "
-                                      "a probe pair, whole recurrence resident)",
-            "achieved": achieved, "peak": FP32_SIMT_TFLOPS, "unit": "TFLOP/s",
-            "frac": (achieved / FP32_SIMT_TFLOPS) if achieved else None, "traffic": traffic,
-            "peak_source": "fp32 FMA peak of the CUDA cores: 152 SMs x 128 lanes x 2 flops x "
-                           "2.07 GHz (the kernel issues fp32 FMAs, not tensor-core MMAs)",
-            "frac_of_tensor_peak": (achieved / tensor_peak) if achieved else None,
+            "bound": "tensor", "kernel": "body_tc_kernel (tcgen05, one CTA per probe pair and "
+                                         "16-sequence chunk, the whole recurrence resident; "
+                                         "its time includes the decode and the loss)",
+            "achieved": achieved, "peak": tensor_peak, "unit": "TFLOP/s",
+            "frac": (achieved / tensor_peak) if achieved else None, "traffic": traffic,
+            "peak_source": f"{peak_src} bf16 dense sustained (MEASURED_PEAKS.json)",
             "flops_per_token": body_flops_per_token(c),
             "launches": sweep_n,
             "kernel_ms_per_launch": sweep_ms / sweep_n if sweep_n else None,

@@ -305,8 +305,10 @@ int soma_spsa_step_static(float* params, int n_experts, soma_dims d, int n_pert,
  * sign, every weight the sparse probe (same Philox stream and bit map as
  * above, keyed by the flat body coordinate).
  * Supported: vocab 256, width 32, blocks 1 or 2; else SOMA_ERR_UNSUPPORTED.
- * The forward runs on CUDA cores in fp32 (losses summed in fp64); one CTA
- * runs one sign of one (expert, probe) pair over up to 16 sequences. */
+ * The forward runs on the tensor cores: one CTA per (expert, probe) pair and
+ * chunk of up to 16 sequences, both signs in one mean/difference pass, fp16
+ * operands split into hi + lo parts, fp32 accumulation and epilogues, losses
+ * summed in fp64. */
 typedef struct soma_body_dims {
   int32_t vocab;  /* must be 256 */
   int32_t width;  /* d = d_t = d_E */

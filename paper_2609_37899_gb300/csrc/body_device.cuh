@@ -10,6 +10,7 @@ namespace soma {
 
 constexpr int kBodyWidth = 32;     // d_t = d_E of the width-32 ensembles
 constexpr int kBodyMaxBlocks = 2;  // D
+constexpr int kBodyRows = 16;      // sequences of one CTA of the forward sweep
 
 // M_body = 16 D d^2 + (2D + 1) d: per block W_ih, W_hh, W_1 [4d][d] and
 // W_2 [d][4d]; then the gains ga_k, gb_k of every block and the final gf.

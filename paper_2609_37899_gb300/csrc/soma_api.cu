@@ -579,8 +579,8 @@ int body_forward(float* params, int n_experts, soma_body_dims d, const float* he
   cudaStream_t st = (cudaStream_t)stream;
   double* partial = static_cast<double*>(workspace);
   float* coef_ws = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + w.partial);
-  cudaError_t e = launch_body_sweep(params, head, byte_batch, n_experts, d.blocks, n_pert, 2,
-                                    batch, seq_len, eps, probe_kind, seed, step, partial, st);
+  cudaError_t e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, n_pert, 2, batch,
+                                 seq_len, eps, probe_kind, seed, step, partial, status, st);
   if (e == cudaSuccess)
     e = launch_body_reduce(partial, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
                            coef_out, coef_ws, status, st);
@@ -640,8 +640,8 @@ int soma_body_eval_loss(const float* params, int n_experts, soma_body_dims d, co
   if (!status) return SOMA_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)stream;
   double* partial = static_cast<double*>(workspace);
-  cudaError_t e = launch_body_sweep(params, head, byte_batch, n_experts, d.blocks, 1, 1, batch,
-                                    seq_len, 0.f, 0, 0, 0, partial, st);
+  cudaError_t e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, 1, 1, batch,
+                                 seq_len, 0.f, 0, 0, 0, partial, status, st);
   if (e == cudaSuccess)
     e = launch_body_reduce(partial, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
                            nullptr, status, st);

@@ -110,14 +110,16 @@ cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& 
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                                const float* coef, const AdamArgs& h, cudaStream_t stream);
 
-// The paper's expert body (body.cu): width kBodyWidth, 1 <= blocks <=
-// kBodyMaxBlocks.  partial [N * n * n_sign][ceil(B / 16)] fp64 NLL sums.
-size_t body_smem_bytes();
+// The paper's expert body (body.cu, body_tc.cu): width kBodyWidth, 1 <=
+// blocks <= kBodyMaxBlocks.  partial [N * n * n_sign][ceil(B / 16)] fp64 NLL sums.
 int body_rows_per_cta();
-cudaError_t launch_body_sweep(const float* params, const float* head, const uint8_t* bytes,
-                              int n_experts, int blocks, int n_pert, int n_sign, int B, int T,
-                              float eps, int sparse, uint64_t seed, uint64_t step,
-                              double* partial, cudaStream_t stream);
+// The antithetic forwards on the tensor cores (body_tc.cu): one CTA per
+// (expert, probe) pair and 16-sequence chunk, both signs in the
+// mean/difference form.
+cudaError_t launch_body_tc(const float* params, const float* head, const uint8_t* bytes,
+                           int n_experts, int blocks, int n_pert, int n_sign, int B, int T,
+                           float eps, int sparse, uint64_t seed, uint64_t step, double* partial,
+                           int* status, cudaStream_t stream);
 cudaError_t launch_body_reduce(const double* partial, int pairs, int n_sign, int B, int T,
                                float eps, float* losses_out, float* coef_out, float* coef_ws,
                                int* status, cudaStream_t stream);
