@@ -60,6 +60,7 @@ constexpr float kLnEps = 1e-5f;
 constexpr uint32_t kGateTile = 128u * 64 * 2;   // [W_ih | W_hh] gate-major, K = 64
 constexpr uint32_t kMlp1Tile = 128u * 32 * 2;   // W_1, K = 32
 constexpr uint32_t kMlp2Tile = 32u * 128 * 2;   // W_2 as the B operand: 32 rows, K = 128
+                                                // (Z_2 right after it: one 64-row operand)
 constexpr uint32_t kBlockBytes = 2 * (kGateTile + kMlp1Tile + kMlp2Tile);  // W and Z
 constexpr uint32_t kSmBlk = 0;                                     // [D][W/Z tiles]
 constexpr uint32_t kSmE = kSmBlk + kBodyMaxBlocks * kBlockBytes;   // E_hi, E_lo: [2][2 tiles][128][32]
@@ -484,7 +485,9 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
         }
       }
       phase_barrier();
-      // ---- MLP2: [mbar | dm] (rows) x W_2^T -----------------------------------
+      // ---- MLP2: [mbar | dm] (rows) x [W_2 ; Z_2]^T ------------------------
+      // W_2 and Z_2 are adjacent 32-row B tiles, i.e. one 64-row B operand:
+      // one MMA of N = 64 gives W_2 m (columns 0-31) and Z_2 m (32-63)
       if (warp == kMmaWarp) {
         if (lane == 0) {
           const uint32_t oa = lo(kSmO3);
@@ -492,9 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
 #pragma unroll
           for (int k16 = 0; k16 < 8; ++k16) {
             const uint32_t ko = 16u * k16, accf = k16 > 0;
-            mma_f16_ss_lohi(tmem + kTW, oa + ko, hi128, wb + ko, hi128, idesc32, accf);
-            mma_f16_ss_lohi(tmem + kTZ, oa + ko, hi128, wb + (kMlp2Tile >> 4) + ko, hi128,
-                            idesc32, accf);
+            mma_f16_ss_lohi(tmem + kTW, oa + ko, hi128, wb + ko, hi128, idesc64, accf);
           }
           mma_commit(mma_bar);
         }
@@ -508,7 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
 #pragma unroll
           for (int cg = 0; cg < 2; ++cg) {
             const uint32_t col = (uint32_t)(8 * sg + 4 * cg);
-            const uint32_t tw = tmem + kTW + col, tz = tmem + kTZ + col;
+            const uint32_t tw = tmem + kTW + col, tz = tw + kD;
             uint32_t wm[2], wdd[2], zm[2], zdd[2];
             tmem_ld_16x128b(tw, wm[0], wm[1]);
             tmem_ld_16x128b(tw + (16u << 16), wdd[0], wdd[1]);
