@@ -52,10 +52,10 @@ TRAFFIC = {
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
                   "source_hash": "dcb065c9f93e4ce8"},
     # profiles/body_tc_kernel_body_n256.md: one full-size launch (T=512)
-    "body_n256": {"bytes_per_launch": 36.064512e6,
+    "body_n256": {"bytes_per_launch": 36.277248e6,
                   "files": ["body_tc.cu", "body_device.cuh", "tc_primitives.cuh",
                             "soma_device.cuh"],
-                  "source_hash": "b42810e86a76a58b"},
+                  "source_hash": "16c79df5bb237a1f"},
 }
 
 

@@ -5,10 +5,9 @@
 // (logits = E y).  Only the body is perturbed.  The antithetic forwards run
 // in body_tc.cu; this file holds the rest of the step.
 //
-// Kernels:
-//   body_reduce_kernel  L+-, the coefficients (L+ - L-) / (2 eps) in fp64.
-//   body_sgd_kernel     theta -= lr (1/n) sum_i c_i z_i (Eq. main-spsa).
-//   body_adam_kernel    Eq. localspsa with coupled weight decay.
+// Kernels: body_reduce_kernel (L+-, the coefficients (L+ - L-) / (2 eps) in
+// fp64) and the probe debug kernel; the SGD and Adam updates are the LSTM
+// expert's (spsa_misc.cu) under the body's probe law.
 //
 // Probe law (App. E): normalisation gains take the dense sign; every other
 // coordinate is the dense sign where the activity stream's bit is set, else
@@ -51,99 +50,6 @@ __global__ void body_reduce_kernel(const double* __restrict__ partial, int pairs
   if (!finite && status) atomicCAS(status, 0, kStatusNonFinite);
 }
 
-constexpr int kUpd = 128;
-
-// theta[e][p] -= lr (1/n) sum_i coef[e][i] z_{e,i}[p]; thread q owns the 32
-// coordinates 32q .. 32q + 31.  An expert with a non-finite coefficient is
-// left unchanged.
-__global__ void __launch_bounds__(kUpd) body_sgd_kernel(float* __restrict__ params, int64_t P,
-                                                        int64_t goff, int n_pert, int sparse,
-                                                        float lr, uint64_t seed, uint64_t step,
-                                                        const float* __restrict__ coef) {
-  extern __shared__ float cf[];
-  __shared__ int all_finite;
-  const int e = blockIdx.y;
-  if (threadIdx.x == 0) all_finite = 1;
-  __syncthreads();
-  for (int i = threadIdx.x; i < n_pert; i += kUpd) {
-    const float c = coef[(int64_t)e * n_pert + i];
-    cf[i] = c;
-    if (!isfinite(c)) all_finite = 0;
-  }
-  __syncthreads();
-  if (!all_finite) return;
-  const int64_t q = (int64_t)blockIdx.x * kUpd + threadIdx.x;
-  const int64_t p0 = q * 32;
-  if (p0 >= P) return;
-  float acc[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-  for (int i = 0; i < n_pert; ++i) {
-    uint32_t neg, act;
-    body_probe_words(make_probe_key(seed, step, (uint32_t)e, (uint32_t)i), (int)q, sparse, goff,
-                     neg, act);
-    const float c = cf[i];
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
-  }
-  const float scale = lr / (float)n_pert;
-  float* th = params + (int64_t)e * P + p0;
-  const int cnt = P - p0 < 32 ? (int)(P - p0) : 32;
-  for (int j = 0; j < cnt; ++j) th[j] -= scale * acc[j];
-}
-
-// Eq. localspsa: the estimate averaged over n_acc batches, coupled decay,
-// bias-corrected Adam moments.
-__global__ void __launch_bounds__(kUpd) body_adam_kernel(float* __restrict__ params,
-                                                         float* __restrict__ m,
-                                                         float* __restrict__ v, int64_t P,
-                                                         int64_t goff, int n_experts, int n_pert,
-                                                         int sparse, uint64_t seed, AdamSteps st,
-                                                         const float* __restrict__ coef,
-                                                         AdamArgs h) {
-  __shared__ int all_finite;
-  const int e = blockIdx.y;
-  if (threadIdx.x == 0) all_finite = 1;
-  __syncthreads();
-  for (int j = threadIdx.x; j < st.n_acc * n_pert; j += kUpd) {
-    const int aa = j / n_pert, i = j % n_pert;
-    if (!isfinite(coef[((int64_t)aa * n_experts + e) * n_pert + i])) all_finite = 0;
-  }
-  __syncthreads();
-  if (!all_finite) return;
-  const int64_t q = (int64_t)blockIdx.x * kUpd + threadIdx.x;
-  const int64_t p0 = q * 32;
-  if (p0 >= P) return;
-  float acc[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-  for (int aa = 0; aa < st.n_acc; ++aa) {
-    const float* ca = coef + ((int64_t)aa * n_experts + e) * n_pert;
-    for (int i = 0; i < n_pert; ++i) {
-      uint32_t neg, act;
-      body_probe_words(make_probe_key(seed, st.step[aa], (uint32_t)e, (uint32_t)i), (int)q,
-                       sparse, goff, neg, act);
-      const float c = ca[i];
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
-    }
-  }
-  const float inv = 1.f / ((float)st.n_acc * (float)n_pert);
-  const int64_t base = (int64_t)e * P + p0;
-  const int cnt = P - p0 < 32 ? (int)(P - p0) : 32;
-  for (int j = 0; j < cnt; ++j) {
-    const float w = params[base + j];
-    const float g = fmaf(h.wd, w, acc[j] * inv);
-    const float mj = fmaf(h.b1, m[base + j], (1.f - h.b1) * g);
-    const float vj = fmaf(h.b2, v[base + j], (1.f - h.b2) * g * g);
-    m[base + j] = mj;
-    v[base + j] = vj;
-    params[base + j] = w - h.lr * (mj * h.inv_bc1) / (sqrtf(vj * h.inv_bc2) + h.delta);
-  }
-}
-
 // z[p - p0] for p in [p0, p0 + count): thread w handles run (p0 >> 5) + w.
 __global__ void debug_body_probe_kernel(ProbeKey pk, int sparse, int64_t goff, int64_t p0,
                                         int64_t count, int8_t* z) {
@@ -178,27 +84,16 @@ cudaError_t launch_body_reduce(const double* partial, int pairs, int n_sign, int
 cudaError_t launch_body_sgd(float* params, int n_experts, int blocks, int n_pert, int sparse,
                             float lr, uint64_t seed, uint64_t step, const float* coef,
                             cudaStream_t stream) {
-  const int64_t P = body_param_count(kD, blocks);
-  const int64_t words = (P + 31) / 32;
-  dim3 grid((unsigned)((words + kUpd - 1) / kUpd), n_experts);
-  trace_begin(SOMA_TRACE_UPDATE, stream);
-  body_sgd_kernel<<<grid, kUpd, n_pert * sizeof(float), stream>>>(
-      params, P, body_gain_offset(kD, blocks), n_pert, sparse, lr, seed, step, coef);
-  trace_end(SOMA_TRACE_UPDATE, stream);
-  return cudaGetLastError();
+  return launch_sgd_update(params, body_param_count(kD, blocks), body_gain_offset(kD, blocks),
+                           n_experts, n_pert, sparse, lr, seed, step, coef, stream);
 }
 
 cudaError_t launch_body_adam(float* params, float* m, float* v, int n_experts, int blocks,
                              int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                              const float* coef, const AdamArgs& h, cudaStream_t stream) {
-  const int64_t P = body_param_count(kD, blocks);
-  const int64_t words = (P + 31) / 32;
-  dim3 grid((unsigned)((words + kUpd - 1) / kUpd), n_experts);
-  trace_begin(SOMA_TRACE_UPDATE, stream);
-  body_adam_kernel<<<grid, kUpd, 0, stream>>>(params, m, v, P, body_gain_offset(kD, blocks),
-                                              n_experts, n_pert, sparse, seed, steps, coef, h);
-  trace_end(SOMA_TRACE_UPDATE, stream);
-  return cudaGetLastError();
+  return launch_probe_adam(params, m, v, body_param_count(kD, blocks),
+                           body_gain_offset(kD, blocks), n_experts, n_pert, sparse, seed, steps,
+                           coef, h, stream);
 }
 
 cudaError_t launch_debug_body_probe(uint64_t seed, uint64_t step, int expert, int pert, int blocks,

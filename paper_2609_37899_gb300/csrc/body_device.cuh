@@ -4,6 +4,7 @@
 
 #include <cstdint>
 
+#include "probe_law.cuh"
 #include "soma_device.cuh"
 
 namespace soma {
@@ -21,23 +22,11 @@ __host__ __device__ inline int64_t body_param_count(int d, int D) {
 // First normalisation-gain coordinate: every coordinate from here on is a gain.
 __host__ __device__ inline int64_t body_gain_offset(int d, int D) { return 16LL * D * d * d; }
 
-// Sign and activity words of the 32 coordinates 32q .. 32q + 31 in natural
-// order (bit j <=> coordinate 32q + j): neg bit set <=> z = -1, act bit
-// clear <=> z = 0.  Dense probes are active everywhere.  The sparse law
-// (App. E) takes the activity stream on weights and keeps every gain active.
+// The body's probe law: sparse on the weights, dense on the gains.
 __host__ __device__ __forceinline__ void body_probe_words(const ProbeKey& pk, int q, int sparse,
                                                           int64_t goff, uint32_t& neg,
                                                           uint32_t& act) {
-  neg = raw_to_natural(probe_raw_word(pk, (uint32_t)q));
-  act = 0xFFFFFFFFu;
-  if (sparse) {
-    act = raw_to_natural(probe_raw_word(activity_key(pk), (uint32_t)q));
-    const int64_t from = goff - 32LL * q;  // offset of the first gain inside the run
-    if (from <= 0)
-      act = 0xFFFFFFFFu;
-    else if (from < 32)
-      act |= 0xFFFFFFFFu << from;
-  }
+  probe_law_words(pk, q, sparse, goff, neg, act);
 }
 
 }  // namespace soma

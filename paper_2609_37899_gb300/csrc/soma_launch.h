@@ -69,6 +69,11 @@ cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B,
 cudaError_t launch_spsa_update(float* params, const Layout& lay, int n_experts, int n_pert,
                                float lr, uint64_t seed, uint64_t step, const float* coef,
                                cudaStream_t stream);
+// The update under a probe law (probe_law.cuh): sparse probes are dense from
+// coordinate dense_from on (the LSTM expert passes P).
+cudaError_t launch_sgd_update(float* params, int64_t P, int64_t dense_from, int n_experts,
+                              int n_pert, int sparse, float lr, uint64_t seed, uint64_t step,
+                              const float* coef, cudaStream_t stream);
 cudaError_t launch_init(float* params, const Layout& lay, int n_experts, uint64_t seed, float std,
                         cudaStream_t stream);
 cudaError_t launch_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
@@ -109,6 +114,10 @@ cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cuda
 cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                                const float* coef, const AdamArgs& h, cudaStream_t stream);
+cudaError_t launch_probe_adam(float* params, float* m, float* v, int64_t P, int64_t dense_from,
+                              int n_experts, int n_pert, int sparse, uint64_t seed,
+                              const AdamSteps& steps, const float* coef, const AdamArgs& h,
+                              cudaStream_t stream);
 
 // The paper's expert body (body.cu, body_tc.cu): width kBodyWidth, 1 <=
 // blocks <= kBodyMaxBlocks.  partial [N * n * n_sign][ceil(B / 16)] fp64 NLL sums.

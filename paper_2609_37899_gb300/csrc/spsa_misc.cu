@@ -1,6 +1,7 @@
 // spsa_misc.cu -- the loss reduction, the SPSA update, the parameter
 // initialisation and the generator test kernels.
 #include "soma_api.h"
+#include "probe_law.cuh"
 #include "soma_launch.h"
 
 namespace soma {
@@ -60,14 +61,15 @@ reduce_losses_kernel(const float* __restrict__ nll, int n_sign, int BT, float ep
 
 constexpr int kUpdThreads = 128;
 
-// theta[e][p] -= lr * (1/n) * sum_i coef[e][i] z_{e,i}[p].  Thread q of
-// expert e owns the 32 parameters 32q .. 32q + 31, whose probe bits are one
-// raw 32-bit Philox output word for every probe (read in the run's bit
-// order, which the unrolled loop resolves at compile time).  An expert whose coefficients
-// are not all finite is left unchanged.
+// theta[e][p] -= lr * (1/n) * sum_i coef[e][i] z_{e,i}[p] (Eq. main-spsa).
+// Thread q of expert e owns the 32 parameters 32q .. 32q + 31, whose probe
+// bits are one Philox word per probe (two for sparse probes), under the probe
+// law of probe_law_words.  An expert whose coefficients are not all finite is
+// left unchanged.
 __global__ void __launch_bounds__(kUpdThreads)
-spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr, uint64_t seed,
-                   uint64_t step, const float* __restrict__ coef) {
+sgd_update_kernel(float* __restrict__ params, int64_t P, int64_t dense_from, int n_pert,
+                  int sparse, float lr, uint64_t seed, uint64_t step,
+                  const float* __restrict__ coef) {
   extern __shared__ float cf[];  // [n_pert]
   __shared__ int all_finite;
   const int e = blockIdx.y;
@@ -82,21 +84,23 @@ spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr,
   if (!all_finite) return;
   const int64_t q = (int64_t)blockIdx.x * kUpdThreads + threadIdx.x;
   const int64_t p0 = q * 32;
-  if (p0 >= lay.P) return;
+  if (p0 >= P) return;
   float acc[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   for (int i = 0; i < n_pert; ++i) {
-    const ProbeKey pk = make_probe_key(seed, step, (uint32_t)e, (uint32_t)i);
-    const uint32_t raw = probe_raw_word(pk, (uint32_t)(p0 >> 5));  // p0 is 32-aligned
+    uint32_t neg, act;
+    probe_law_words(make_probe_key(seed, step, (uint32_t)e, (uint32_t)i), (int)q, sparse,
+                    dense_from, neg, act);
     const float c = cf[i];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) acc[j] += ((raw >> raw_bit(j)) & 1u) ? -c : c;
+    for (int j = 0; j < 32; ++j)
+      if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
   }
   const float scale = lr / (float)n_pert;
-  float* th = params + (int64_t)e * lay.P + p0;
-  if (p0 + 32 <= lay.P) {
-    // P is a multiple of 4 and p0 of 32: 16-byte aligned
+  float* th = params + (int64_t)e * P + p0;
+  if (p0 + 32 <= P && (P & 3) == 0) {
+    // P a multiple of 4 and p0 of 32: 16-byte aligned
 #pragma unroll
     for (int j4 = 0; j4 < 8; ++j4) {
       float4 v = reinterpret_cast<float4*>(th)[j4];
@@ -107,7 +111,7 @@ spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr,
       reinterpret_cast<float4*>(th)[j4] = v;
     }
   } else {
-    for (int j = 0; j < 32 && p0 + j < lay.P; ++j) th[j] -= scale * acc[j];
+    for (int j = 0; j < 32 && p0 + j < P; ++j) th[j] -= scale * acc[j];
   }
 }
 
@@ -115,14 +119,14 @@ spsa_update_kernel(float* __restrict__ params, Layout lay, int n_pert, float lr,
 //   g = (1/(A n)) sum_a sum_i coef[a][e][i] z_{e,i}^{(a)} + wd * theta,
 //   m = b1 m + (1 - b1) g,  v = b2 v + (1 - b2) g^2,
 //   theta -= lr * (m / bc1) / (sqrt(v / bc2) + delta),
-// with z^{(a)} drawn with step counter steps[a] (dense or sparse).  As in the
-// SGD kernel, thread q owns the 32 parameters 32q .. 32q + 31 and reads one
-// raw Philox word per probe (two for sparse probes).  An expert whose
-// coefficients are not all finite is left unchanged, moments included.
+// with z^{(a)} drawn with step counter steps[a] under the probe law of
+// probe_law_words.  Thread q owns the 32 parameters 32q .. 32q + 31.  An
+// expert whose coefficients are not all finite is left unchanged, moments
+// included.
 __global__ void __launch_bounds__(kUpdThreads)
 adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __restrict__ v,
-                   Layout lay, int n_experts, int n_pert, int sparse, uint64_t seed,
-                   AdamSteps steps, const float* __restrict__ coef, AdamArgs h) {
+                   int64_t P, int64_t dense_from, int n_experts, int n_pert, int sparse,
+                   uint64_t seed, AdamSteps steps, const float* __restrict__ coef, AdamArgs h) {
   __shared__ int all_finite;
   const int e = blockIdx.y;
   if (threadIdx.x == 0) all_finite = 1;
@@ -135,28 +139,25 @@ adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __r
   if (!all_finite) return;
   const int64_t q = (int64_t)blockIdx.x * kUpdThreads + threadIdx.x;
   const int64_t p0 = q * 32;
-  if (p0 >= lay.P) return;
+  if (p0 >= P) return;
   float acc[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   for (int a = 0; a < steps.n_acc; ++a) {
     const float* ca = coef + ((int64_t)a * n_experts + e) * n_pert;
     for (int i = 0; i < n_pert; ++i) {
-      const ProbeKey pk = make_probe_key(seed, steps.step[a], (uint32_t)e, (uint32_t)i);
-      const uint32_t w = (uint32_t)(p0 >> 5);  // p0 is 32-aligned
-      const uint32_t raw = probe_raw_word(pk, w);
-      const uint32_t act = sparse ? probe_raw_word(activity_key(pk), w) : 0xFFFFFFFFu;
+      uint32_t neg, act;
+      probe_law_words(make_probe_key(seed, steps.step[a], (uint32_t)e, (uint32_t)i), (int)q,
+                      sparse, dense_from, neg, act);
       const float c = ca[i];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const uint32_t rb = (uint32_t)raw_bit(j);
-        if ((act >> rb) & 1u) acc[j] += ((raw >> rb) & 1u) ? -c : c;
-      }
+      for (int j = 0; j < 32; ++j)
+        if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
     }
   }
   const float inv = 1.f / ((float)steps.n_acc * (float)n_pert);
-  const int64_t base = (int64_t)e * lay.P + p0;
-  const int cnt = lay.P - p0 < 32 ? (int)(lay.P - p0) : 32;
+  const int64_t base = (int64_t)e * P + p0;
+  const int cnt = P - p0 < 32 ? (int)(P - p0) : 32;
   for (int j = 0; j < cnt; ++j) {
     const float th = params[base + j];
     const float g = fmaf(h.wd, th, acc[j] * inv);
@@ -249,16 +250,23 @@ cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B,
   return cudaGetLastError();
 }
 
+cudaError_t launch_sgd_update(float* params, int64_t P, int64_t dense_from, int n_experts,
+                              int n_pert, int sparse, float lr, uint64_t seed, uint64_t step,
+                              const float* coef, cudaStream_t stream) {
+  const int64_t words = (P + 31) / 32;
+  dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
+  trace_begin(SOMA_TRACE_UPDATE, stream);
+  sgd_update_kernel<<<grid, kUpdThreads, n_pert * sizeof(float), stream>>>(
+      params, P, dense_from, n_pert, sparse, lr, seed, step, coef);
+  trace_end(SOMA_TRACE_UPDATE, stream);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_spsa_update(float* params, const Layout& lay, int n_experts, int n_pert,
                                float lr, uint64_t seed, uint64_t step, const float* coef,
                                cudaStream_t stream) {
-  const int64_t words = (lay.P + 31) / 32;
-  dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
-  trace_begin(SOMA_TRACE_UPDATE, stream);
-  spsa_update_kernel<<<grid, kUpdThreads, n_pert * sizeof(float), stream>>>(params, lay, n_pert,
-                                                                             lr, seed, step, coef);
-  trace_end(SOMA_TRACE_UPDATE, stream);
-  return cudaGetLastError();
+  return launch_sgd_update(params, lay.P, lay.P, n_experts, n_pert, 0, lr, seed, step, coef,
+                           stream);
 }
 
 cudaError_t launch_init(float* params, const Layout& lay, int n_experts, uint64_t seed, float std,
@@ -291,16 +299,24 @@ cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cuda
   return cudaGetLastError();
 }
 
+cudaError_t launch_probe_adam(float* params, float* m, float* v, int64_t P, int64_t dense_from,
+                              int n_experts, int n_pert, int sparse, uint64_t seed,
+                              const AdamSteps& steps, const float* coef, const AdamArgs& h,
+                              cudaStream_t stream) {
+  const int64_t words = (P + 31) / 32;
+  dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
+  trace_begin(SOMA_TRACE_UPDATE, stream);
+  adam_update_kernel<<<grid, kUpdThreads, 0, stream>>>(params, m, v, P, dense_from, n_experts,
+                                                       n_pert, sparse, seed, steps, coef, h);
+  trace_end(SOMA_TRACE_UPDATE, stream);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& lay, int n_experts,
                                int n_pert, int sparse, uint64_t seed, const AdamSteps& steps,
                                const float* coef, const AdamArgs& h, cudaStream_t stream) {
-  const int64_t words = (lay.P + 31) / 32;
-  dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
-  trace_begin(SOMA_TRACE_UPDATE, stream);
-  adam_update_kernel<<<grid, kUpdThreads, 0, stream>>>(params, m, v, lay, n_experts, n_pert, sparse,
-                                                       seed, steps, coef, h);
-  trace_end(SOMA_TRACE_UPDATE, stream);
-  return cudaGetLastError();
+  return launch_probe_adam(params, m, v, lay.P, lay.P, n_experts, n_pert, sparse, seed, steps,
+                           coef, h, stream);
 }
 
 }  // namespace soma
