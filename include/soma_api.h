@@ -258,6 +258,13 @@ int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, in
                           int64_t count, int8_t* z_out, void* stream);
 int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int probe_kind,
                      int64_t p0, int64_t count, int8_t* z_out, void* stream);
+/* soma_debug_wait_timeout: one kernel waits on a barrier that nothing
+ *   completes.  Its bounded wait gives up after max_polls polls (1 ..
+ *   2^22; each poll suspends for at most ~100 ns) and records
+ *   SOMA_ERR_TIMEOUT in the status word, which soma_get_status() then
+ *   returns; the context stays usable.  This is the path every kernel of the
+ *   library takes when one of its waits runs out. */
+int soma_debug_wait_timeout(uint32_t max_polls, void* stream);
 /* soma_debug_tc_gemm: d[128][n] = a[128][k] * b[n][k]^T (fp16 inputs as
  *   uint16 bit patterns, row-major; fp32 output) through the same shared-
  *   memory descriptors, tcgen05.mma and tensor-memory read-back as the

@@ -107,6 +107,7 @@ def lib():
         _sig(L, "soma_spsa_estimate_opts", i32, [vp, i32, soma_dims, i32,
                                                  ctypes.POINTER(soma_estimate_options), f32, u64,
                                                  u64, vp, i32, i32, vp, vp, vp, sz, vp])
+        _sig(L, "soma_debug_wait_timeout", i32, [ctypes.c_uint32, vp])
         bd = soma_body_dims
         _sig(L, "soma_body_param_count", i64, [bd])
         _sig(L, "soma_body_workspace_bytes", sz, [bd, i32, i32, i32, i32])
@@ -319,6 +320,11 @@ def debug_probe(seed: int, step: int, expert: int, probe: int, kind: str, p0: in
                                   _dev(z, torch.int8, "z"), _stream(stream)),
            "soma_debug_probe")
     return z
+
+
+def debug_wait_timeout(max_polls: int, stream=None):
+    """Launch a kernel whose bounded wait runs out (see soma_api.h)."""
+    _check(lib().soma_debug_wait_timeout(max_polls, _stream(stream)), "soma_debug_wait_timeout")
 
 
 def debug_tc_gemm(a: torch.Tensor, b: torch.Tensor, stream=None) -> torch.Tensor:

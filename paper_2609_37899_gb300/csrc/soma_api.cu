@@ -385,6 +385,13 @@ int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, in
   return cuda_status(launch_debug_tc_gemm(a, b, d, n, k, status, (cudaStream_t)stream));
 }
 
+int soma_debug_wait_timeout(uint32_t max_polls, void* stream) {
+  if (max_polls < 1 || max_polls > (1u << 22)) return SOMA_ERR_INVALID_ARG;
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  return cuda_status(launch_debug_wait_timeout(max_polls, status, (cudaStream_t)stream));
+}
+
 int soma_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int64_t p0,
                           int64_t count, int8_t* z_out, void* stream) {
   if (!z_out || count < 0 || p0 < 0 || expert < 0 || pert < 0) return SOMA_ERR_INVALID_ARG;

@@ -76,6 +76,7 @@ cudaError_t launch_sgd_update(float* params, int64_t P, int64_t dense_from, int 
                               const float* coef, cudaStream_t stream);
 cudaError_t launch_init(float* params, const Layout& lay, int n_experts, uint64_t seed, float std,
                         cudaStream_t stream);
+cudaError_t launch_debug_wait_timeout(uint32_t max_polls, int* status, cudaStream_t stream);
 cudaError_t launch_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
                                 cudaStream_t stream);
 cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int sparse,

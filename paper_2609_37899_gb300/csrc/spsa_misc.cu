@@ -3,6 +3,7 @@
 #include "soma_api.h"
 #include "probe_law.cuh"
 #include "soma_launch.h"
+#include "tc_primitives.cuh"
 
 namespace soma {
 
@@ -238,6 +239,20 @@ __global__ void debug_rademacher_kernel(ProbeKey pk, int sparse, int64_t p0, int
     z[q0 + j] = ((bits.act >> j) & 1u) ? (((bits.neg >> j) & 1u) ? -1 : 1) : 0;
 }
 
+
+// A wait that nothing completes.  The bounded wait gives up after max_polls
+// polls and the kernel records SOMA_ERR_TIMEOUT, as every kernel of the
+// library does when one of its waits runs out; the context stays usable.
+__global__ void debug_wait_timeout_kernel(uint32_t max_polls, int* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    tc::mbar_fence_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !tc::mbar_wait(&bar, 0u, max_polls))
+    atomicCAS(status, 0, kStatusTimeout);
+}
 }  // namespace
 
 cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B, int T, float eps,
@@ -317,6 +332,11 @@ cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& 
                                const float* coef, const AdamArgs& h, cudaStream_t stream) {
   return launch_probe_adam(params, m, v, lay.P, lay.P, n_experts, n_pert, sparse, seed, steps,
                            coef, h, stream);
+}
+
+cudaError_t launch_debug_wait_timeout(uint32_t max_polls, int* status, cudaStream_t stream) {
+  debug_wait_timeout_kernel<<<1, 32, 0, stream>>>(max_polls, status);
+  return cudaGetLastError();
 }
 
 }  // namespace soma

@@ -167,4 +167,6 @@ def test_body_sizes_and_validation(soma):
     assert L.soma_body_adam_update(fake, fake, fake, 1, d, 4, 1, 0, steps, 1, fake, cfg,
                                    None) == 1
     assert L.soma_debug_body_probe(0, 0, 0, 0, d, 1, -1, 4, fake, None) == 1
+    assert L.soma_debug_wait_timeout(0, None) == 1
+    assert L.soma_debug_wait_timeout((1 << 22) + 1, None) == 1
     assert L.soma_debug_body_probe(0, 0, 0, 0, d, 1, 1 << 30, 4, fake, None) == 1
