@@ -44,9 +44,9 @@ UNIT = "perturbed tokens/s"
 TRAFFIC = {
     # profiles/tc_persistent_kernel_soma_n2.md: the gate launch, captured on
     # the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
-    "soma_n2": {"bytes_per_launch": 64.078848e6 + 5.233920e6,
+    "soma_n2": {"bytes_per_launch": 64.062720e6 + 5.382400e6,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "58cd4ba846f2a849"},
+                "source_hash": "3e7bcb1f936434e5"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
     "soma_n256": {"bytes_per_launch": 39.559168e6 + 2304,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],

@@ -116,8 +116,12 @@ __device__ __forceinline__ uint32_t z_run_raw(const ProbeKey& pk, int64_t p0, ZS
 template <bool SPARSE, int J>
 __device__ __forceinline__ uint32_t z_pair(uint32_t raw, uint32_t act) {
   if (!SPARSE) return pm_pair<J>(raw, 0x3C003C00u);
-  const uint32_t a = (act << (15 - J)) & 0x80008000u;  // activity at the sign positions
-  return ((raw << (15 - J)) & 0x80008000u) | (0x3C003C00u & (a - (a >> 15)));
+  // activity bits at the sign positions (bits 15 and 31), each spread over
+  // its 16-bit half by a byte permute that replicates the top bit of bytes 1
+  // and 3: a mask of 1.0 magnitudes where the coordinate is active
+  uint32_t m;
+  asm("prmt.b32 %0, %1, %2, 0xBB99;" : "=r"(m) : "r"(act << (15 - J)), "r"(0u));
+  return ((raw << (15 - J)) & 0x80008000u) | (m & 0x3C003C00u);
 }
 
 // Writes 32 elements of a Z tile row in the canonical K-major layout from one
