@@ -25,6 +25,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -46,16 +47,16 @@ TRAFFIC = {
     # the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
     "soma_n2": {"bytes_per_launch": 64.062720e6 + 5.382400e6,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "3e7bcb1f936434e5"},
+                "source_hash": "91304d8250931a36"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
     "soma_n256": {"bytes_per_launch": 39.559168e6 + 2304,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                  "source_hash": "dcb065c9f93e4ce8"},
+                  "source_hash": "81adb1efd931ba90"},
     # profiles/body_tc_kernel_body_n256.md: one full-size launch (T=512)
     "body_n256": {"bytes_per_launch": 36.277248e6,
                   "files": ["body_tc.cu", "body_device.cuh", "tc_primitives.cuh",
                             "soma_device.cuh"],
-                  "source_hash": "16c79df5bb237a1f"},
+                  "source_hash": "0600bd36a9c58263"},
 }
 
 
@@ -269,12 +270,17 @@ def reference_arm(args):
 
 
 def source_hash(files):
-    """Hash of the sources a traffic figure was measured on."""
+    """Hash of the sources a traffic figure was measured on, comments and
+    blank lines left out (an edited comment does not change the kernel)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_37899_gb300", "csrc")
     for f in files:
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(csrc, f), encoding="utf-8") as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        code = "\n".join(line.rstrip() for line in text.splitlines() if line.strip())
+        h.update(code.encode())
     return h.hexdigest()[:16]
 
 

@@ -19,8 +19,8 @@
 //   MLP hidden operand -> MLP2 MMA (the hidden rows as the A operand,
 //   W_2 as B) -> residual;
 // then the final LN, the decode MMA (E, two 128-row tiles) and the NLL.
-// The CTA's NLL sums per sign go to the same partial-sum layout as the
-// CUDA-core sweep, reduced by body_reduce_kernel.
+// The CTA's NLL sums per sign go to partial[(pair, sign)][chunk], which
+// body_reduce_kernel (body.cu) turns into L+- and the coefficients.
 //
 // Precision.  With plain fp16 operands the losses were off by up to ~2e-4
 // nats/byte and the coefficients by ~1-2% on small batches: the rounding of
