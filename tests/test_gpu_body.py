@@ -69,6 +69,8 @@ def test_body_probe_bit_exact(oracle_mod, kind, D, seed, step, e, i, p0, count):
     (2, 4, 3, 20, 2),    # one chunk, ragged rows
     (1, 3, 19, 9, 2),    # two chunks, the second ragged
     (2, 2, 16, 6, 1),    # one full chunk, one block
+    (1, 1, 1, 1, 2),     # one sequence of one target, one probe
+    (1, 2, 17, 1, 1),    # a second chunk of one sequence, T = 1
 ])
 def test_body_estimate_matches_oracle(oracle_mod, kind, N, n, B, T, D):
     theta, head, bx = _inputs(N, B, T, D, seed=N * 10 + B)
