@@ -16,6 +16,7 @@ Independent references:
 - The probe law uses the independent Philox (tests/philox_ref.py): gains
   take the dense sign, every other coordinate the sparse probe.  The
   estimator's mean is q_j g_j with q = 1 on gains and 1/2 elsewhere (App. E).
+- The dense estimator's error obeys the variance law (P - 1) / n of Prop. 1.
 - Also checked: eps = 0, experts batched versus alone, and the update's
   closed forms.
 """
@@ -231,3 +232,20 @@ def test_update_closed_forms(oracle_mod):
         assert np.all(z[:, g0:] != 0)
         untouched = np.all(z == 0, axis=0)
         np.testing.assert_array_equal(to[e][untouched], th[e][untouched])
+
+
+def test_dense_estimator_variance_law(oracle_mod):
+    # Prop. 1 for the body: with dense probes, E|ghat - g|^2 / |g|^2 = (P - 1) / n
+    # (one probe: E[(g.z)^2 |z|^2] = P |g|^2, so E|X - g|^2 = (P - 1) |g|^2)
+    d, D = 4, 1
+    theta, head, bx = _setup(d, D, B=2, T=5, seed=19, wstd=0.6)
+    th = theta.astype(np.float64)
+    _, g = _torch_body_grad(th[0], d, D, head, bx[0])
+    P, n, reps = g.size, 64, 24
+    rel = []
+    for r in range(reps):
+        _, c = oracle_mod.body_spsa_losses(th, d, D, head, 1e-4, 31, r, bx, n_pert=n,
+                                           kind="dense", n_threads=1)
+        gh = th[0] - oracle_mod.body_spsa_update(th, d, D, 1.0, 31, r, c, kind="dense")[0]
+        rel.append(np.sum((gh - g) ** 2) / np.sum(g ** 2))
+    assert np.mean(rel) == pytest.approx((P - 1) / n, rel=0.2), (np.mean(rel), (P - 1) / n)
