@@ -115,16 +115,33 @@ DTYPE = "f16/f32"
 def gate_kernel_name(B, resident):
     if resident:
         return ("res_kernel (tcgen05, the whole recurrence of a probe pair resident in one CTA: "
-                "gate GEMM + cell + head + loss; its time includes the head)")
+                "gate GEMM + cell + head + loss)")
     if B <= 64:
-        return "tc_persistent_kernel<gate> (tcgen05 gate GEMM + fused cell)"
+        return ("tc_persistent_kernel (tcgen05; launch t = gate GEMM + fused cell of timestep t "
+                "and output head + softmax partials of t - 1)")
     return "gate_step_kernel (fp32 CUDA-core gate GEMM + cell)"
 
 
 def gate_flops_per_timestep(c):
-    # one launch = one timestep of every (expert, probe, sign) lane:
-    # [B, E+H] x [E+H, 4H] per lane, 2 flops per multiply-add
+    # one timestep of every (expert, probe, sign) lane: [B, E+H] x [E+H, 4H]
+    # per lane, 2 flops per multiply-add (the direct form's algorithmic count)
     return c["n_experts"] * c["n_pert"] * 2 * c["batch"] * 8 * c["H"] * (c["E"] + c["H"])
+
+
+def head_flops_per_timestep(c):
+    # the output head of one timestep of every lane: [B, H] x [H, 256]
+    return c["n_experts"] * c["n_pert"] * 2 * c["batch"] * 2 * 256 * c["H"]
+
+
+def applicable_peak(peaks, clocks):
+    """The burst bf16 peak applies when the sampled SM clock sat at its
+    maximum with no power cap (the burst figure was measured that way); the
+    sustained one otherwise (it was measured under the power cap)."""
+    sm, mx = clocks.get("sm_mhz"), clocks.get("sm_max_mhz")
+    at_max = sm is not None and mx is not None and sm >= 0.97 * mx
+    if at_max and "sw_power_cap" not in clocks.get("reasons", []):
+        return "burst", peaks["bf16_tflops"]
+    return "sustained", peaks["bf16_tflops_sustained"]
 
 
 def shard_seeds(rank):
@@ -353,8 +370,7 @@ def our_arm(args):
     for s in range(W):
         do_step(resident[s], s)
     barrier()
-    api.trace_enable(True)
-    api.trace_read(reset=True)
+    # the timed region: tracing off, so no event is recorded between launches
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         barrier()
@@ -364,10 +380,21 @@ def our_arm(args):
             do_step(resident[W + s], W + s)
         stop.record(stream)
         barrier()
-    api.trace_enable(False)
-    traced = api.trace_read(reset=True)
     ms = start.elapsed_time(stop)
     status = api.get_status()
+
+    # a second pass of the same K steps with the library's trace hooks on: the
+    # per-kernel device time (CUDA events on the launching stream around every
+    # launch) for kernel_ms and the roofline
+    api.trace_enable(True)
+    api.trace_read(reset=True)
+    barrier()
+    for s in range(K):
+        flush.fill_(s & 0xFF)
+        do_step(resident[W + s], W + s)
+    barrier()
+    api.trace_enable(False)
+    traced = api.trace_read(reset=True)
 
     # end to end through the public API: H2D of the step's bytes, the step,
     # D2H of its losses, every step
@@ -395,13 +422,15 @@ def our_arm(args):
     value = tok * K / (ms / 1e3)
     gate_ms, gate_n = traced["gate"]
     peaks, peak_src = measured_peaks()
-    peak = peaks["bf16_tflops_sustained"]
-    # all gate work of the timed region over the gate kernel's traced time:
-    # K steps x A estimates x T timesteps, whether a launch covers one
-    # timestep (persistent kernel) or all of them (resident kernel)
+    clocks = clk.summary()
+    peak_kind, peak = applicable_peak(peaks, clocks)
+    # all algorithmic gate and head work of the traced pass over the dominant
+    # kernel's traced time: K steps x A estimates x T timesteps, whether a
+    # launch covers one timestep (persistent kernel, the head of the previous
+    # timestep inside) or all of them (resident kernel)
     one_launch = traced["head"][1] == 0 and gate_n == K * A  # the resident kernel
-    gate_flops_total = gate_flops_per_timestep(c) * T * K * A
-    achieved = gate_flops_total / (gate_ms / 1e3) / 1e12 if gate_n else None
+    flops_total = (gate_flops_per_timestep(c) + head_flops_per_timestep(c)) * T * K * A
+    achieved = flops_total / (gate_ms / 1e3) / 1e12 if gate_n else None
     tr = TRAFFIC.get(args.config)
     traffic = (tr["bytes_per_launch"]
                if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
@@ -429,18 +458,26 @@ def our_arm(args):
             "bound": "tensor", "kernel": gate_kernel_name(B, one_launch),
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": (achieved / peak) if achieved else None, "traffic": traffic,
-            "peak_source": f"{peak_src} bf16 dense sustained (MEASURED_PEAKS.json)",
-            "flops_per_launch": gate_flops_total / gate_n if gate_n else None,
+            "peak_source": f"{peak_src} bf16 dense {peak_kind} (MEASURED_PEAKS.json): the "
+                           "burst figure when the sampled SM clock sat at its maximum with no "
+                           "power cap, the sustained one otherwise",
+            "frac_burst": (achieved / peaks["bf16_tflops"]) if achieved else None,
+            "frac_sustained": (achieved / peaks["bf16_tflops_sustained"]) if achieved else None,
+            "flops": "algorithmic gate + head flops of the direct form: "
+                     "8H(E+H) + 512H per perturbed token",
+            "flops_per_launch": flops_total / gate_n if gate_n else None,
             "launches": gate_n,
             "kernel_ms_per_launch": gate_ms / gate_n if gate_n else None,
             "share_of_step": gate_ms / ms if ms else None,
+            "step_frac_burst": (flops_total / K / (ms / 1e3) / 1e12 / peaks["bf16_tflops"])
+                               if ms else None,
         },
         "kernel_ms": {k: v[0] / K for k, v in traced.items()},
         "e2e": {"value": tok * K / (ms_e2e / 1e3), "unit": UNIT,
                 "h2d_bytes_per_step": int(sum(r.numel() for r in resident[0])),
                 "d2h_bytes_per_step": int(A * N * n * 2 * 4)},
         "gpu_launches": launches,
-        "clocks": clk.summary(),
+        "clocks": clocks,
         "status": api.STATUS_NAMES.get(status, status),
     }
     if not args.no_cpu_baseline and world == 1:
@@ -663,8 +700,7 @@ def body_arm(args):
     for s in range(W):
         do_step(resident[s], s)
     barrier()
-    api.trace_enable(True)
-    api.trace_read(reset=True)
+    # the timed region with tracing off; then a traced pass of the same steps
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         barrier()
@@ -674,10 +710,17 @@ def body_arm(args):
             do_step(resident[W + s], W + s)
         stop.record(stream)
         barrier()
-    api.trace_enable(False)
-    traced = api.trace_read(reset=True)
     ms = start.elapsed_time(stop)
     status = api.get_status()
+    api.trace_enable(True)
+    api.trace_read(reset=True)
+    barrier()
+    for s in range(K):
+        flush.fill_(s & 0xFF)
+        do_step(resident[W + s], W + s)
+    barrier()
+    api.trace_enable(False)
+    traced = api.trace_read(reset=True)
     losses_host = torch.empty(A, N, n, 2, dtype=torch.float32).pin_memory()
     dev_bytes = [torch.empty_like(r) for r in resident[0]]
     barrier()
@@ -702,7 +745,8 @@ def body_arm(args):
     flops = body_flops_per_token(c) * tokens_per_step(c) * A * K
     achieved = flops / (sweep_ms / 1e3) / 1e12 if sweep_n else None
     peaks, peak_src = measured_peaks()
-    tensor_peak = peaks["bf16_tflops_sustained"]
+    clocks = clk.summary()
+    peak_kind, tensor_peak = applicable_peak(peaks, clocks)
     tr = TRAFFIC.get(args.config)
     traffic = (tr["bytes_per_launch"]
                if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
@@ -729,7 +773,11 @@ def body_arm(args):
                                          "its time includes the decode and the loss)",
             "achieved": achieved, "peak": tensor_peak, "unit": "TFLOP/s",
             "frac": (achieved / tensor_peak) if achieved else None, "traffic": traffic,
-            "peak_source": f"{peak_src} bf16 dense sustained (MEASURED_PEAKS.json)",
+            "peak_source": f"{peak_src} bf16 dense {peak_kind} (MEASURED_PEAKS.json): the "
+                           "burst figure when the sampled SM clock sat at its maximum with no "
+                           "power cap, the sustained one otherwise",
+            "frac_burst": (achieved / peaks["bf16_tflops"]) if achieved else None,
+            "frac_sustained": (achieved / peaks["bf16_tflops_sustained"]) if achieved else None,
             "flops_per_token": body_flops_per_token(c),
             "launches": sweep_n,
             "kernel_ms_per_launch": sweep_ms / sweep_n if sweep_n else None,
@@ -740,7 +788,7 @@ def body_arm(args):
                 "h2d_bytes_per_step": int(sum(r.numel() for r in resident[0])),
                 "d2h_bytes_per_step": int(A * N * n * 2 * 4)},
         "gpu_launches": sum(v[1] for v in traced.values()),
-        "clocks": clk.summary(),
+        "clocks": clocks,
         "status": api.STATUS_NAMES.get(status, status),
     }
     if not args.no_cpu_baseline and world == 1:

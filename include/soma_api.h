@@ -272,6 +272,14 @@ int soma_debug_wait_timeout(uint32_t max_polls, void* stream);
 int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
                        void* stream);
 
+/* soma_debug_tc_gemm_ts: the same product with a staged in tensor memory
+ *   (lane = row, each 32-bit column one k pair) and read by tcgen05.mma from
+ *   there, the form in which the forward kernels feed their probe tiles Z
+ *   (the A operand of the Z products of Sec. 4, Eq. main-spsa, in the
+ *   mean/difference form).  Same arguments, limits and errors. */
+int soma_debug_tc_gemm_ts(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                          void* stream);
+
 /* SPSA step without a workspace argument, for callers that cannot allocate
  * device memory (a host runtime that only passes on buffers it was given, or
  * a loop that must not risk an allocation that blocks or fails).  The paper

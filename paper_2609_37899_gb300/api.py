@@ -94,6 +94,7 @@ def lib():
         _sig(L, "soma_debug_philox", i32, [u64, vp, vp, i32, vp])
         _sig(L, "soma_debug_rademacher", i32, [u64, u64, i32, i32, i64, i64, vp, vp])
         _sig(L, "soma_debug_tc_gemm", i32, [vp, vp, vp, i32, i32, vp])
+        _sig(L, "soma_debug_tc_gemm_ts", i32, [vp, vp, vp, i32, i32, vp])
         _sig(L, "soma_spsa_estimate", i32, [vp, i32, soma_dims, i32, i32, f32, u64, u64, vp, i32,
                                             i32, vp, vp, vp, sz, vp])
         _sig(L, "soma_adam_update", i32, [vp, vp, vp, i32, soma_dims, i32, i32, u64,
@@ -327,14 +328,16 @@ def debug_wait_timeout(max_polls: int, stream=None):
     _check(lib().soma_debug_wait_timeout(max_polls, _stream(stream)), "soma_debug_wait_timeout")
 
 
-def debug_tc_gemm(a: torch.Tensor, b: torch.Tensor, stream=None) -> torch.Tensor:
-    """a [128, K] fp16, b [N, K] fp16 (CUDA) -> a @ b.T [128, N] fp32 on the tensor cores."""
+def debug_tc_gemm(a: torch.Tensor, b: torch.Tensor, stream=None,
+                  a_in_tmem: bool = False) -> torch.Tensor:
+    """a [128, K] fp16, b [N, K] fp16 (CUDA) -> a @ b.T [128, N] fp32 on the tensor cores;
+    with a_in_tmem, a is staged in tensor memory (soma_debug_tc_gemm_ts)."""
     n, k = b.shape
     d = torch.empty(128, n, dtype=torch.float32, device=a.device)
-    _check(lib().soma_debug_tc_gemm(_dev(a, torch.float16, "a", 128 * k),
-                                    _dev(b, torch.float16, "b", n * k),
-                                    _dev(d, torch.float32, "d"), n, k, _stream(stream)),
-           "soma_debug_tc_gemm")
+    name = "soma_debug_tc_gemm_ts" if a_in_tmem else "soma_debug_tc_gemm"
+    _check(getattr(lib(), name)(_dev(a, torch.float16, "a", 128 * k),
+                                _dev(b, torch.float16, "b", n * k),
+                                _dev(d, torch.float32, "d"), n, k, _stream(stream)), name)
     return d
 
 

@@ -3,14 +3,18 @@
 // One CTA runs one (expert, probe) pair, both signs, over a chunk of up to 16
 // sequences for all T timesteps, in the mean/difference form of the LSTM
 // kernels applied to every linear layer.  With v+- = vbar +- dv (dv the half
-// difference) and the perturbed weights W +- eps Z:
-//   (W +- eps Z)(vbar +- dv) = C +- D,  C = W vbar + eps Z dv,  D = W dv + eps Z vbar,
-// so one MMA of W and one of Z against the operand rows [vbar | dv] give both
-// signs.  Everything between the linear layers (LayerNorm with perturbed
-// gains, the LSTM cell, GELU, the residual stream, the decode's log-sum-exp)
-// runs per sign in fp32 on the epilogue warps, which write the next operand
-// back as [vbar | dv] in fp16.  The tied head E is not perturbed: its logits
-// are E ybar +- E dy.
+// difference), its scaled form dhat = dv / eps, and the perturbed weights
+// W +- eps Z:
+//   (W +- eps Z)(vbar +- dv) = C +- eps D,  C = W vbar + eps^2 Z dhat,
+//   D = W dhat + Z vbar,
+// so one MMA of W and one of Z against the operand rows [vbar | dhat] give
+// both signs.  dhat is O(1), so its fp16 rounding stays relative (2^-11) at
+// any eps, where dv itself would fall into fp16's subnormal range.
+// Everything between the linear layers (LayerNorm with perturbed gains, the
+// LSTM cell, GELU, the residual stream, the decode's log-sum-exp) runs per
+// sign in fp32 on the epilogue warps (the residual stream as fp32 mean and
+// half difference), which write the next operand back as [vbar | dhat] in
+// fp16.  The tied head E is not perturbed: its logits are E ybar +- eps E dhat_y.
 //
 // Per timestep and block (17 warps: 16 epilogue warps, one MMA warp; one
 // barrier between phases):
@@ -27,7 +31,7 @@
 // W and vbar shifts the model both signs see, and the LayerNorms pass the
 // shift on.  So, except in the MLP's second layer:
 //  - every operand value is split, v = hi + lo (both fp16), as four row
-//    groups [vbar_hi | dv_hi | vbar_lo | dv_lo], so one W and one Z MMA
+//    groups [vbar_hi | dhat_hi | vbar_lo | dhat_lo], so one W and one Z MMA
 //    (N = 64) give both parts of both halves;
 //  - W = W_hi + W_lo: W_hi in shared memory, W_lo in tensor memory as the A
 //    operand of one more MMA (N = 32, the hi rows);
@@ -48,8 +52,8 @@ namespace {
 constexpr int kD = kBodyWidth;  // 32
 constexpr int kG = 4 * kD;      // 128
 constexpr int kBp = kBodyRows;  // sequences per CTA (16)
-constexpr int kN = 2 * kBp;     // operand rows [vbar | dv] (hi parts; MLP2 operand)
-constexpr int kNQ = 4 * kBp;    // operand rows [vbar_hi | dv_hi | vbar_lo | dv_lo]
+constexpr int kN = 2 * kBp;     // operand rows [vbar | dhat] (hi parts; MLP2 operand)
+constexpr int kNQ = 4 * kBp;    // operand rows [vbar_hi | dhat_hi | vbar_lo | dhat_lo]
 constexpr int kEpiWarps = 16;
 constexpr int kMmaWarp = kEpiWarps;
 constexpr int kThreads = (kEpiWarps + 1) * 32;
@@ -155,11 +159,12 @@ __device__ __forceinline__ uint32_t lo_pair(float w0, float w1) {
 }
 
 // out rows b + {0, 1, 2, 3} Bp of a K-major operand with K columns, features at
-// column offset k0: mean and half difference of the two signs' LN outputs.
-// Warp w runs sequence b = w (lane = feature).
+// column offset k0: mean and scaled half difference (times inv_eps = 1 / eps,
+// 0 when eps = 0) of the two signs' LN outputs.  Warp w runs sequence b = w
+// (lane = feature).
 __device__ __forceinline__ void ln_pair(const float* xbar, const float* dx, const float* gp,
                                         const float* gm, uint8_t* op, int K, int k0, int b,
-                                        int lane) {
+                                        int lane, float inv_eps) {
   const float xb = xbar[b * kD + lane], d = dx[b * kD + lane];
   const float xp = xb + d, xm = xb - d;
   const float mp = wsum(xp) * (1.f / kD), mm = wsum(xm) * (1.f / kD);
@@ -167,17 +172,19 @@ __device__ __forceinline__ void ln_pair(const float* xbar, const float* dx, cons
   const float vp = wsum(cp * cp) * (1.f / kD), vm = wsum(cm * cm) * (1.f / kD);
   const float up = cp * rsqrtf(vp + kLnEps) * gp[lane];
   const float um = cm * rsqrtf(vm + kLnEps) * gm[lane];
-  store_split(op, K, b, k0 + lane, 0.5f * (up + um), 0.5f * (up - um));
+  store_split(op, K, b, k0 + lane, 0.5f * (up + um), 0.5f * (up - um) * inv_eps);
 }
 
-// C and D of one layer for this thread's 16x128b view (TMEM lanes tq: rows
-// 0, 1 of the view; tq2: rows 2, 3; column = the thread's sequence):
-//   C = W (vbar_hi + vbar_lo) + eps Z (dv_hi + dv_lo),
-//   D = W (dv_hi + dv_lo) + eps Z (vbar_hi + vbar_lo),
+// C and the half difference D of one layer for this thread's 16x128b view
+// (TMEM lanes tq: rows 0, 1 of the view; tq2: rows 2, 3; column = the
+// thread's sequence):
+//   C = W (vbar_hi + vbar_lo) + eps^2 Z (dhat_hi + dhat_lo),
+//   D = eps [W (dhat_hi + dhat_lo) + Z (vbar_hi + vbar_lo)],
 // from the W accumulator (columns c + {0, 1, 2, 3} Bp; W_lo already added
 // to the hi columns) and the Z accumulator.
 __device__ __forceinline__ void layer_cd(uint32_t tq, uint32_t tq2, float eps, float (&C)[4],
                                          float (&D)[4]) {
+  const float eps2 = eps * eps;
   uint32_t w[4][4], z[4][4];  // [row group][row of the view]
 #pragma unroll
   for (int g = 0; g < 4; ++g) {
@@ -193,8 +200,8 @@ __device__ __forceinline__ void layer_cd(uint32_t tq, uint32_t tq2, float eps, f
     const float wd = __uint_as_float(w[1][k]) + __uint_as_float(w[3][k]);
     const float zv = __uint_as_float(z[0][k]) + __uint_as_float(z[2][k]);
     const float zd = __uint_as_float(z[1][k]) + __uint_as_float(z[3][k]);
-    C[k] = fmaf(eps, zd, wv);
-    D[k] = fmaf(eps, zv, wd);
+    C[k] = fmaf(eps2, zd, wv);
+    D[k] = eps * (wd + zv);
   }
 }
 
@@ -211,6 +218,8 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
   const int D = a.blocks;
   const float eps = a.eps;
   const bool do_z = eps != 0.f;
+  const float eps2 = eps * eps;
+  const float inv_eps = do_z ? 1.f / eps : 0.f;  // the operand's difference rows are dv / eps
   const float* th = a.params + (int64_t)e * a.P;
   const ProbeKey pk = make_probe_key(a.seed, a.step, (uint32_t)e, (uint32_t)i);
   uint64_t* mma_bar = reinterpret_cast<uint64_t*>(smem + kSmCtl);
@@ -392,7 +401,8 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
       uint8_t* o1 = smem + kSmO1 + b * (kNQ * 64 * 2);
       // ---- LN_a -> u part of the gate operand ------------------------------
       if (warp < kEpiWarps)
-        ln_pair(xbar, dx, gains + 2 * b * kD, gains + ng + 2 * b * kD, o1, 64, 0, warp, lane);
+        ln_pair(xbar, dx, gains + 2 * b * kD, gains + ng + 2 * b * kD, o1, 64, 0, warp, lane,
+                inv_eps);
       phase_barrier();
       if (warp == kMmaWarp) {
         if (lane == 0) {
@@ -403,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
             mma_f16_ss_lohi(tmem + kTW, lo(blk) + ko, hi64, ob + ko, hi64, idesc64, accf);
             mma_f16_ss_lohi(tmem + kTZ, lo(blk + kGateTile) + ko, hi64, ob + ko, hi64, idesc64,
                             accf);
-            // W_lo [vbar_hi | dv_hi], added to the hi columns
+            // W_lo [vbar_hi | dhat_hi], added to the hi columns
             mma_f16_ts_lohi(tmem + kTW, tmem + kTWloGate + 32 * b + 8 * k16, ob + ko, hi64,
                             idesc32, 1u);
           }
@@ -438,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
         const float hm = am[3] * fmaf(sigm_b(2.f * cm), 2.f, -1.f);
         const int U = 8 * q4 + u8;
         const float hb = 0.5f * (hp + hm), hd = 0.5f * (hp - hm);
-        store_split(o1, 64, bseq, kD + U, hb, hd);
+        store_split(o1, 64, bseq, kD + U, hb, hd * inv_eps);
         xbar[bseq * kD + U] += hb;
         dx[bseq * kD + U] += hd;
       }
@@ -446,7 +456,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
       // ---- LN_b -> MLP1 operand ---------------------------------------------
       if (warp < kEpiWarps)
         ln_pair(xbar, dx, gains + 2 * b * kD + kD, gains + ng + 2 * b * kD + kD,
-                smem + kSmO2, 32, 0, warp, lane);
+                smem + kSmO2, 32, 0, warp, lane, inv_eps);
       phase_barrier();
       if (warp == kMmaWarp) {
         if (lane == 0) {
@@ -481,11 +491,11 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
           *reinterpret_cast<__half*>(o3 + kmajor_offset(bseq, j, 128)) =
               __float2half_rn(0.5f * (mp + mm));
           *reinterpret_cast<__half*>(o3 + kmajor_offset(kBp + bseq, j, 128)) =
-              __float2half_rn(0.5f * (mp - mm));
+              __float2half_rn(0.5f * (mp - mm) * inv_eps);
         }
       }
       phase_barrier();
-      // ---- MLP2: [mbar | dm] (rows) x [W_2 ; Z_2]^T ------------------------
+      // ---- MLP2: [mbar | mhat] (rows) x [W_2 ; Z_2]^T ----------------------
       // W_2 and Z_2 are adjacent 32-row B tiles, i.e. one 64-row B operand:
       // one MMA of N = 64 gives W_2 m (columns 0-31) and Z_2 m (32-63)
       if (warp == kMmaWarp) {
@@ -504,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
       } else {
         mma_wait();
         if (q4 == 0) {
-          // lanes 0-15: rows mbar of sequences, 16-31: dm; columns: features.
+          // lanes 0-15: rows mbar of sequences, 16-31: mhat; columns: features.
           // Warp 4 sg takes features 8 sg .. 8 sg + 7.
 #pragma unroll
           for (int cg = 0; cg < 2; ++cg) {
@@ -520,8 +530,8 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
               const int s = u8 + 8 * h;  // sequence
-              const float C = fmaf(eps, __uint_as_float(zdd[h]), __uint_as_float(wm[h]));
-              const float Dd = fmaf(eps, __uint_as_float(zm[h]), __uint_as_float(wdd[h]));
+              const float C = fmaf(eps2, __uint_as_float(zdd[h]), __uint_as_float(wm[h]));
+              const float Dd = eps * (__uint_as_float(wdd[h]) + __uint_as_float(zm[h]));
               xbar[s * kD + j] += C;
               dx[s * kD + j] += Dd;
             }
@@ -534,7 +544,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
     // ---- y = LN(x) gf -> decode operand; logits = E y ---------------------
     if (warp < kEpiWarps)
       ln_pair(xbar, dx, gains + 2 * D * kD, gains + ng + 2 * D * kD, smem + kSmO4, 32, 0, warp,
-              lane);
+              lane, inv_eps);
     phase_barrier();
     if (warp == kMmaWarp) {
       if (lane == 0) {
@@ -581,7 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
         for (int k = 0; k < 4; ++k) {
           const float C = __uint_as_float(yq[0][k]) +
                           (__uint_as_float(yq[2][k]) + __uint_as_float(ye[k]));
-          const float Dh = __uint_as_float(yq[1][k]) + __uint_as_float(yq[3][k]);
+          const float Dh = eps * (__uint_as_float(yq[1][k]) + __uint_as_float(yq[3][k]));
           lp[k] = C + Dh;
           lm[k] = C - Dh;
         }

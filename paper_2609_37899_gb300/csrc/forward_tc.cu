@@ -2,34 +2,46 @@
 // perturbed LSTM experts in the mean/difference form.
 //
 // For one expert e and probe i, the two antithetic copies of the LSTM take
-// inputs v+- = [x+-; h+-_{t-1}].  Write vbar = (v+ + v-)/2 and dv = (v+ - v-)/2.
-// With the perturbed weights W +- eps Z (Z = z_{e,i} reshaped, entries +-1),
-//   (W +- eps Z)(vbar +- dv) = [W vbar + eps Z dv] +- [W dv + eps Z vbar]
-// exactly, so the gate pre-activations are a+- = C +- D with
-//   C = W vbar + eps (Z dv) + b,       D = W dv + eps (Z vbar) + eps z_b.
-// The four products W vbar, W dv, Z vbar, Z dv are fp16 x fp16 -> fp32
-// tensor-core GEMMs; eps multiplies only in fp32 (epilogue), so no operand
-// ever holds a rounded w +- eps z.  dv is an explicit operand, so the
-// rounding of the operands perturbs the difference of the two copies only
-// relatively (fp16: 2^-11), never by cancellation.  The cell state c+- and
-// the activations are fp32 per sign.  The output head uses the same split:
-// logits+- = [W_out hbar + eps Z_out dh + b_out] +- [W_out dh + eps Z_out hbar
-// + eps z_bo].
+// inputs v+- = [x+-; h+-_{t-1}].  Write vbar = (v+ + v-)/2 and the scaled half
+// difference dhat = (v+ - v-)/(2 eps), an O(1) quantity.  With the perturbed
+// weights W +- eps Z (Z = z_{e,i} reshaped, entries +-1, or 0 for inactive
+// sparse coordinates),
+//   (W +- eps Z)(vbar +- eps dhat) = [W vbar + eps^2 Z dhat] +- eps [W dhat + Z vbar]
+// exactly, so the gate pre-activations are a+- = C +- eps D with
+//   C = W vbar + eps^2 (Z dhat) + b,       D = W dhat + Z vbar + z_b.
+// The products are fp16 x fp16 -> fp32 tensor-core GEMMs and eps multiplies
+// only in fp32 (epilogue), so no operand ever holds a rounded w +- eps z, and
+// the rounding of dhat is relative (2^-11) at any eps: the difference of the
+// two copies is never formed by cancelling two rounded numbers, and never
+// falls into fp16's subnormal range.  The cell state c+- and the
+// activations are fp32 per sign.  The output head uses the same split.
 //
-// Per timestep t, two launches of one persistent kernel:
-//   gate tasks  (expert, 32-unit row tile, group of P probes):
-//               D_W[128 x 2BpP] = W_tile x [vbar|dv]^T (shared by the P
-//               probes) and D_Z,p[128 x 2Bp] = Z_p x [vbar_p|dv_p]^T, Z_p
-//               generated from Philox into shared memory stage by stage;
-//               epilogue: gates, cell update, next timestep's operand
-//               [hbar|dh] (fp16).
-//   head tasks  (expert, 128-row vocabulary half, probe group): the same
-//               MMAs over the h part of the operand, then per (sequence,
-//               sign) max and sum-exp partials of the half and the target
-//               logit; extra blocks of the same launch write the embedding
-//               part of the next operand.
-// A final reduction merges the two halves into per-target NLL and the
-// per-(expert, probe) losses and coefficients.
+// Operand tiles.  P <= 2 probes share one operand group tile; its rows are,
+// in blocks of Bp sequences,
+//   P = 2:  [eps^2 dhat_0 | vbar_0 | dhat_0 | dhat_1 | vbar_1 | eps^2 dhat_1]
+//   P = 1:  [eps^2 dhat_0 | vbar_0 | dhat_0]
+// so that every product lands in one accumulator per probe, [C_p | D_p]:
+//   W x rows Bp .. (1 + 2P) Bp  -> columns [C_0 | D_0 | D_1 | C_1] (one MMA),
+//   Z_0 x rows 0 .. 2 Bp        -> [C_0 | D_0]    (eps^2 dhat_0 -> C, vbar_0 -> D),
+//   Z_1 x rows 4 Bp .. 6 Bp     -> [D_1 | C_1]    (vbar_1 -> D, eps^2 dhat_1 -> C).
+// The eps^2 dhat rows carry a term of order eps^2 |Z dhat|; their fp16
+// rounding (subnormal below |eps^2 dhat| = 6e-5) costs at most 3e-8 per
+// element, below the rounding of W vbar that C already carries.
+//
+// Per timestep t, one launch of one persistent kernel with two kinds of task:
+//   gate tasks  (expert, 32-unit row tile, group of P probes), t < T: the
+//               W tile (shared memory) and the P probe tiles Z_p (generated
+//               from Philox straight into tensor memory, the A operand of a
+//               tcgen05.mma with A in TMEM) against the operand tiles of
+//               timestep t; epilogue: gates, cell update, the h part of the
+//               operand of t + 1;
+//   head tasks  (expert, 128-row vocabulary half, probe group) of timestep
+//               t - 1, t >= 1: the same MMAs over the h part of the same
+//               operand (h_{t-1}), then per (sequence, sign) max and sum-exp
+//               partials of the half and the target logit.
+// Extra blocks of the launch write the embedding part of the operand of
+// t + 1.  A final reduction merges the two halves into per-target NLL and
+// the per-(expert, probe) losses and coefficients.
 #include <cuda_fp16.h>
 
 #include "soma_api.h"
@@ -43,21 +55,29 @@ using namespace tc;
 
 namespace {
 
-constexpr int kZWarps = 8;
-constexpr int kStages = 3;
-constexpr int kLoaders = kStages;  // one issuing thread per ring slot (the copies of
-                                   // one thread complete one after another)
-constexpr int kEpiWarps = 8;
-constexpr int kEpiProbeStep = kEpiWarps / 4;  // warp ew runs probes ew / 4, + kEpiProbeStep, ...
-static_assert(kZWarps * 32 == 256, "one Z generator thread per (probe, row): 2 x 128");
-static_assert(kEpiWarps == 4 || kEpiWarps == 8, "epilogue warps: 4 lane quarters x 1 or 2 probes");
-constexpr int kThreads = (kLoaders + 1 + kZWarps + kEpiWarps) * 32;  // loaders, MMA, Z, epilogue
-constexpr int kKt = 64;                 // K per stage (fp16 elements)
+constexpr int kStages = 4;       // ring slots: shared-memory operands and TMEM probe tiles
+// The bulk-copy instructions of one warp complete one after another (~750
+// cycles each, whatever the size up to 48 KB), while the lanes of one
+// instruction and different warps copy in parallel.  So each stage's two
+// copies are one instruction of two lanes, and the stages rotate over three
+// loader warps.
+constexpr int kLoaders = 1;
+constexpr int kMmaWarp = 1;
+constexpr int kZWarp0 = 4;       // Z generators: a multiple of 4 (TMEM lane quarters)
+constexpr int kZWarps = 8;       // (probe, lane quarter)
+constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
+constexpr int kEpiWarps = 8;     // (probe, lane quarter)
+constexpr int kEpiProbeStep = kEpiWarps / 4;  // head: warp group eg runs probes eg, eg + 2, ...
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
+static_assert(kZWarp0 % 4 == 0 && kEpiWarp0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
+constexpr int kKt = 64;                     // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
-constexpr uint32_t kSbo = kKt * 16;     // bytes between 8-row groups
-constexpr uint32_t kLbo = 128;          // bytes between core matrices along K
-constexpr uint32_t kZCols = 128;        // Z products start 128 columns into a buffer
-constexpr uint32_t kTmemCols = 512;     // two accumulator buffers of 256 columns
+constexpr uint32_t kSbo = kKt * 16;         // bytes between 8-row groups
+constexpr uint32_t kLbo = 128;              // bytes between core matrices along K
+constexpr uint32_t kAccCols = 128;          // one accumulator buffer: 2 Bp P <= 128 columns
+constexpr uint32_t kZCol0 = 2 * kAccCols;   // probe tiles: slot q at kZCol0 + 64 q (+ 32 p)
+constexpr uint32_t kTmemCols = 512;
+static_assert(kZCol0 + kStages * 64 <= kTmemCols, "probe tiles fit tensor memory");
 
 __device__ __forceinline__ uint32_t compact16(uint32_t x) {
   x &= 0x55555555u;
@@ -76,17 +96,24 @@ __device__ __forceinline__ uint32_t natural_to_raw(uint32_t n) {
 
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
 
-// Shared-memory carve-up of one stage.
+// Row blocks (units of Bp) of probe p inside an operand group tile and the
+// accumulator columns (units of Bp) of its C and D parts; see the header.
+__host__ __device__ __forceinline__ int row_mean(int p) { return p == 0 ? 1 : 4; }
+__host__ __device__ __forceinline__ int row_dhat(int p) { return p == 0 ? 2 : 3; }
+__host__ __device__ __forceinline__ int row_e2(int p) { return p == 0 ? 0 : 5; }
+__host__ __device__ __forceinline__ int col_c(int p) { return row_mean(p) - 1; }
+__host__ __device__ __forceinline__ int col_d(int p) { return row_dhat(p) - 1; }
+
+// Shared-memory carve-up of one ring slot.
 struct StageLayout {
-  uint32_t a_off, b_off, z_off, bytes;
+  uint32_t a_off, b_off, bytes;
 };
 
 __host__ __device__ inline StageLayout stage_layout(const TcGeom& g) {
   StageLayout L;
   L.a_off = 0;
   L.b_off = kTileA;
-  L.z_off = L.b_off + g.tileB;
-  L.bytes = L.z_off + (uint32_t)g.P * kTileA;
+  L.bytes = (L.b_off + g.tileB + 1023u) & ~1023u;
   return L;
 }
 
@@ -124,74 +151,80 @@ __device__ __forceinline__ uint32_t z_pair(uint32_t raw, uint32_t act) {
   return ((raw << (15 - J)) & 0x80008000u) | (m & 0x3C003C00u);
 }
 
-// Writes 32 elements of a Z tile row in the canonical K-major layout from one
-// raw sign word (and, for sparse probes, its activity word); `row` points at
-// the first element, consecutive 8-element chunks are 128 bytes apart.
+// The 16 fp16 pair words of one 32-parameter run: word J holds elements 2J
+// (low half) and 2J + 1 (high half), i.e. one TMEM column of an A operand.
 template <bool SPARSE>
-__device__ __forceinline__ void store_z_row_at(uint8_t* row, uint32_t raw, uint32_t act) {
-  uint4 c0, c1, c2, c3;
-  c0.x = z_pair<SPARSE, 0>(raw, act);   c0.y = z_pair<SPARSE, 1>(raw, act);
-  c0.z = z_pair<SPARSE, 2>(raw, act);   c0.w = z_pair<SPARSE, 3>(raw, act);
-  c1.x = z_pair<SPARSE, 4>(raw, act);   c1.y = z_pair<SPARSE, 5>(raw, act);
-  c1.z = z_pair<SPARSE, 6>(raw, act);   c1.w = z_pair<SPARSE, 7>(raw, act);
-  c2.x = z_pair<SPARSE, 8>(raw, act);   c2.y = z_pair<SPARSE, 9>(raw, act);
-  c2.z = z_pair<SPARSE, 10>(raw, act);  c2.w = z_pair<SPARSE, 11>(raw, act);
-  c3.x = z_pair<SPARSE, 12>(raw, act);  c3.y = z_pair<SPARSE, 13>(raw, act);
-  c3.z = z_pair<SPARSE, 14>(raw, act);  c3.w = z_pair<SPARSE, 15>(raw, act);
-  *reinterpret_cast<uint4*>(row) = c0;
-  *reinterpret_cast<uint4*>(row + 128) = c1;
-  *reinterpret_cast<uint4*>(row + 256) = c2;
-  *reinterpret_cast<uint4*>(row + 384) = c3;
+__device__ __forceinline__ void z_run_pairs(uint32_t raw, uint32_t act, uint32_t* o) {
+  o[0] = z_pair<SPARSE, 0>(raw, act);    o[1] = z_pair<SPARSE, 1>(raw, act);
+  o[2] = z_pair<SPARSE, 2>(raw, act);    o[3] = z_pair<SPARSE, 3>(raw, act);
+  o[4] = z_pair<SPARSE, 4>(raw, act);    o[5] = z_pair<SPARSE, 5>(raw, act);
+  o[6] = z_pair<SPARSE, 6>(raw, act);    o[7] = z_pair<SPARSE, 7>(raw, act);
+  o[8] = z_pair<SPARSE, 8>(raw, act);    o[9] = z_pair<SPARSE, 9>(raw, act);
+  o[10] = z_pair<SPARSE, 10>(raw, act);  o[11] = z_pair<SPARSE, 11>(raw, act);
+  o[12] = z_pair<SPARSE, 12>(raw, act);  o[13] = z_pair<SPARSE, 13>(raw, act);
+  o[14] = z_pair<SPARSE, 14>(raw, act);  o[15] = z_pair<SPARSE, 15>(raw, act);
+}
+
+// 32 consecutive 32-bit columns of this thread's TMEM lane <- r[0..31].
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]),
+      "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]),
+      "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]),
+      "r"(r[30]), "r"(r[31])
+      : "memory");
 }
 
 // The MMAs of one stage, fully unrolled over K (NP = probes with a Z tile):
-// W x operand into [0, rowsB) and Z_p x operand_p into kZCols + 2 Bp p.  The
-// descriptors arrive as their low words (start address of the stage's tiles;
-// a step along K or to the next probe is an addition), so the issuing thread
-// spends a few instructions per MMA and keeps the tensor pipe fed.
+//   W (shared memory) x operand rows from w_row   -> d, N = 2 Bp P;
+//   Z_0 (TMEM, zt)    x operand rows from 0       -> d, N = 2 Bp;
+//   Z_1 (TMEM, zt+32) x operand rows from z1_row  -> d + dz1, N = 2 Bp.
+// Descriptors arrive as their low words (start address in 16-byte units; a
+// step along K is an addition), so the issuing thread spends a few
+// instructions per MMA and keeps the tensor pipe fed.
 template <int NP>
-__device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo, uint32_t z_lo,
-                                            uint32_t hi, uint32_t zp_step, uint32_t bp_step,
-                                            uint32_t idesc_w, uint32_t idesc_z, uint32_t dz_step,
+__device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo, uint32_t hi,
+                                            uint32_t w_row, uint32_t z1_row, uint32_t zt,
+                                            uint32_t idesc_w, uint32_t idesc_z, uint32_t dz1,
                                             uint32_t acc0) {
 #pragma unroll
   for (int k16 = 0; k16 < kKt / 16; ++k16) {
-    const uint32_t ko = (uint32_t)k16 * 16;
+    const uint32_t ko = (uint32_t)k16 * 16;  // 256 bytes: two core matrices along K
     const uint32_t acc = k16 > 0 ? 1u : acc0;
-    mma_f16_ss_lohi(d, a_lo + ko, hi, b_lo + ko, hi, idesc_w, acc);
-    if (NP >= 1) mma_f16_ss_lohi(d + kZCols, z_lo + ko, hi, b_lo + ko, hi, idesc_z, acc);
+    mma_f16_ss_lohi(d, a_lo + ko, hi, b_lo + w_row + ko, hi, idesc_w, acc);
+    if (NP >= 1) mma_f16_ts_lohi(d, zt + 8u * k16, b_lo + ko, hi, idesc_z, 1u);
     if (NP >= 2)
-      mma_f16_ss_lohi(d + kZCols + dz_step, z_lo + ko + zp_step, hi, b_lo + ko + bp_step, hi,
-                      idesc_z, acc);
+      mma_f16_ts_lohi(d + dz1, zt + 32u + 8u * k16, b_lo + z1_row + ko, hi, idesc_z, 1u);
   }
 }
 
 // ---------------------------------------------------------------------------
 // Persistent warp-specialised kernel.  One CTA per SM walks a static list of
-// tasks (blockIdx.x, blockIdx.x + n_ctas, ...; the head launch appends
-// n_ctas-independent blocks for the embedding operand, so the stride is
-// n_ctas, not the grid size).  Roles:
-//   warps 0..2    loaders: warp j bulk-copies the A tile and the operand
-//                 group tile of every stage that uses ring slot j (16 KB
-//                 copies; the copies of one issuing thread complete one
-//                 after another, so each slot has its own issuer);
-//   warp 3        MMA issuer: W x operand and Z_p x operand_p per stage into
-//                 one of two TMEM accumulator buffers (256 columns each);
-//   warps 4..11   Z generators: the +-1 tiles of the stage, from Philox
-//                 (one (probe, row) pair per thread);
+// tasks (blockIdx.x, blockIdx.x + n_ctas, ...): the gate tasks of timestep
+// t, then the head tasks of t - 1.  Extra blocks (blockIdx.x >= n_ctas)
+// write the embedding part of the next operand.  Roles:
+//   warps 0, 2, 3 loaders: stage gs belongs to loader gs % 3, whose lanes 0
+//                 and 1 bulk-copy its A tile and its operand group tile in
+//                 one instruction;
+//   warp 1        MMA issuer (lane 0 alone, so no warp-wide step sits
+//                 between consecutive stages): W x operand (shared memory)
+//                 and Z_p x operand (Z_p in tensor memory) per stage into one
+//                 of two TMEM accumulator buffers;
+//   warps 4..11   Z generators: thread (probe, row) expands Philox words into
+//                 the fp16 +-1 row of its probe tile and stores it into the
+//                 slot's TMEM columns (lane = row);
 //   warps 12..19  epilogue: reads a finished accumulator buffer while the
 //                 MMAs of the next task fill the other one; warp w reads the
-//                 TMEM lanes of quarter w % 4 for probe (w - 12) / 4.
-// Barriers: full (the slot's copies landed and its Z tiles are written),
-// slot_free (the slot's MMAs are done), acc_full (a buffer's task is
+//                 TMEM lanes of quarter w % 4 for probe group (w - 12) / 4.
+// Barriers: full (the slot's copies landed and its Z tiles are stored: the
+// loader's arrival with the copies' bytes and one arrival per Z warp, so the
+// issuer waits once per stage), slot_free (the slot's MMAs are done), acc_full (a buffer's task is
 // accumulated), acc_empty (its epilogue has read it), mma_done (all MMAs of
 // the CTA completed).  Every wait is bounded (wait_or_abort, mbar_wait).
 // ---------------------------------------------------------------------------
-constexpr int kMmaWarp = kLoaders;
-constexpr int kZWarp0 = kMmaWarp + 1;
-constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
-constexpr int kAccCols = 256;
-
 struct Ctl {
   uint64_t full[kStages];
   uint64_t slot_free[kStages];
@@ -206,8 +239,7 @@ struct Ctl {
 // the CTA's abort flag; a wait that is still pending sees the flag within 64
 // polls and returns false, so the CTA winds down without issuing further
 // copies or MMAs.  A phase that is already complete costs one poll and no
-// read of the flag (the flag shares the shared-memory pipe with the
-// epilogue's shuffles, and every handoff of the main loop passes here).
+// read of the flag.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               int* status) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -220,15 +252,51 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
+// Ring position of the next stage: slot q and the parity of its phase.
+struct RingPos {
+  uint32_t q, ph;
+  __device__ __forceinline__ void next() {
+    if (++q == kStages) {
+      q = 0;
+      ph ^= 1u;
+    }
+  }
+};
+
+// The MMAs of one task, issued by one thread: per stage, wait for the
+// copies and the probe tiles (one barrier), issue, and release the slot
+// with a commit.
+// The probe count NP is fixed per task, so the loop carries no dispatch.
+template <int NP>
+__device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
+                                         RingPos& rp, int nst, uint32_t d, uint32_t tmem,
+                                         uint32_t a_lo0, uint32_t b_lo0, uint32_t slot_step,
+                                         uint32_t hi, uint32_t w_row, uint32_t z1_row,
+                                         uint32_t idesc_w, uint32_t idesc_z, uint32_t dz1,
+                                         volatile int* abort, int* status) {
+  for (int st = 0; st < nst; ++st) {
+    if (!wait_or_abort(&full[rp.q], rp.ph, abort, status)) return false;
+    tc_fence_after();
+    const uint32_t so = rp.q * slot_step;
+    issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.q,
+                    idesc_w, idesc_z, dz1, st > 0 ? 1u : 0u);
+    mma_commit(&slot_free[rp.q]);
+    rp.next();
+  }
+  return true;
+}
+
 struct TcArgs {
   Sweep sw;
   TcGeom g;
-  int t;
+  int t_gate;            // timestep of the gate tasks, -1: none
+  int t_head;            // timestep of the head tasks, -1: none
+  int n_gate, n_head;    // task counts
   const uint8_t* w16;    // [N][MT][S] A tiles
   const uint8_t* wo16;   // [N][2][Sh] A tiles
-  const uint8_t* op_in;  // [N][S][G] operand group tiles of this timestep
-  uint8_t* op_out;       // next timestep's operand
-  float* cst;            // [N*n*2][Hp][Bp] cell state
+  const uint8_t* op_in;  // [N][S][G] operand group tiles: [x_t | h_{t-1}]
+  uint8_t* op_out;       // operand of t + 1
+  float* cst;            // [N*n][Hp][Bp] cell state (float2: sign +, -)
   float* pm;             // [N*n*2][B][T][2] head max partials
   float* ps;             // sum-exp partials
   float* ply;            // [N*n*2][B][T] target logits
@@ -239,24 +307,28 @@ struct TcArgs {
 // 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
 // half.
 struct Task {
-  int e, m, grp, p_valid;
+  bool head;
+  int e, m, grp, p_valid, nst;
   const uint8_t* a;  // A tile of stage 0
   const uint8_t* b;  // operand group tile of stage 0
 };
 
-template <bool HEAD>
 __device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
   const TcGeom& g = a.g;
   Task T;
-  T.grp = task % g.G;
-  const int rows = HEAD ? 2 : g.MT;
-  T.m = (task / g.G) % rows;
-  T.e = task / (g.G * rows);
+  T.head = task >= a.n_gate;
+  const int j = T.head ? task - a.n_gate : task;
+  T.grp = j % g.G;
+  const int rows = T.head ? 2 : g.MT;
+  T.m = (j / g.G) % rows;
+  T.e = j / (g.G * rows);
   T.p_valid = min(g.P, a.sw.n_pert - T.grp * g.P);
-  if (HEAD) {
+  if (T.head) {
+    T.nst = g.Sh;
     T.a = a.wo16 + (((size_t)T.e * 2 + T.m) * g.Sh) * kTileA;
     T.b = a.op_in + (((size_t)T.e * g.S + g.Sx) * g.G + T.grp) * g.tileB;
   } else {
+    T.nst = g.S;
     T.a = a.w16 + (((size_t)T.e * g.MT + T.m) * g.S) * kTileA;
     T.b = a.op_in + (((size_t)T.e * g.S) * g.G + T.grp) * g.tileB;
   }
@@ -264,30 +336,51 @@ __device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
 }
 
 // Flat parameter index of element (row r, k = 0) of the stage-st Z run.
-template <bool HEAD>
 __device__ __forceinline__ int64_t z_param(const TcArgs& a, const Task& T, int r, int st) {
   const Layout& L = a.sw.lay;
-  if (HEAD) return L.w_out + (int64_t)(128 * T.m + r) * a.g.H + (int64_t)kKt * st;
+  if (T.head) return L.w_out + (int64_t)(128 * T.m + r) * a.g.H + (int64_t)kKt * st;
   const int64_t R = (int64_t)tile_gate(r) * a.g.H + 32 * T.m + tile_unit(r);  // W row of tile row r
   return st < a.g.Sx ? L.w_ih + R * a.g.E + (int64_t)kKt * st
                      : L.w_hh + R * a.g.H + (int64_t)kKt * (st - a.g.Sx);
 }
 
-// Gate epilogue of one task for one warp: probe p, TMEM lane quarter q4
-// (units 8 q4 .. 8 q4 + 7 of the tile).  Thread l runs the cells of unit
-// l / 4 for sequences b0 + l % 4 and b0 + 4 + l % 4 of every 8-sequence
-// chunk, both signs, in fp32: 16x128b loads give it all four gates of its
-// unit (gate-major rows), so no data moves between threads.  Cell state
-// layout: [e, i][Hp][Bp][sign].
-__device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, const ProbeKey& pk,
-                              int q4, int p) {
+// Gate epilogue of one task for one warp of TMEM lane quarter q4 (units
+// 8 q4 .. 8 q4 + 7 of the tile).  With P = 2 the warps of group eg = 0, 1 run
+// probe eg; with P = 1 both groups run probe 0 and split its 8-sequence
+// chunks.  Thread l runs the cells of unit l / 4 for sequences b0 + l % 4 and
+// b0 + 4 + l % 4 of each of its chunks, both signs, in fp32: 16x128b loads
+// give it all four gates of its unit (gate-major rows), so no data moves
+// between threads.  It writes the three operand rows of its (unit,
+// sequence) for timestep t + 1: vbar, dhat and eps^2 dhat.  Cell state
+// layout: [e, i][Hp][Bp] float2 (+, -).
+//
+// gate_prepare runs before the accumulator is ready: it loads the bias, its
+// probe signs and the previous cell states, so that their latency overlaps
+// the task's MMAs.
+constexpr int kEpiMaxChunks = 4;  // Bp <= 32 with P = 2; Bp <= 64 split over two groups with P = 1
+
+struct GatePre {
+  float bias[4], dbias[4];
+  float2 cprev[kEpiMaxChunks][2];
+  int p, c0, cstep;
+  bool on;
+};
+
+__device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int q4, int eg,
+                                             GatePre& G) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
   const int lane = threadIdx.x & 31;
   const int H = g.H;
+  G.p = g.P == 2 ? eg : 0;
+  G.c0 = g.P == 2 ? 0 : eg;
+  G.cstep = g.P == 2 ? 1 : 2;
+  G.on = G.p < T.p_valid;
+  if (!G.on) return;
+  const int i = T.grp * g.P + G.p;
+  const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)i);
   const float eps = s.eps;
-  const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
   // bias and its probe sign for the row in this lane's TMEM lane, handed to
   // the threads that run that row's unit
@@ -297,19 +390,45 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
     if (Ur < H) {
       const int64_t pb = L.b + (int64_t)tile_gate(32 * q4 + lane) * H + Ur;
       bias_r = th[pb];
-      if (do_z) {
+      if (eps != 0.f) {
         const ProbeBits zb = probe_bits(pk, pb, s.sparse);
         dbias_r = eps_z(zb.neg & 1u, zb.act & 1u, eps);
       }
     }
   }
   const int u8 = lane >> 2, bq = lane & 3;
-  float bias[4], dbias[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    bias[k] = __shfl_sync(0xffffffffu, bias_r, 8 * k + u8);
-    dbias[k] = __shfl_sync(0xffffffffu, dbias_r, 8 * k + u8);
+    G.bias[k] = __shfl_sync(0xffffffffu, bias_r, 8 * k + u8);
+    G.dbias[k] = __shfl_sync(0xffffffffu, dbias_r, 8 * k + u8);
   }
+  const int U = 32 * T.m + 8 * q4 + u8;
+  const float2* cell = reinterpret_cast<const float2*>(a.cst) +
+                       (((int64_t)T.e * s.n_pert + i) * g.Hp + U) * (int64_t)g.Bp;
+  const bool load = U < H && a.t_gate > 0;
+#pragma unroll
+  for (int j = 0; j < kEpiMaxChunks; ++j) {
+    const int b0 = 8 * (G.c0 + j * G.cstep);
+    G.cprev[j][0] = G.cprev[j][1] = make_float2(0.f, 0.f);
+    if (load && b0 < g.Bp) {
+      G.cprev[j][0] = cell[b0 + bq];
+      G.cprev[j][1] = cell[b0 + 4 + bq];
+    }
+  }
+}
+
+__device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q4,
+                            const GatePre& G) {
+  if (!G.on) return;
+  const TcGeom& g = a.g;
+  const Sweep& s = a.sw;
+  const int lane = threadIdx.x & 31;
+  const int H = g.H;
+  const float eps = s.eps;
+  const float half_inv_eps = eps != 0.f ? 0.5f / eps : 0.f;
+  const float half_eps = 0.5f * eps;
+  const int p = G.p;
+  const int u8 = lane >> 2, bq = lane & 3;
   const int U = 32 * T.m + 8 * q4 + u8;
   const bool unit_ok = U < H;
   // a stage of the next operand holds kKt / 32 of the 32-unit row tiles
@@ -321,27 +440,21 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
                  (((int64_t)T.e * s.n_pert + i) * g.Hp + U) * (int64_t)g.Bp;
   const uint32_t tq = tacc + ((uint32_t)(32 * q4) << 16);  // gates 0, 1
   const uint32_t tq2 = tq + (16u << 16);                    // gates 2, 3
-  for (int b0 = 0; b0 < g.Bp; b0 += 8) {
-    float2 cprev[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-    if (unit_ok && a.t > 0) {
-      cprev[0] = cell[b0 + bq];
-      cprev[1] = cell[b0 + 4 + bq];
-    }
-    // [seq half][gate]: W vbar, W dv, Z vbar, Z dv
-    uint32_t wv[2][4], wd[2][4], zv[2][4], zd[2][4];
+  const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
+  const int rM = row_mean(p) * g.Bp, rD = row_dhat(p) * g.Bp, rE = row_e2(p) * g.Bp;
+#pragma unroll
+  for (int j = 0; j < kEpiMaxChunks; ++j) {
+    const int b0 = 8 * (G.c0 + j * G.cstep);
+    if (b0 >= g.Bp) break;
+    // [seq half][gate]: C (W vbar + eps^2 Z dhat) and D (W dhat + Z vbar)
+    uint32_t vc[2][4], vd[2][4];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0 + 4 * h);
-      tmem_ld_16x128b(tq + cw, wv[h][0], wv[h][1]);
-      tmem_ld_16x128b(tq2 + cw, wv[h][2], wv[h][3]);
-      tmem_ld_16x128b(tq + cw + g.Bp, wd[h][0], wd[h][1]);
-      tmem_ld_16x128b(tq2 + cw + g.Bp, wd[h][2], wd[h][3]);
-      if (do_z) {
-        tmem_ld_16x128b(tq + kZCols + cw, zv[h][0], zv[h][1]);
-        tmem_ld_16x128b(tq2 + kZCols + cw, zv[h][2], zv[h][3]);
-        tmem_ld_16x128b(tq + kZCols + cw + g.Bp, zd[h][0], zd[h][1]);
-        tmem_ld_16x128b(tq2 + kZCols + cw + g.Bp, zd[h][2], zd[h][3]);
-      }
+      const uint32_t cw = (uint32_t)(b0 + 4 * h);
+      tmem_ld_16x128b(tq + cC + cw, vc[h][0], vc[h][1]);
+      tmem_ld_16x128b(tq2 + cC + cw, vc[h][2], vc[h][3]);
+      tmem_ld_16x128b(tq + cD + cw, vd[h][0], vd[h][1]);
+      tmem_ld_16x128b(tq2 + cD + cw, vd[h][2], vd[h][3]);
     }
     tmem_wait_ld();
 #pragma unroll
@@ -349,10 +462,8 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
       float actp[4], actm[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const float zvk = do_z ? __uint_as_float(zv[h][k]) : 0.f;
-        const float zdk = do_z ? __uint_as_float(zd[h][k]) : 0.f;
-        const float C = fmaf(eps, zdk, __uint_as_float(wv[h][k])) + bias[k];
-        const float D = fmaf(eps, zvk, __uint_as_float(wd[h][k])) + dbias[k];
+        const float C = __uint_as_float(vc[h][k]) + G.bias[k];
+        const float D = fmaf(eps, __uint_as_float(vd[h][k]), G.dbias[k]);
         if (k == 2) {  // g: tanh(x) = 2 sigmoid(2x) - 1
           actp[k] = fmaf(sigm(2.f * (C + D)), 2.f, -1.f);
           actm[k] = fmaf(sigm(2.f * (C - D)), 2.f, -1.f);
@@ -361,19 +472,21 @@ __device__ void gate_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, con
           actm[k] = sigm(C - D);
         }
       }
-      const float cp = fmaf(actp[1], cprev[h].x, actp[0] * actp[2]);
-      const float cm = fmaf(actm[1], cprev[h].y, actm[0] * actm[2]);
+      const float cp = fmaf(actp[1], G.cprev[j][h].x, actp[0] * actp[2]);
+      const float cm = fmaf(actm[1], G.cprev[j][h].y, actm[0] * actm[2]);
       const float hp = actp[3] * fmaf(sigm(2.f * cp), 2.f, -1.f);
       const float hm = actm[3] * fmaf(sigm(2.f * cm), 2.f, -1.f);
       const int b = b0 + 4 * h + bq;
       if (unit_ok) {
         cell[b] = make_float2(cp, cm);
         if (b < s.B) {
-          const int row = 2 * g.Bp * p + b;
-          *reinterpret_cast<__half*>(out_tile + kmajor_offset(row, kk, kKt)) =
+          const float dh = hp - hm;
+          *reinterpret_cast<__half*>(out_tile + kmajor_offset(rM + b, kk, kKt)) =
               __float2half_rn(0.5f * (hp + hm));
-          *reinterpret_cast<__half*>(out_tile + kmajor_offset(row + g.Bp, kk, kKt)) =
-              __float2half_rn(0.5f * (hp - hm));
+          *reinterpret_cast<__half*>(out_tile + kmajor_offset(rD + b, kk, kKt)) =
+              __float2half_rn(dh * half_inv_eps);
+          *reinterpret_cast<__half*>(out_tile + kmajor_offset(rE + b, kk, kKt)) =
+              __float2half_rn(dh * half_eps);
         }
       }
     }
@@ -399,7 +512,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
   const float* th = s.params + (int64_t)T.e * L.P;
   const int vq = 128 * T.m + 32 * q4;  // first vocabulary row of the quarter
   const float bo_r = th[L.b_out + vq + lane];
-  const int t = a.t;
+  const int t = a.t_head;
   const int bq = lane & 3, r4 = lane >> 2;
   // rows of this thread: vq + r4 + 8 k, k = 0..3 (k = 2 h + reg)
   float bo[4];
@@ -419,26 +532,21 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
       for (int k = 0; k < 4; ++k) dbo[k] = __shfl_sync(0xffffffffu, dbo_r, r4 + 8 * k);
     }
     const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
+    const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
     for (int b0 = 0; b0 < g.Bp; b0 += 4) {
-      // [k]: W vbar, W dv, Z vbar, Z dv of row r4 + 8 k, sequence b0 + bq
-      uint32_t wv[4], wd[4], zv[4] = {0u, 0u, 0u, 0u}, zd[4] = {0u, 0u, 0u, 0u};
-      const uint32_t cw = (uint32_t)(2 * g.Bp * p + b0);
-      tmem_ld_16x128b(tq + cw, wv[0], wv[1]);
-      tmem_ld_16x128b(tq2 + cw, wv[2], wv[3]);
-      tmem_ld_16x128b(tq + cw + g.Bp, wd[0], wd[1]);
-      tmem_ld_16x128b(tq2 + cw + g.Bp, wd[2], wd[3]);
-      if (do_z) {
-        tmem_ld_16x128b(tq + kZCols + cw, zv[0], zv[1]);
-        tmem_ld_16x128b(tq2 + kZCols + cw, zv[2], zv[3]);
-        tmem_ld_16x128b(tq + kZCols + cw + g.Bp, zd[0], zd[1]);
-        tmem_ld_16x128b(tq2 + kZCols + cw + g.Bp, zd[2], zd[3]);
-      }
+      // [k]: C and D of row r4 + 8 k, sequence b0 + bq
+      uint32_t vc[4], vd[4];
+      const uint32_t cw = (uint32_t)b0;
+      tmem_ld_16x128b(tq + cC + cw, vc[0], vc[1]);
+      tmem_ld_16x128b(tq2 + cC + cw, vc[2], vc[3]);
+      tmem_ld_16x128b(tq + cD + cw, vd[0], vd[1]);
+      tmem_ld_16x128b(tq2 + cD + cw, vd[2], vd[3]);
       tmem_wait_ld();
       float lp[4], lm[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const float C = fmaf(eps, __uint_as_float(zd[k]), __uint_as_float(wv[k])) + bo[k];
-        const float D = fmaf(eps, __uint_as_float(zv[k]), __uint_as_float(wd[k])) + dbo[k];
+        const float C = __uint_as_float(vc[k]) + bo[k];
+        const float D = fmaf(eps, __uint_as_float(vd[k]), dbo[k]);
         lp[k] = C + D;
         lm[k] = C - D;
       }
@@ -508,27 +616,25 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 
 __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk);
 
-// grid: min(tasks, SMs) persistent CTAs (+ for the head, the embedding-part
-// blocks of the next timestep's operand), kThreads threads.
-template <bool HEAD, bool SPARSE>
-__global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_tasks,
-                                                                    int n_ctas) {
+// grid: min(tasks, SMs) persistent CTAs plus the embedding-part blocks of the
+// next timestep's operand, kThreads threads.
+template <bool SPARSE>
+__global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
   extern __shared__ uint8_t dyn_smem[];
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  if (HEAD && (int)blockIdx.x >= n_ctas) {
-    // the embedding part of timestep t + 1's operand (the head reads only
-    // the h part of the same buffer)
-    if (a.t + 1 < s.T)
-      xpart_block(a, const_cast<uint8_t*>(a.op_in), a.t + 1, blockIdx.x - n_ctas);
+  if ((int)blockIdx.x >= n_ctas) {
+    // the embedding part of timestep t + 1's operand (the gate tasks write
+    // its h part)
+    xpart_block(a, a.op_out, a.t_gate + 1, blockIdx.x - n_ctas);
     return;
   }
+  const int n_tasks = a.n_gate + a.n_head;
   uint8_t* smem = align1024(dyn_smem);
   const StageLayout SL = stage_layout(g);
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + kStages * SL.bytes);
   float2* red = reinterpret_cast<float2*>(smem + kStages * SL.bytes + 1024);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nst = HEAD ? g.Sh : g.S;
   const bool do_z = s.eps != 0.f;
   int* status = a.status;
   volatile int* abort = &ctl->abort;
@@ -536,8 +642,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   if (tid == 0) {
     ctl->abort = 0;
     for (int q = 0; q < kStages; ++q) {
-      // the loader's arrival (with the copies' bytes) and, when probes are
-      // generated, one arrival per Z warp: the MMA warp waits once per stage
+      // the loader's arrival with the copies' bytes and, when probes are
+      // generated, one arrival per Z warp
       mbar_init(&ctl->full[q], do_z ? 1 + kZWarps : 1);
       mbar_init(&ctl->slot_free[q], 1);
     }
@@ -554,112 +660,121 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   tc_fence_after();
   const uint32_t tmem = ctl->tmem_slot;
 
-  if (warp < kLoaders) {
-    // ---------------------------------------------------------------- loaders
-    // the whole warp walks the stages (so that it never sits diverged at the
-    // CTA barrier); lanes 0 and 1 issue one copy each (the copies of one
-    // thread complete one after another)
+  if (warp < kLoaders + (kLoaders > 1 ? 1 : 0) && warp != kMmaWarp) {
+    // --------------------------------------------------------------- loaders
+    // the whole warp walks the stages in order and waits for the slots of
+    // its own stages; lanes 0 and 1 issue the stage's two copies together
+    const int li = warp == 0 ? 0 : warp - 1;  // loader index: warps 0, 2, 3, ...
     uint32_t gs = 0;
-    int last_use = -1;
-    for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
-      const Task T = make_task<HEAD>(a, task);
-      for (int st = 0; st < nst; ++st, ++gs) {
+    bool done = true;
+    for (int task = blockIdx.x; task < n_tasks && done; task += n_ctas) {
+      const Task T = make_task(a, task);
+      for (int st = 0; st < T.nst; ++st, ++gs) {
+        if ((int)(gs % kLoaders) != li) continue;
         const int q = gs % kStages;
-        if (q != warp) continue;
         const uint32_t use = gs / kStages;
-        if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
-          continue;
+        if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
+          done = false;
+          break;
+        }
         uint8_t* slot = smem + q * SL.bytes;
         if (lane == 0) mbar_arrive_expect_tx(&ctl->full[q], kTileA + g.tileB);
         __syncwarp();
-        if (lane == 0)
-          bulk_g2s(slot + SL.a_off, T.a + (size_t)st * kTileA, kTileA, &ctl->full[q]);
-        else if (lane == 1)
-          bulk_g2s(slot + SL.b_off, T.b + (size_t)st * g.G * g.tileB, g.tileB, &ctl->full[q]);
-        last_use = (int)use;
+        if (lane < 2) {
+          uint8_t* dst = lane == 0 ? slot + SL.a_off : slot + SL.b_off;
+          const uint8_t* src =
+              lane == 0 ? T.a + (size_t)st * kTileA : T.b + (size_t)st * g.G * g.tileB;
+          bulk_g2s(dst, src, lane == 0 ? kTileA : g.tileB, &ctl->full[q]);
+        }
         __syncwarp();
       }
     }
-    // copies still in flight land before the CTA exits.  After an abort the
-    // Z warps stop arriving and this wait runs to its bound instead; copies
-    // take microseconds, the bound is tenths of a second.
-    if (last_use >= 0) mbar_wait(&ctl->full[warp], (uint32_t)last_use & 1u);
+    // The copies of the last stage of each slot land before the CTA exits;
+    // the loader that issued that stage waits for them (earlier phases of a
+    // slot completed before its later copies were issued).  After an abort
+    // the copies issued so far are not tracked: the slot waits that failed
+    // above were bounded, and copies take microseconds against that bound.
+    if (done) {
+#pragma unroll
+      for (int q = 0; q < kStages; ++q) {
+        if ((int)gs <= q) continue;
+        const uint32_t last = gs - 1 - ((gs - 1 - (uint32_t)q) % kStages);  // last stage of slot q
+        if ((int)(last % kLoaders) == li) mbar_wait(&ctl->full[q], (last / kStages) & 1u);
+      }
+    }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
-    // the whole warp waits; lane 0 issues the MMAs and commits
-    {
-      const uint32_t idesc_w = idesc_f16_f32(128, g.rowsB);
+    if (lane == 0) {
       const uint32_t idesc_z = idesc_f16_f32(128, 2 * g.Bp);
-      // descriptors of slot 0; slot q is q * SL.bytes further, k16 = 1 is
-      // 256 bytes further (two core matrices along K)
+      // W covers the P probes of the group (2 Bp P columns); a group with
+      // one valid probe still multiplies the whole window (the rows of the
+      // missing probe are zero)
+      const uint32_t idesc_w = idesc_f16_f32(128, 2 * g.Bp * g.P);
+      // descriptors of slot 0; slot q is q * SL.bytes further
       const uint64_t d0 = smem_desc(smem_u32(smem), kLbo, kSbo);
       const uint32_t hi = (uint32_t)(d0 >> 32);
       const uint32_t lo0 = (uint32_t)d0;
       const uint32_t slot_step = SL.bytes >> 4;
       const uint32_t a_lo0 = lo0 + (SL.a_off >> 4), b_lo0 = lo0 + (SL.b_off >> 4);
-      const uint32_t z_lo0 = lo0 + (SL.z_off >> 4);
-      const uint32_t zp_step = kTileA >> 4;                       // next probe's Z tile
-      const uint32_t bp_step = (uint32_t)(2 * g.Bp / 8) * (kSbo >> 4);  // next probe's rows
-      const uint32_t dz_step = (uint32_t)(2 * g.Bp);                    // next probe's columns
-      uint32_t gs = 0;
+      const uint32_t grp_step = kSbo >> 4;                     // 8 operand rows
+      const uint32_t w_row = (uint32_t)(g.Bp / 8) * grp_step;  // the W window starts at row Bp
+      const uint32_t z1_row = (uint32_t)(4 * g.Bp / 8) * grp_step;
+      const uint32_t dz1 = (uint32_t)(2 * g.Bp);
+      RingPos rp = {0u, 0u};
       int k = 0;
       for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-        const Task T = make_task<HEAD>(a, task);
+        const Task T = make_task(a, task);
         const int buf = k & 1;
-        if (k >= 2) wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status);
+        if (k >= 2 &&
+            !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
+          break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(buf * kAccCols);
+        const uint32_t d = tmem + (uint32_t)buf * kAccCols;
         const int np = do_z ? T.p_valid : 0;
-        for (int st = 0; st < nst; ++st, ++gs) {
-          const int q = gs % kStages;
-          const uint32_t use = gs / kStages;
-          const bool ok = wait_or_abort(&ctl->full[q], use & 1u, abort, status);
-          tc_fence_after();
-          if (ok && lane == 0) {
-            const uint32_t so = (uint32_t)q * slot_step;
-            const uint32_t acc0 = st > 0 ? 1u : 0u;
-            if (np == 2)
-              issue_stage<2>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
-                             idesc_z, dz_step, acc0);
-            else if (np == 1)
-              issue_stage<1>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
-                             idesc_z, dz_step, acc0);
-            else
-              issue_stage<0>(d, a_lo0 + so, b_lo0 + so, z_lo0 + so, hi, zp_step, bp_step, idesc_w,
-                             idesc_z, dz_step, acc0);
-          }
-          if (lane == 0) mma_commit(&ctl->slot_free[q]);
-          __syncwarp();
-        }
-        if (lane == 0) mma_commit(&ctl->acc_full[buf]);
-        __syncwarp();
+        bool ok;
+        if (np == 2)
+          ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
+                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
+                           status);
+        else if (np == 1)
+          ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
+                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
+                           status);
+        else
+          ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
+                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
+                           status);
+        if (!ok) break;
+        mma_commit(&ctl->acc_full[buf]);
       }
       // every MMA of this CTA completes before its tensor memory is freed
-      if (lane == 0) mma_commit(&ctl->mma_done);
+      mma_commit(&ctl->mma_done);
       mbar_wait(&ctl->mma_done, 0);
     }
-  } else if (warp < kEpiWarp0) {
+    __syncwarp();
+  } else if (warp >= kZWarp0 && warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
-    // Thread (probe gtid / 128, row gtid % 128).  The raw words of the next
-    // stage are drawn before waiting for its slot, so the Philox rounds
-    // overlap the wait instead of following it.
+    // Thread (probe gtid / 128, row gtid % 128 = TMEM lane).  The raw words
+    // of the next stage are drawn before waiting for its slot, so the Philox
+    // rounds overlap the wait instead of following it.
     if (do_z) {
       const int gtid = tid - kZWarp0 * 32;
       const int r = gtid & 127, pz = gtid >> 7;
+      const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kZCol0 + 32u * pz;
       uint32_t gs = 0;
-      for (int task = blockIdx.x; task < n_tasks; task += n_ctas) {
-        const Task T = make_task<HEAD>(a, task);
-        const bool active = pz < T.p_valid;
+      bool alive = true;
+      for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
+        const Task T = make_task(a, task);
+        const bool active = pz < T.p_valid;  // uniform over the warp
         const ProbeKey pk =
             make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pz));
         const ProbeKey pka = activity_key(pk);
         ZSlot cache, cache_a;
         cache.blk = 0xFFFFFFFFu;
         cache_a.blk = 0xFFFFFFFFu;
-        const int split = HEAD ? nst : g.Sx;
-        const int64_t seg0 = z_param<HEAD>(a, T, r, 0);
-        const int64_t seg1 = z_param<HEAD>(a, T, r, split) - (int64_t)kKt * split;
-        uint8_t* zrow = smem + SL.z_off + pz * kTileA + kmajor_offset(r, 0, kKt);
+        const int split = T.head ? T.nst : g.Sx;
+        const int64_t seg0 = z_param(a, T, r, 0);
+        const int64_t seg1 = z_param(a, T, r, split) - (int64_t)kKt * split;
         uint32_t raw[kKt / 32] = {}, act[kKt / 32] = {};
         if (active) {
 #pragma unroll
@@ -668,23 +783,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
             if (SPARSE) act[w] = z_run_raw(pka, seg0 + 32 * w, cache_a);
           }
         }
-        for (int st = 0; st < nst; ++st, ++gs) {
+        for (int st = 0; st < T.nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
           // after an abort the generators stop: an arrival on a phase that
           // can no longer complete would overfill it
-          if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status))
+          if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
+            alive = false;
             break;
-          if (active) {
-            uint8_t* zr = zrow + q * SL.bytes;
-#pragma unroll
-            for (int w = 0; w < kKt / 32; ++w)
-              store_z_row_at<SPARSE>(zr + w * 4 * 128, raw[w], act[w]);
           }
-          fence_async_smem();
+          tc_fence_after();
+          if (active) {
+            uint32_t zw[kKt / 2];
+#pragma unroll
+            for (int w = 0; w < kKt / 32; ++w) z_run_pairs<SPARSE>(raw[w], act[w], zw + 16 * w);
+            tmem_st32(trow + 64u * (uint32_t)q, zw);
+            tmem_wait_st();
+          }
+          tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->full[q]);
-          if (active && st + 1 < nst) {
+          if (active && st + 1 < T.nst) {
             const int64_t p1 = (st + 1 < split ? seg0 : seg1) + (int64_t)kKt * (st + 1);
 #pragma unroll
             for (int w = 0; w < kKt / 32; ++w) {
@@ -695,26 +814,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         }
       }
     }
-  } else {
+  } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
     int k = 0;
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-      const Task T = make_task<HEAD>(a, task);
+      const Task T = make_task(a, task);
       const int buf = k & 1;
-      wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status);
+      GatePre G;
+      if (!wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status)) break;
+      if (!T.head) gate_prepare(a, T, q4, ew >> 2, G);
       tc_fence_after();
-      const uint32_t tacc = tmem + (uint32_t)(buf * kAccCols);
-      if (HEAD) {
+      const uint32_t tacc = tmem + (uint32_t)buf * kAccCols;
+      if (T.head)
         head_epilogue(a, T, tacc, q4, ew, red);
-      } else {
-        for (int p = ew >> 2; p < T.p_valid; p += kEpiProbeStep) {
-          const ProbeKey pk =
-              make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + p));
-          gate_epilogue(a, T, tacc, pk, q4, p);
-        }
-      }
+      else
+        gate_finish(a, T, tacc, q4, G);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
@@ -725,7 +841,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 }
 
-// Embedding part of the operand of timestep t: x = Emb[byte_t], dx = eps z_emb.
+// Embedding part of the operand of timestep t: per probe p of the group the
+// rows vbar = Emb[byte_t], dhat = z_emb[byte_t] (+-1, or 0) and eps^2 dhat.
 // Block `blk` of Sx * G * N writes one (expert, stage, group) tile.
 __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   const TcGeom& g = a.g;
@@ -734,27 +851,29 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   const int e = blk / (g.G * g.Sx);
   const Layout& L = s.lay;
   const float* th = s.params + (int64_t)e * L.P;
+  const float eps2 = s.eps * s.eps;
   uint8_t* tile = op + (((size_t)e * g.S + st) * g.G + grp) * g.tileB;
   const int chunks = g.rowsB * (kKt / 8);
   for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
     const int row = c / (kKt / 8), kc = c % (kKt / 8);
-    const int p = row / (2 * g.Bp), rr = row % (2 * g.Bp);
+    const int blkr = row / g.Bp, b = row % g.Bp;  // row block 0..3P-1, sequence
+    const int p = blkr < 3 ? 0 : 1;
+    const bool mean = blkr == row_mean(p), e2 = blkr == row_e2(p);
     const int i = grp * g.P + p;
-    const bool delta = rr >= g.Bp;
-    const int b = delta ? rr - g.Bp : rr;
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
     if (i < s.n_pert && b < s.B) {
       const int y = s.bytes[seq_offset(s, e, i, b) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
       ProbeBits bits = {0u, 0u};
-      if (delta && s.eps != 0.f)
+      if (!mean && s.eps != 0.f)
         bits = probe_bits(make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i), p0, s.sparse);
+      const float mag = e2 ? eps2 : 1.f;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         float x = 0.f;
         if (k0 + j < g.E)
-          x = delta ? eps_z((bits.neg >> j) & 1u, (bits.act >> j) & 1u, s.eps) : th[p0 + j];
+          x = mean ? th[p0 + j] : eps_z((bits.neg >> j) & 1u, (bits.act >> j) & 1u, mag);
         v[j] = __float2half_rn(x);
       }
     } else {
@@ -770,8 +889,8 @@ __global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
   xpart_block(a, op, t, blockIdx.x);
 }
 
-// fp16 A tiles of the gate weights ([x part | h part], rows unit-major:
-// tile row r = 4 * unit + gate) and of the head weights.
+// fp16 A tiles of the gate weights ([x part | h part], gate-major rows) and
+// of the head weights.
 // grid (MT * S + 2 * Sh, N), 128 threads: thread r writes row r of a tile.
 __global__ void prep_tiles_kernel(const TcArgs a) {
   const TcGeom& g = a.g;
@@ -838,7 +957,8 @@ reduce_tc_kernel(const float* __restrict__ pm, const float* __restrict__ ps,
     }
     sp += (double)nll[0];
     sm += (double)nll[1];
-    sd += (double)(nll[0] - nll[1]);
+    // the difference in fp64: exact for any two fp32 values
+    sd += (double)nll[0] - (double)nll[1];
   }
   red[0][threadIdx.x] = sp;
   red[1][threadIdx.x] = sm;
@@ -873,9 +993,13 @@ reduce_tc_kernel(const float* __restrict__ pm, const float* __restrict__ ps,
 // Debug GEMM: D[128][N] = A[128][K] * B[N][K]^T through the same descriptors,
 // instruction descriptor and TMEM read-back as the forward kernels.  A and B
 // are fp16 row-major in global memory; 128 threads stage them into the
-// canonical layout (K <= 256, N <= 256, both multiples of 16).
+// canonical layout (K <= 256, N <= 256, both multiples of 16).  With
+// a_in_tmem, A is stored into tensor memory instead (lane = row, column c =
+// the k pair 2c, 2c + 1) and the MMA takes it from there, as the probe
+// tiles of the forward kernel.
 __global__ void __launch_bounds__(128, 1)
-debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, int* status) {
+debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, int a_in_tmem,
+                     int* status) {
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = align1024(dyn_smem);
   uint8_t* sa = smem;
@@ -887,11 +1011,12 @@ debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, i
     mbar_init(&bar, 1);
     mbar_fence_init();
   }
-  if (tid < 32) tmem_alloc(&slot, 256);
+  if (tid < 32) tmem_alloc(&slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = slot;
+  const int warp = tid >> 5, lane = tid & 31;
   for (int c = tid; c < 128 * (K / 8); c += 128) {
     const int r = c / (K / 8), kc = c % (K / 8);
     *reinterpret_cast<uint4*>(sa + kmajor_offset(r, 8 * kc, K)) =
@@ -902,19 +1027,38 @@ debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, i
     *reinterpret_cast<uint4*>(sb + kmajor_offset(r, 8 * kc, K)) =
         *reinterpret_cast<const uint4*>(B + (size_t)r * K + 8 * kc);
   }
+  const uint32_t ta = tmem + 256;  // A in TMEM: columns 256 .. 256 + K / 2
+  if (a_in_tmem) {
+    // thread = row (lane quarter of its warp), 16 columns (32 k) per store
+    const uint32_t trow = ta + ((uint32_t)(32 * warp) << 16);
+    const uint32_t* arow = reinterpret_cast<const uint32_t*>(A + (size_t)(32 * warp + lane) * K);
+    for (int c0 = 0; c0 < K / 2; c0 += 16) {
+      uint32_t r[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) r[j] = arow[c0 + j];
+      tmem_st16(trow + c0, r);
+    }
+    tmem_wait_st();
+  }
   fence_async_smem();
+  tc_fence_before();
   __syncthreads();
   if (tid == 0) {
     tc_fence_after();
     const uint32_t idesc = idesc_f16_f32(128, N);
-    for (int k16 = 0; k16 < K / 16; ++k16)
-      mma_f16_ss(tmem, smem_desc(smem_u32(sa) + k16 * 256, 128, K * 16),
-                 smem_desc(smem_u32(sb) + k16 * 256, 128, K * 16), idesc, k16 > 0 ? 1u : 0u);
+    const uint64_t db = smem_desc(smem_u32(sb), 128, K * 16);
+    for (int k16 = 0; k16 < K / 16; ++k16) {
+      if (a_in_tmem)
+        mma_f16_ts_lohi(tmem, ta + 8 * k16, (uint32_t)db + 16 * k16, (uint32_t)(db >> 32), idesc,
+                        k16 > 0 ? 1u : 0u);
+      else
+        mma_f16_ss(tmem, smem_desc(smem_u32(sa) + k16 * 256, 128, K * 16),
+                   smem_desc(smem_u32(sb) + k16 * 256, 128, K * 16), idesc, k16 > 0 ? 1u : 0u);
+    }
     mma_commit(&bar);
   }
   if (!mbar_wait(&bar, 0) && tid == 0) atomicCAS(status, 0, kStatusTimeout);
   tc_fence_after();
-  const int warp = tid >> 5, lane = tid & 31;
   for (int c0 = 0; c0 < N; c0 += 8) {
     float v[8];
     tmem_ld8(tmem + ((uint32_t)(32 * warp) << 16) + c0, v);
@@ -922,7 +1066,7 @@ debug_tc_gemm_kernel(const __half* A, const __half* B, float* D, int N, int K, i
   }
   tc_fence_before();
   __syncthreads();
-  if (tid < 32) tmem_dealloc(tmem, 256);
+  if (tid < 32) tmem_dealloc(tmem, 512);
 }
 
 size_t kernel_smem_bytes(const TcGeom& g) {
@@ -957,13 +1101,13 @@ TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T) 
   g.S = g.Sx + g.Sh;
   g.MT = g.Hp / 32;
   g.Bp = (B + 7) / 8 * 8;
-  int P = 64 / g.Bp;  // rowsB = 2 Bp P <= 128 TMEM columns per product
-  if (P > 2) P = 2;
+  // the accumulator of a group, 2 Bp P columns, fits one 128-column buffer
+  int P = g.Bp <= 32 ? 2 : 1;
   if (P > n_pert) P = n_pert;
   if (P < 1) P = 1;
   g.P = P;
   g.G = (n_pert + P - 1) / P;
-  g.rowsB = 2 * g.Bp * P;
+  g.rowsB = 3 * g.Bp * P;
   g.tileB = (uint32_t)g.rowsB * kKt * 2;
   g.n_experts = n_experts;
   g.n_pert = n_pert;
@@ -989,27 +1133,27 @@ TcSizes tc_sizes(const TcGeom& g) {
 cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
                               cudaStream_t stream) {
   const size_t smem = kernel_smem_bytes(g);
-  auto gate_kernel = s.sparse ? tc_persistent_kernel<false, true> : tc_persistent_kernel<false, false>;
-  auto head_kernel = s.sparse ? tc_persistent_kernel<true, true> : tc_persistent_kernel<true, false>;
-  cudaError_t e = cudaFuncSetAttribute(gate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  auto kernel = s.sparse ? tc_persistent_kernel<true> : tc_persistent_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const TcSizes z = tc_sizes(g);
   TcArgs a;
   a.sw = s;
   a.g = g;
-  a.t = 0;
   a.w16 = tb.w16;
   a.wo16 = tb.wo16;
-  a.op_in = tb.op[0];
-  a.op_out = tb.op[1];
   a.cst = tb.cst;
   a.pm = tb.pm;
   a.ps = tb.ps;
   a.ply = tb.ply;
   a.status = status;
+  a.t_gate = -1;
+  a.t_head = -1;
+  a.n_gate = 0;
+  a.n_head = 0;
+  a.op_in = tb.op[0];
+  a.op_out = tb.op[0];
 
   trace_begin(SOMA_TRACE_PREP, stream);
   prep_tiles_kernel<<<dim3(g.MT * g.S + 2 * g.Sh, g.n_experts), 128, 0, stream>>>(a);
@@ -1022,22 +1166,21 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   const int sms = sm_count();
   const int gate_tasks = g.n_experts * g.MT * g.G;
   const int head_tasks = g.n_experts * 2 * g.G;
-  const int gate_ctas = gate_tasks < sms ? gate_tasks : sms;
-  const int head_ctas = head_tasks < sms ? head_tasks : sms;
-  for (int t = 0; t < s.T; ++t) {
-    a.t = t;
+  // launch t: the gate of t (t < T) and the head of t - 1 (t >= 1), both
+  // reading the operand [x_t | h_{t-1}]
+  for (int t = 0; t <= s.T; ++t) {
+    a.t_gate = t < s.T ? t : -1;
+    a.t_head = t - 1;
+    a.n_gate = t < s.T ? gate_tasks : 0;
+    a.n_head = t >= 1 ? head_tasks : 0;
     a.op_in = tb.op[t & 1];
     a.op_out = tb.op[(t + 1) & 1];
+    const int tasks = a.n_gate + a.n_head;
+    const int ctas = tasks < sms ? tasks : sms;
+    const int extra = t + 1 < s.T ? xblocks : 0;
     trace_begin(SOMA_TRACE_GATE, stream);
-    gate_kernel<<<gate_ctas, kThreads, smem, stream>>>(a, gate_tasks, gate_ctas);
+    kernel<<<ctas + extra, kThreads, smem, stream>>>(a, ctas);
     trace_end(SOMA_TRACE_GATE, stream);
-    // head of timestep t (h part of the operand of t + 1) and, in the same
-    // launch, the embedding part of that operand
-    a.op_in = tb.op[(t + 1) & 1];
-    trace_begin(SOMA_TRACE_HEAD, stream);
-    head_kernel<<<head_ctas + (t + 1 < s.T ? xblocks : 0), kThreads, smem, stream>>>(
-        a, head_tasks, head_ctas);
-    trace_end(SOMA_TRACE_HEAD, stream);
   }
   return cudaGetLastError();
 }
@@ -1052,14 +1195,15 @@ cudaError_t launch_reduce_tc(const TcBuffers& tb, int pairs, int n_sign, int B, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K, int* status,
-                                 cudaStream_t stream) {
+cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K,
+                                 int a_in_tmem, int* status, cudaStream_t stream) {
   const size_t smem = (size_t)(128 + N) * K * 2 + 1024;
   cudaError_t e = cudaFuncSetAttribute(debug_tc_gemm_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   debug_tc_gemm_kernel<<<1, 128, smem, stream>>>(static_cast<const __half*>(A),
-                                                 static_cast<const __half*>(B), D, N, K, status);
+                                                 static_cast<const __half*>(B), D, N, K, a_in_tmem,
+                                                 status);
   return cudaGetLastError();
 }
 

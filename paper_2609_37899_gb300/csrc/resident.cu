@@ -2,12 +2,13 @@
 // resident in one CTA (tcgen05 / TMEM).
 //
 // One CTA runs one (expert, probe) pair, both signs, over all T timesteps in
-// the mean/difference form of forward_tc.cu:
-//   a+- = C +- D,  C = W vbar + eps (Z dv) + b,  D = W dv + eps (Z vbar) + eps z_b.
+// the mean/difference form of forward_tc.cu, with the difference operand
+// scaled by 1 / eps (dhat = dv / eps, an O(1) quantity):
+//   a+- = C +- eps D,  C = W vbar + eps^2 (Z dhat) + b,  D = W dhat + Z vbar + z_b.
 // The gate weights W = [W_ih | W_hh], the head weights W_out and the probe
 // tiles Z of this pair are converted to fp16 tiles in shared memory once,
 // and the probes are therefore drawn once per step, not once per timestep.
-// The operand [vbar | dv] (rows) x [x | h] (K) also lives in shared memory,
+// The operand [vbar | dhat] (rows) x [x | h] (K) also lives in shared memory,
 // in two buffers: buffer t % 2 holds [x_t | h_{t-1}].  Cell states stay in
 // registers, and the losses are summed in the CTA.  Per timestep t, after
 // the barrier that publishes buffer t % 2:
@@ -71,10 +72,10 @@ ResGeom make_res_geom(const Layout& lay, int B, int T) {
   r.zg = o; o = res_align(o + r.MTg * gate_tile);
   r.wo = o; o = res_align(o + 2 * head_tile);
   r.zo = o; o = res_align(o + 2 * head_tile);
-  r.opsz = 2u * r.Bp * r.K * 2;  // one operand buffer [vbar | dv] x K, fp16
+  r.opsz = 2u * r.Bp * r.K * 2;  // one operand buffer [vbar | dhat] x K, fp16
   r.op = o; o = res_align(o + 2u * r.opsz);
   r.emb = o; o += 256u * r.Ek * 2;   // fp16 Emb rows [V][Ek]
-  r.dx = o; o += 256u * r.Ek * 2;    // fp16 eps z of the Emb rows
+  r.dx = o; o += 256u * r.Ek * 2;    // fp16 z of the Emb rows (dhat of x = z_emb)
   r.red = o; o += 2u * 4 * 2 * r.Bp * sizeof(float2);  // [half][quarter][sign][Bp]
   r.ylog = o; o += 2u * r.Bp * sizeof(float);          // [sign][Bp]
   o = (o + 7u) & ~7u;
@@ -118,6 +119,9 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
   const float eps = s.eps;
   const bool do_z = eps != 0.f;
+  const float eps2 = eps * eps;
+  // dhat_h = (h+ - h-) / (2 eps); 0 when eps = 0 (both signs coincide)
+  const float half_inv_eps = do_z ? 0.5f / eps : 0.f;
   uint64_t* gate_bar = reinterpret_cast<uint64_t*>(smem + g.ctl);
   uint64_t* head_bar = reinterpret_cast<uint64_t*>(smem + g.ctl + 8);  // [2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + g.ctl + 24);
@@ -185,8 +189,9 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   }
   for (int c = tid; c < 2 * (2 * g.Bp * g.K / 8); c += kResThreads)
     reinterpret_cast<uint4*>(smem + g.op)[c] = make_uint4(0u, 0u, 0u, 0u);
-  // the embedding table and its eps z, so that the operand of a timestep is
-  // gathered from shared memory
+  // the embedding table and its probe z (the scaled difference of the two
+  // signs' inputs, dhat_x = (x+ - x-) / (2 eps) = z_emb), so that the operand
+  // of a timestep is gathered from shared memory
   for (int c = tid; c < 256 * (g.Ek / 8); c += kResThreads) {
     const int v = c / (g.Ek / 8), k0 = 8 * (c % (g.Ek / 8));
     const int64_t p0 = L.emb + (int64_t)v * g.E + k0;
@@ -198,7 +203,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
     for (int j = 0; j < 8; ++j) {
       const bool ok = j < kmax;
       x[j] = __float2half_rn(ok ? th[p0 + j] : 0.f);
-      d[j] = __float2half_rn(ok ? eps_z((zb.neg >> j) & 1u, (zb.act >> j) & 1u, eps) : 0.f);
+      d[j] = ok ? z_half(zb, j) : __float2half_rn(0.f);
     }
     reinterpret_cast<uint4*>(smem + g.emb)[c] = *reinterpret_cast<const uint4*>(x);
     reinterpret_cast<uint4*>(smem + g.dx)[c] = *reinterpret_cast<const uint4*>(d);
@@ -271,7 +276,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
   const int xb = x_delta ? xrow - g.Bp : xrow;
   const uint4* xtab = reinterpret_cast<const uint4*>(smem + (x_delta ? g.dx : g.emb));
   // the embedding part of operand buffer 0 (x_0; h_{-1} = 0): rows
-  // [vbar (Bp) | dv (Bp)], 16-byte chunks of the Emb / eps z tables
+  // [vbar (Bp) | dhat (Bp)], 16-byte chunks of the Emb / z tables
   int ynext = 0;
   if (xc >= 0 && xb < g.B) {
     const int y0 = s.bytes[seq_offset(s, e, i, xb)];
@@ -355,8 +360,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
             float actp[4], actm[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-              const float C = fmaf(eps, __uint_as_float(zd[h][k]), __uint_as_float(wv[h][k])) + bias[k];
-              const float D = fmaf(eps, __uint_as_float(zv[h][k]), __uint_as_float(wd[h][k])) + dbias[k];
+              const float C = fmaf(eps2, __uint_as_float(zd[h][k]), __uint_as_float(wv[h][k])) + bias[k];
+              const float D = fmaf(eps, __uint_as_float(wd[h][k]) + __uint_as_float(zv[h][k]), dbias[k]);
               if (k == 2) {
                 actp[k] = fmaf(sigm_res(2.f * (C + D)), 2.f, -1.f);
                 actm[k] = fmaf(sigm_res(2.f * (C - D)), 2.f, -1.f);
@@ -376,7 +381,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
               *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(b, g.Ek + U, g.K)) =
                   __float2half_rn(0.5f * (hp + hm));
               *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(g.Bp + b, g.Ek + U, g.K)) =
-                  __float2half_rn(0.5f * (hp - hm));
+                  __float2half_rn((hp - hm) * half_inv_eps);
             }
           }
         }
@@ -420,8 +425,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
         float lp[4], lm[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          const float C = fmaf(eps, __uint_as_float(zd[k]), __uint_as_float(wv[k])) + bo[k];
-          const float D = fmaf(eps, __uint_as_float(zv[k]), __uint_as_float(wd[k])) + dbo[k];
+          const float C = fmaf(eps2, __uint_as_float(zd[k]), __uint_as_float(wv[k])) + bo[k];
+          const float D = fmaf(eps, __uint_as_float(wd[k]) + __uint_as_float(zv[k]), dbo[k]);
           lp[k] = C + D;
           lm[k] = C - D;
         }
@@ -473,7 +478,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
         }
         acc[tid] += (double)nll[0];
         acc[g.Bp + tid] += (double)nll[1];
-        acc[2 * g.Bp + tid] += (double)(nll[0] - nll[1]);
+        acc[2 * g.Bp + tid] += (double)nll[0] - (double)nll[1];  // exact in fp64
       }
     }
 

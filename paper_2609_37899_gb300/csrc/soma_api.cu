@@ -45,7 +45,7 @@ constexpr size_t kAlign = 256;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Workspace of one sweep with `n_pert` probes and `n_sign` signs.  Batches of
-// up to 128 sequences run on the tensor cores (both signs always); larger
+// up to 64 sequences run on the tensor cores (both signs always); larger
 // batches on the fp32 CUDA-core kernels.
 struct WsPlan {
   bool res;  // the resident small-expert kernel: no scratch but the coefficients
@@ -375,14 +375,24 @@ int soma_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int c
   return cuda_status(launch_debug_philox(seed, ctr4, out4, count, (cudaStream_t)stream));
 }
 
-int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
-                       void* stream) {
+static int debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                         int a_in_tmem, void* stream) {
   if (!a || !b || !d || !aligned16(a) || !aligned16(b) || n < 16 || n > 256 || n % 16 ||
       k < 16 || k > 256 || k % 16)
     return SOMA_ERR_INVALID_ARG;
   int* status = status_ptr();
   if (!status) return SOMA_ERR_CUDA;
-  return cuda_status(launch_debug_tc_gemm(a, b, d, n, k, status, (cudaStream_t)stream));
+  return cuda_status(launch_debug_tc_gemm(a, b, d, n, k, a_in_tmem, status, (cudaStream_t)stream));
+}
+
+int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                       void* stream) {
+  return debug_tc_gemm(a, b, d, n, k, 0, stream);
+}
+
+int soma_debug_tc_gemm_ts(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
+                          void* stream) {
+  return debug_tc_gemm(a, b, d, n, k, 1, stream);
 }
 
 int soma_debug_wait_timeout(uint32_t max_polls, void* stream) {

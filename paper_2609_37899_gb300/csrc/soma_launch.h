@@ -28,9 +28,10 @@ cudaError_t launch_forward_simt(const Sweep& s, const ForwardBuffers& fb, cudaSt
 
 // ---- tensor-core path ------------------------------------------------------
 // Geometry of one sweep on the tensor cores.  K of the gate GEMM is
-// [x part padded to Ep | h part padded to Hp], in stages of 32; rows are
-// 32-unit tiles of 4 gates; sequences are padded to Bp and P probes share one
-// operand group tile of rowsB = 2 Bp P rows ([hbar | dh] per probe).
+// [x part padded to Ep | h part padded to Hp], in stages of 64; rows are
+// 32-unit tiles of 4 gates; sequences are padded to Bp and P <= 2 probes
+// share one operand group tile of rowsB = 3 Bp P rows (vbar, dhat and
+// eps^2 dhat per probe, forward_tc.cu).
 struct TcGeom {
   int E, H, Ep, Hp, S, Sx, Sh, MT, Bp, P, G, rowsB;
   uint32_t tileB;  // bytes of one operand group tile of one stage
@@ -59,8 +60,8 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
 cudaError_t launch_reduce_tc(const TcBuffers& tb, int pairs, int n_sign, int B, int T, float eps,
                              float* losses_out, float* coef_out, float* coef_ws, int* status,
                              cudaStream_t stream);
-cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K, int* status,
-                                 cudaStream_t stream);
+cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K,
+                                 int a_in_tmem, int* status, cudaStream_t stream);
 
 // losses_out [pairs][n_sign]; coef_out / coef_ws [pairs] (either may be null).
 cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B, int T, float eps,

@@ -27,7 +27,7 @@ reduce_losses_kernel(const float* __restrict__ nll, int n_sign, int BT, float ep
     if (n_sign == 2) {
       const float b = np[BT + j];
       sm += (double)b;
-      sd += (double)(a - b);  // exact: a and b are within a factor of two
+      sd += (double)a - (double)b;  // exact in fp64 for any two fp32 values
     }
   }
   red[0][threadIdx.x] = sp;

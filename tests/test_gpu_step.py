@@ -72,6 +72,34 @@ def test_ragged_shapes_full_step(oracle_mod, N, E, H, B, T, n):
     _full_parity(oracle_mod, theta, bx, E, H, n, 1e-3, 1e-2, 77, 5)
 
 
+# The difference operand is stored as dhat = (v+ - v-) / (2 eps), an O(1)
+# quantity, so the fp16 rounding of the difference stays relative at any eps.
+# The sweep covers the resident kernel (tiny, H <= 64), the persistent kernel
+# with one probe per operand group (B = 35) and with two (H = 96, B = 8, an
+# odd probe count so the last group holds one probe).
+EPS_SHAPES = {
+    "tiny": None,
+    "ragged_p1": (2, 33, 65, 35, 40, 2),
+    "persistent_p2": (2, 16, 96, 8, 12, 5),
+}
+
+
+@pytest.mark.parametrize("eps", [1e-2, 1e-3, 1e-4])
+@pytest.mark.parametrize("shape", list(EPS_SHAPES))
+def test_eps_sweep_full_step(oracle_mod, shape, eps):
+    if shape == "tiny":
+        c = inputs.CONFIGS["tiny"]
+        theta = inputs.config_params("tiny")
+        bx = inputs.config_batch("tiny")
+        E, H, n, lr = c["E"], c["H"], c["n_pert"], c["lr"]
+    else:
+        N, E, H, B, T, n = EPS_SHAPES[shape]
+        theta = inputs.init_params(N, E, H, seed=N + H, std=None)
+        bx = inputs.expert_batch(N, B, T, 2, seed=4, step=0)
+        lr = 1e-2
+    _full_parity(oracle_mod, theta, bx, E, H, n, eps, lr, 11, 3)
+
+
 def test_eps_zero_is_the_unperturbed_loss():
     E, H, N, n = 16, 40, 2, 4
     theta = inputs.init_params(N, E, H, seed=1, std=0.2)
@@ -193,7 +221,7 @@ def test_init_experts():
 
 
 def test_large_batch_uses_the_cuda_core_path(oracle_mod):
-    # more than 128 sequences per expert: the fp32 CUDA-core kernels
+    # more than 64 sequences per expert: the fp32 CUDA-core kernels
     N, E, H, B, T, n = 1, 3, 5, 130, 4, 2
     theta = inputs.init_params(N, E, H, seed=21, std=0.3)
     bx = inputs.expert_batch(N, B, T, 1, seed=22, step=0)
@@ -203,7 +231,7 @@ def test_large_batch_uses_the_cuda_core_path(oracle_mod):
 @pytest.mark.parametrize("n", [160, 304])
 def test_many_tasks_per_cta(oracle_mod, n):
     # more probe groups than SMs: every persistent CTA runs several gate and
-    # head tasks (and the head launch carries the embedding-operand blocks)
+    # head tasks (and each launch carries the embedding-operand blocks)
     N, E, H, B, T = 1, 64, 96, 8, 6
     theta = inputs.init_params(N, E, H, seed=n, std=None)
     bx = inputs.expert_batch(N, B, T, 2, seed=31, step=0)

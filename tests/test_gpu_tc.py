@@ -14,14 +14,15 @@ pytestmark = pytest.mark.gpu
 OUT = os.environ.get("SOMA_TEST_DUMP", "")
 
 
+@pytest.mark.parametrize("a_in_tmem", [False, True])
 @pytest.mark.parametrize("n", [16, 32, 64, 128, 256])
 @pytest.mark.parametrize("k", [16, 32, 64, 256])
-def test_tc_gemm_small_integers_exact(n, k):
+def test_tc_gemm_small_integers_exact(n, k, a_in_tmem):
     # entries in -2..2: every product and partial sum is exact in fp32
     g = torch.Generator().manual_seed(n * 1000 + k)
     a = torch.randint(-2, 3, (128, k), generator=g).to(torch.float16)
     b = torch.randint(-2, 3, (n, k), generator=g).to(torch.float16)
-    d = api().debug_tc_gemm(a.cuda(), b.cuda()).cpu()
+    d = api().debug_tc_gemm(a.cuda(), b.cuda(), a_in_tmem=a_in_tmem).cpu()
     assert api().get_status() == 0
     ref = a.float() @ b.float().T
     if OUT and not torch.equal(d, ref):
