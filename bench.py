@@ -116,10 +116,8 @@ def gate_kernel_name(B, resident):
     if resident:
         return ("res_kernel (tcgen05, the whole recurrence of a probe pair resident in one CTA: "
                 "gate GEMM + cell + head + loss)")
-    if B <= 64:
-        return ("tc_persistent_kernel (tcgen05; launch t = gate GEMM + fused cell of timestep t "
-                "and output head + softmax partials of t - 1)")
-    return "gate_step_kernel (fp32 CUDA-core gate GEMM + cell)"
+    return ("tc_persistent_kernel (tcgen05; launch t = gate GEMM + fused cell of timestep t "
+            "and output head + softmax partials of t - 1)")
 
 
 def gate_flops_per_timestep(c):

@@ -76,7 +76,9 @@ typedef enum soma_status {
   SOMA_ERR_WORKSPACE = 3,   /* workspace NULL or smaller than soma_workspace_bytes() */
   SOMA_ERR_CUDA = 4,        /* a CUDA launch or runtime call failed */
   SOMA_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
-  SOMA_ERR_NONFINITE = 6    /* a loss or coefficient was NaN or infinite */
+  SOMA_ERR_NONFINITE = 6,   /* a loss or coefficient was NaN or infinite */
+  SOMA_ERR_BOUNDS = 7       /* an index check of the checked build failed (never raised
+                               by the default build; see soma_checked_build) */
 } soma_status;
 
 /* Number of parameters P of one expert (layout above); -1 if d is invalid. */
@@ -279,6 +281,26 @@ int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, in
  *   mean/difference form).  Same arguments, limits and errors. */
 int soma_debug_tc_gemm_ts(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
                           void* stream);
+
+/* The checked build.  The library built with -DSOMA_CHECKED
+ * (libsoma_checked.so, `python -m paper_2609_37899_gb300.build --checked`)
+ * guards the shared-memory offsets, tensor-memory columns and global indices
+ * of its kernels with index checks, and surrounds every workspace region with
+ * 256-byte canary words that it writes before a step and verifies after it.
+ * A failed check records SOMA_ERR_BOUNDS in the status word and skips the
+ * access (no trap, the context stays usable).  These are test aids with no
+ * counterpart in the paper; the default build has none of the checks and no
+ * canaries.
+ *  - soma_checked_build: 1 in the checked build, 0 otherwise.
+ *  - soma_debug_check_line: syncs `stream`, returns and clears the position
+ *    of the first failed check (10000 * file id + source line; 90000 + gap
+ *    index for a canary), 0 if none; -1 if the synchronisation failed.
+ *  - soma_debug_check_fail: enqueues one check whose condition is false and
+ *    that guards no access (the checked build's reporting path; a no-op in
+ *    the default build). */
+int soma_checked_build(void);
+int soma_debug_check_line(void* stream);
+int soma_debug_check_fail(void* stream);
 
 /* SPSA step without a workspace argument, for callers that cannot allocate
  * device memory (a host runtime that only passes on buffers it was given, or

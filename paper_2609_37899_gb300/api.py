@@ -23,7 +23,7 @@ _lib = None
 SOMA_OK = 0
 STATUS_NAMES = {0: "SOMA_OK", 1: "SOMA_ERR_INVALID_ARG", 2: "SOMA_ERR_UNSUPPORTED",
                 3: "SOMA_ERR_WORKSPACE", 4: "SOMA_ERR_CUDA", 5: "SOMA_ERR_TIMEOUT",
-                6: "SOMA_ERR_NONFINITE"}
+                6: "SOMA_ERR_NONFINITE", 7: "SOMA_ERR_BOUNDS"}
 
 
 class SomaError(RuntimeError):
@@ -77,7 +77,31 @@ def lib():
         if not os.path.exists(LIB_PATH):
             raise RuntimeError(f"libsoma.so not found at {LIB_PATH}: build it with "
                                "`python -m paper_2609_37899_gb300.build`")
-        L = ctypes.CDLL(LIB_PATH)
+        _lib = _open(LIB_PATH)
+        return _lib
+
+
+def use_library(path: str):
+    """Route every call of this module to the library at `path` (for
+    instance the checked build, libsoma_checked.so) and return the handle in
+    use before, or None; use_library_handle() puts it back."""
+    global _lib
+    with _lock:
+        old = _lib
+        _lib = _open(path)
+        return old
+
+
+def use_library_handle(handle):
+    global _lib
+    with _lock:
+        _lib = handle
+
+
+def _open(path: str):
+    """Load one build of the library and declare the C signatures."""
+    if True:
+        L = ctypes.CDLL(path)
         vp, sz, i32, i64, u64, f32 = (ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int,
                                       ctypes.c_int64, ctypes.c_uint64, ctypes.c_float)
         _sig(L, "soma_param_count", i64, [soma_dims])
@@ -121,7 +145,9 @@ def lib():
                                                ctypes.POINTER(ctypes.c_uint64), i32, vp,
                                                soma_adam_config, vp])
         _sig(L, "soma_debug_body_probe", i32, [u64, u64, i32, i32, bd, i32, i64, i64, vp, vp])
-        _lib = L
+        _sig(L, "soma_checked_build", i32, [])
+        _sig(L, "soma_debug_check_line", i32, [vp])
+        _sig(L, "soma_debug_check_fail", i32, [vp])
         return L
 
 

@@ -1,6 +1,10 @@
 """Compile libsoma.so in-tree for sm_103a (nvcc, one object per .cu in parallel).
 
-    python -m paper_2609_37899_gb300.build
+    python -m paper_2609_37899_gb300.build [--checked]
+
+--checked builds libsoma_checked.so instead: the same sources with
+-DSOMA_CHECKED (index checks in the kernels, canary words around the
+workspace regions; see include/soma_api.h), a test aid.
 """
 from __future__ import annotations
 
@@ -16,6 +20,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJ_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsoma.so")
+CHECKED_OBJ_DIR = os.path.join(PKG, "_build_checked")
+CHECKED_LIB = os.path.join(PKG, "libsoma_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -36,15 +42,18 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
-    os.makedirs(OBJ_DIR, exist_ok=True)
+def build(verbose: bool = False, force: bool = False, extra_flags=(), checked: bool = False) -> str:
+    obj_dir, lib_path = (CHECKED_OBJ_DIR, CHECKED_LIB) if checked else (OBJ_DIR, LIB)
+    if checked:
+        extra_flags = (*extra_flags, "-DSOMA_CHECKED")
+    os.makedirs(obj_dir, exist_ok=True)
     sources = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
     headers = glob.glob(os.path.join(CSRC, "*.cuh")) + glob.glob(os.path.join(CSRC, "*.h")) + \
         glob.glob(os.path.join(INCLUDE, "*.h"))
     jobs = []
     objs = []
     for src in sources:
-        obj = os.path.join(OBJ_DIR, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(obj_dir, os.path.basename(src)[:-3] + ".o")
         objs.append(obj)
         if force or _stale(obj, [src, *headers]):
             jobs.append([nvcc(), *_flags(extra_flags), "-c", src, "-o", obj])
@@ -55,18 +64,18 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
             sys.stderr.write(" ".join(cmd) + "\n" + r.stdout + r.stderr)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {cmd[-3]}")
-    if force or jobs or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if force or jobs or _stale(lib_path, objs):
+        tmp = lib_path + f".tmp{os.getpid()}"
         cuda_lib = os.path.join(os.path.dirname(os.path.dirname(nvcc())), "lib64")
         link = [nvcc(), "-shared", *ARCH, "-cudart", "shared", "-Xlinker", f"-rpath,{cuda_lib}",
                 "-o", tmp, *objs]
         r = subprocess.run(link, capture_output=True, text=True)
         if r.returncode != 0:
             sys.stderr.write(" ".join(link) + "\n" + r.stdout + r.stderr)
-            raise RuntimeError("link of libsoma.so failed")
-        os.replace(tmp, LIB)
-    return LIB
+            raise RuntimeError(f"link of {os.path.basename(lib_path)} failed")
+        os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build(verbose="-v" in sys.argv, force="-f" in sys.argv))
+    print(build(verbose="-v" in sys.argv, force="-f" in sys.argv, checked="--checked" in sys.argv))

@@ -38,6 +38,8 @@
 //  - the tied head likewise, E = E_hi + E_lo (E_lo in shared memory).
 #include <cuda_fp16.h>
 
+#define SOMA_CHECK_FILE 3
+#include "checked.cuh"
 #include "body_device.cuh"
 #include "soma_device.cuh"
 #include "soma_launch.h"
@@ -119,6 +121,7 @@ struct BodyTcArgs {
 // their weights, as two 16-byte chunks.
 __device__ __forceinline__ void chunk8(const float* th, int64_t p0, int kmax, const ProbeKey& pk,
                                        const BodyTcArgs& a, bool do_z, uint4& wout, uint4& zout) {
+  if (!SOMA_CHECK(p0 >= 0 && p0 + kmax <= a.P, a.status)) kmax = 0;  // inside the expert
   uint32_t neg = 0, act = 0;
   if (do_z && kmax > 0) {
     body_probe_words(pk, (int)(p0 >> 5), a.sparse, a.goff, neg, act);
@@ -213,6 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
   const int pair = blockIdx.x;
   const int e = pair / a.n_pert, i = pair % a.n_pert;
   const int chunk = blockIdx.y;
+  // the CTA's sequences, its expert's parameters and its NLL partials lie
+  // inside the caller's buffers (gridDim.x = N n pairs, gridDim.y = chunks)
+  if (!SOMA_CHECK(chunk < a.chunks && chunk * kBp < a.B && pair < (int)gridDim.x, a.status))
+    return;
   const int b0c = chunk * kBp;
   const int rows = min(kBp, a.B - b0c);
   const int D = a.blocks;
@@ -651,7 +658,10 @@ __global__ void __launch_bounds__(kThreads, 1) body_tc_kernel(const BodyTcArgs a
   if (tid < a.n_sign) {
     double tot = 0.0;
     for (int b = 0; b < rows; ++b) tot += acc[tid * kBp + b];
-    a.partial[((int64_t)pair * a.n_sign + tid) * a.chunks + chunk] = tot;
+    if (SOMA_CHECK(((int64_t)pair * a.n_sign + tid) * a.chunks + chunk <
+                       (int64_t)gridDim.x * a.n_sign * a.chunks,
+                   a.status))
+      a.partial[((int64_t)pair * a.n_sign + tid) * a.chunks + chunk] = tot;
   }
   tc_fence_before();
   __syncthreads();

@@ -44,6 +44,8 @@
 // the per-(expert, probe) losses and coefficients.
 #include <cuda_fp16.h>
 
+#define SOMA_CHECK_FILE 1
+#include "checked.cuh"
 #include "soma_api.h"
 #include "soma_device.cuh"
 #include "soma_launch.h"
@@ -277,6 +279,14 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
   for (int st = 0; st < nst; ++st) {
     if (!wait_or_abort(&full[rp.q], rp.ph, abort, status)) return false;
     tc_fence_after();
+    // the accumulator block, the probe tiles of the slot and the operand
+    // windows (rows of 128 bytes per 8-row group step) stay inside their
+    // allocations
+    if (!SOMA_CHECK((d & 0xFFFFu) + dz1 + (NP >= 2 ? dz1 : 0) <= 2 * kAccCols &&
+                        kZCol0 + 64u * rp.q + 32u * (NP > 0 ? NP : 1) <= kTmemCols &&
+                        rp.q < (uint32_t)kStages,
+                    status))
+      return false;
     const uint32_t so = rp.q * slot_step;
     issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.q,
                     idesc_w, idesc_z, dz1, st > 0 ? 1u : 0u);
@@ -297,10 +307,15 @@ struct TcArgs {
   const uint8_t* op_in;  // [N][S][G] operand group tiles: [x_t | h_{t-1}]
   uint8_t* op_out;       // operand of t + 1
   float* cst;            // [N*n][Hp][Bp] cell state (float2: sign +, -)
-  float* pm;             // [N*n*2][B][T][2] head max partials
+  float* pm;             // [N*n*2][B_mem][T][2] head max partials
   float* ps;             // sum-exp partials
-  float* ply;            // [N*n*2][B][T] target logits
+  float* ply;            // [N*n*2][B_mem][T] target logits
   int* status;
+  // extents for the index checks of the checked build (bytes of w16, wo16,
+  // each op buffer and the byte batch; floats of cst, pm / ps, ply, params;
+  // bytes of the dynamic shared memory)
+  size_t n_w16, n_wo16, n_op, n_bytes, n_cst, n_pm, n_ply, n_params;
+  uint32_t smem_bytes;
 };
 
 // One task: (expert, row tile, probe group).  For the gate the row tile is
@@ -387,8 +402,8 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   float bias_r = 0.f, dbias_r = 0.f;
   {
     const int Ur = 32 * T.m + tile_unit(32 * q4 + lane);
-    if (Ur < H) {
-      const int64_t pb = L.b + (int64_t)tile_gate(32 * q4 + lane) * H + Ur;
+    const int64_t pb = L.b + (int64_t)tile_gate(32 * q4 + lane) * H + Ur;
+    if (Ur < H && SOMA_CHECK((size_t)(T.e * L.P + pb) < a.n_params, a.status)) {
       bias_r = th[pb];
       if (eps != 0.f) {
         const ProbeBits zb = probe_bits(pk, pb, s.sparse);
@@ -410,7 +425,9 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   for (int j = 0; j < kEpiMaxChunks; ++j) {
     const int b0 = 8 * (G.c0 + j * G.cstep);
     G.cprev[j][0] = G.cprev[j][1] = make_float2(0.f, 0.f);
-    if (load && b0 < g.Bp) {
+    if (load && b0 < g.Bp &&
+        SOMA_CHECK((size_t)(cell - reinterpret_cast<const float2*>(a.cst) + b0 + 8) * 2 <= a.n_cst,
+                   a.status)) {
       G.cprev[j][0] = cell[b0 + bq];
       G.cprev[j][1] = cell[b0 + 4 + bq];
     }
@@ -448,6 +465,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
     if (b0 >= g.Bp) break;
     // [seq half][gate]: C (W vbar + eps^2 Z dhat) and D (W dhat + Z vbar)
     uint32_t vc[2][4], vd[2][4];
+    if (!SOMA_CHECK(cC + b0 + 8 <= kAccCols && cD + b0 + 8 <= kAccCols, a.status)) break;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const uint32_t cw = (uint32_t)(b0 + 4 * h);
@@ -477,7 +495,12 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
       const float hp = actp[3] * fmaf(sigm(2.f * cp), 2.f, -1.f);
       const float hm = actm[3] * fmaf(sigm(2.f * cm), 2.f, -1.f);
       const int b = b0 + 4 * h + bq;
-      if (unit_ok) {
+      const size_t tile_off = (size_t)(out_tile - a.op_out);
+      if (unit_ok &&
+          SOMA_CHECK((size_t)(cell - reinterpret_cast<float2*>(a.cst) + b + 1) * 2 <= a.n_cst &&
+                         tile_off + g.tileB <= a.n_op && rE + b < g.rowsB && rD + b < g.rowsB &&
+                         rM + b < g.rowsB && kk < kKt,
+                     a.status)) {
         cell[b] = make_float2(cp, cm);
         if (b < s.B) {
           const float dh = hp - hm;
@@ -511,7 +534,10 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
   const bool do_z = eps != 0.f;
   const float* th = s.params + (int64_t)T.e * L.P;
   const int vq = 128 * T.m + 32 * q4;  // first vocabulary row of the quarter
-  const float bo_r = th[L.b_out + vq + lane];
+  const float bo_r =
+      SOMA_CHECK((size_t)(T.e * L.P + L.b_out + vq + lane) < a.n_params, a.status)
+          ? th[L.b_out + vq + lane]
+          : 0.f;
   const int t = a.t_head;
   const int bq = lane & 3, r4 = lane >> 2;
   // rows of this thread: vq + r4 + 8 k, k = 0..3 (k = 2 h + reg)
@@ -569,19 +595,23 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
         sm_ += __shfl_xor_sync(0xffffffffu, sm_, o);
       }
       const int b = b0 + bq;
-      if (r4 == 0) {
+      if (r4 == 0 && SOMA_CHECK(((p * g.Bp + b) * 2 + 1) * 4 + q4 < g.P * g.Bp * 8, a.status)) {
         red[((p * g.Bp + b) * 2 + 0) * 4 + q4] = make_float2(mp, sp);
         red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
       }
-      if (b < s.B) {
+      if (b < s.B &&
+          SOMA_CHECK((size_t)(seq_offset(s, T.e, i, b) + t + 1) < a.n_bytes &&
+                         (size_t)(((lane_plus + 1) * s.B_mem + s.b0 + b) * (int64_t)s.T + t) <
+                             a.n_ply,
+                     a.status)) {
         const int y = s.bytes[seq_offset(s, T.e, i, b) + t + 1] - vq - r4;
         // y = 8 k for the thread that holds the target row
         if (y >= 0 && y < 32 && (y & 7) == 0) {
           const int k = y >> 3;
           const float vp = k == 0 ? lp[0] : k == 1 ? lp[1] : k == 2 ? lp[2] : lp[3];
           const float vm = k == 0 ? lm[0] : k == 1 ? lm[1] : k == 2 ? lm[2] : lm[3];
-          a.ply[((lane_plus + 0) * s.B + b) * (int64_t)s.T + t] = vp;
-          a.ply[((lane_plus + 1) * s.B + b) * (int64_t)s.T + t] = vm;
+          a.ply[((lane_plus + 0) * s.B_mem + s.b0 + b) * (int64_t)s.T + t] = vp;
+          a.ply[((lane_plus + 1) * s.B_mem + s.b0 + b) * (int64_t)s.T + t] = vm;
         }
       }
     }
@@ -602,7 +632,8 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     for (int k = 0; k < 4; ++k) S += q[k].y * __expf(q[k].x - M);
     const int i = T.grp * g.P + pp;
     const int64_t ln = ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
-    const int64_t o = ((ln * s.B + b) * (int64_t)s.T + t) * 2 + T.m;
+    const int64_t o = ((ln * s.B_mem + s.b0 + b) * (int64_t)s.T + t) * 2 + T.m;
+    if (!SOMA_CHECK((size_t)o < a.n_pm, a.status)) continue;
     a.pm[o] = M;
     a.ps[o] = S;
   }
@@ -684,7 +715,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           uint8_t* dst = lane == 0 ? slot + SL.a_off : slot + SL.b_off;
           const uint8_t* src =
               lane == 0 ? T.a + (size_t)st * kTileA : T.b + (size_t)st * g.G * g.tileB;
-          bulk_g2s(dst, src, lane == 0 ? kTileA : g.tileB, &ctl->full[q]);
+          const uint32_t nb = lane == 0 ? kTileA : g.tileB;
+          const uint8_t* gbase = lane == 1 ? a.op_in : (T.head ? a.wo16 : a.w16);
+          const size_t gsize = lane == 1 ? a.n_op : (T.head ? a.n_wo16 : a.n_w16);
+          if (SOMA_CHECK((size_t)(dst - dyn_smem) + nb <= a.smem_bytes &&
+                             src >= gbase && (size_t)(src - gbase) + nb <= gsize,
+                         status))
+            bulk_g2s(dst, src, nb, &ctl->full[q]);
         }
         __syncwarp();
       }
@@ -793,7 +830,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
             break;
           }
           tc_fence_after();
-          if (active) {
+          if (active &&
+              SOMA_CHECK(kZCol0 + 64u * (uint32_t)q + 32u * pz + 32u <= kTmemCols, status)) {
             uint32_t zw[kKt / 2];
 #pragma unroll
             for (int w = 0; w < kKt / 32; ++w) z_run_pairs<SPARSE>(raw[w], act[w], zw + 16 * w);
@@ -862,9 +900,13 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
     const int i = grp * g.P + p;
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
-    if (i < s.n_pert && b < s.B) {
+    if (i < s.n_pert && b < s.B &&
+        SOMA_CHECK((size_t)seq_offset(s, e, i, b) + t < a.n_bytes, a.status)) {
       const int y = s.bytes[seq_offset(s, e, i, b) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
+      if (!SOMA_CHECK(k0 >= g.E || (size_t)(e * L.P + p0 + min(8, g.E - k0)) <= a.n_params,
+                      a.status))
+        continue;
       ProbeBits bits = {0u, 0u};
       if (!mean && s.eps != 0.f)
         bits = probe_bits(make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i), p0, s.sparse);
@@ -880,8 +922,9 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
 #pragma unroll
       for (int j = 0; j < 8; ++j) v[j] = __float2half_rn(0.f);
     }
-    *reinterpret_cast<uint4*>(tile + kmajor_offset(row, 8 * kc, kKt)) =
-        *reinterpret_cast<const uint4*>(v);
+    if (SOMA_CHECK((size_t)(tile - op) + kmajor_offset(row, 8 * kc, kKt) + 16 <= a.n_op, a.status))
+      *reinterpret_cast<uint4*>(tile + kmajor_offset(row, 8 * kc, kKt)) =
+          *reinterpret_cast<const uint4*>(v);
   }
 }
 
@@ -911,10 +954,14 @@ __global__ void prep_tiles_kernel(const TcArgs a) {
       if (U < g.H) {
         if (st < g.Sx) {
           const int k = kKt * st + kk;
-          if (k < g.E) w = th[L.w_ih + R * g.E + k];
+          if (k < g.E && SOMA_CHECK((size_t)(e * L.P + L.w_ih + R * g.E + k) < a.n_params,
+                                    a.status))
+            w = th[L.w_ih + R * g.E + k];
         } else {
           const int k = kKt * (st - g.Sx) + kk;
-          if (k < g.H) w = th[L.w_hh + R * g.H + k];
+          if (k < g.H && SOMA_CHECK((size_t)(e * L.P + L.w_hh + R * g.H + k) < a.n_params,
+                                    a.status))
+            w = th[L.w_hh + R * g.H + k];
         }
       }
       v[kk] = __float2half_rn(w);
@@ -926,10 +973,16 @@ __global__ void prep_tiles_kernel(const TcArgs a) {
     const int vrow = 128 * vh + r;
     for (int kk = 0; kk < kKt; ++kk) {
       const int k = kKt * st + kk;
-      v[kk] = __float2half_rn(k < g.H ? th[L.w_out + (int64_t)vrow * g.H + k] : 0.f);
+      const bool in =
+          k < g.H && SOMA_CHECK((size_t)(e * L.P + L.w_out + (int64_t)vrow * g.H + k) < a.n_params,
+                                a.status);
+      v[kk] = __float2half_rn(in ? th[L.w_out + (int64_t)vrow * g.H + k] : 0.f);
     }
     tile = const_cast<uint8_t*>(a.wo16) + (((size_t)e * 2 + vh) * g.Sh + st) * kTileA;
   }
+  const bool head = tix >= g.MT * g.S;
+  const size_t off = (size_t)(tile - (head ? a.wo16 : a.w16));
+  if (!SOMA_CHECK(off + kTileA <= (head ? a.n_wo16 : a.n_w16), a.status)) return;
 #pragma unroll
   for (int kc = 0; kc < kKt / 8; ++kc)
     *reinterpret_cast<uint4*>(tile + kmajor_offset(r, 8 * kc, kKt)) =
@@ -941,12 +994,13 @@ __global__ void prep_tiles_kernel(const TcArgs a) {
 __global__ void __launch_bounds__(256)
 reduce_tc_kernel(const float* __restrict__ pm, const float* __restrict__ ps,
                  const float* __restrict__ ply, int n_sign, int BT, float eps, float* losses_out,
-                 float* coef_out, float* coef_ws, int* status) {
+                 float* coef_out, float* coef_ws, int* status, size_t n_ply) {
   __shared__ double red[3][256];
   const int pair = blockIdx.x;
   const int64_t lp = (int64_t)pair * 2, lm = lp + 1;
   double sp = 0.0, sm = 0.0, sd = 0.0;
   for (int j = threadIdx.x; j < BT; j += 256) {
+    if (!SOMA_CHECK((size_t)(lm * BT + j) < n_ply, status)) break;
     float nll[2];
     for (int sg = 0; sg < 2; ++sg) {
       const int64_t ln = sg ? lm : lp;
@@ -1090,7 +1144,7 @@ int sm_count() {
 
 }  // namespace
 
-TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T) {
+TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem) {
   TcGeom g;
   g.E = lay.E;
   g.H = lay.H;
@@ -1112,11 +1166,10 @@ TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T) 
   g.n_experts = n_experts;
   g.n_pert = n_pert;
   g.B = B;
+  g.Bm = B_mem;
   g.T = T;
   return g;
 }
-
-bool tc_supported(int B) { return B >= 1 && B <= 64; }
 
 TcSizes tc_sizes(const TcGeom& g) {
   TcSizes z;
@@ -1125,8 +1178,8 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.wo16 = N * 2 * g.Sh * kTileA;
   z.op = N * g.S * g.G * g.tileB;
   z.cst = N * n * 2 * (size_t)g.Hp * g.Bp * sizeof(float);
-  z.pm = N * n * 2 * g.B * (size_t)g.T * 2 * sizeof(float);
-  z.ply = N * n * 2 * g.B * (size_t)g.T * sizeof(float);
+  z.pm = N * n * 2 * g.Bm * (size_t)g.T * 2 * sizeof(float);
+  z.ply = N * n * 2 * g.Bm * (size_t)g.T * sizeof(float);
   return z;
 }
 
@@ -1152,6 +1205,16 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.t_head = -1;
   a.n_gate = 0;
   a.n_head = 0;
+  a.n_w16 = z.w16;
+  a.n_wo16 = z.wo16;
+  a.n_op = z.op;
+  a.n_bytes = (size_t)(s.batch_per_probe ? s.n_experts * s.n_pert : s.n_experts) * s.B_mem *
+              (size_t)(s.T + 1);
+  a.n_cst = z.cst / sizeof(float);
+  a.n_pm = z.pm / sizeof(float);
+  a.n_ply = z.ply / sizeof(float);
+  a.n_params = (size_t)s.n_experts * s.lay.P;
+  a.smem_bytes = (uint32_t)smem;
   a.op_in = tb.op[0];
   a.op_out = tb.op[0];
 
@@ -1190,7 +1253,8 @@ cudaError_t launch_reduce_tc(const TcBuffers& tb, int pairs, int n_sign, int B, 
                              cudaStream_t stream) {
   trace_begin(SOMA_TRACE_REDUCE, stream);
   reduce_tc_kernel<<<pairs, 256, 0, stream>>>(tb.pm, tb.ps, tb.ply, n_sign, B * T, eps,
-                                               losses_out, coef_out, coef_ws, status);
+                                               losses_out, coef_out, coef_ws, status,
+                                               (size_t)pairs * 2 * B * T);
   trace_end(SOMA_TRACE_REDUCE, stream);
   return cudaGetLastError();
 }

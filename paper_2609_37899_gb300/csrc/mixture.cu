@@ -41,18 +41,6 @@ __global__ void token_nll_tc_kernel(const float* __restrict__ pm, const float* _
   nll[((int64_t)e * b_max + b0 + b) * T + t] = v;
 }
 
-// The same for the CUDA-core path's per-target NLL [N][Bc][T].
-__global__ void token_nll_copy_kernel(const float* __restrict__ src, int N, int Bc, int T,
-                                      int b_max, int b0, float* __restrict__ nll) {
-  const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= (int64_t)N * Bc * T) return;
-  const int t = (int)(j % T);
-  const int b = (int)((j / T) % Bc);
-  const int e = (int)(j / ((int64_t)T * Bc));
-  if (b0 + b >= b_max) return;
-  nll[((int64_t)e * b_max + b0 + b) * T + t] = src[j];
-}
-
 // out[r][t - t0] = log k - logsumexp_j(-nll[e_j][slot_j][t]): the NLL of the
 // average of the k routed experts' probabilities of the target.
 __global__ void mixture_kernel(const float* __restrict__ nll, const int32_t* __restrict__ route,
@@ -89,14 +77,6 @@ cudaError_t launch_token_nll_tc(const TcBuffers& tb, int N, int Bc, int T, int b
   const int64_t n = (int64_t)N * Bc * T;
   token_nll_tc_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(tb.pm, tb.ps, tb.ply, N, Bc,
                                                                        T, b_max, b0, nll);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_token_nll_copy(const float* src, int N, int Bc, int T, int b_max, int b0,
-                                  float* nll, cudaStream_t stream) {
-  const int64_t n = (int64_t)N * Bc * T;
-  token_nll_copy_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(src, N, Bc, T, b_max, b0,
-                                                                         nll);
   return cudaGetLastError();
 }
 

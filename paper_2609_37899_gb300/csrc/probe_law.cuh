@@ -29,4 +29,17 @@ __host__ __device__ __forceinline__ void probe_law_words(const ProbeKey& pk, int
   }
 }
 
+// The activity word of run q under the probe law, from its raw activity
+// word (sparse probes only): coordinates from dense_from on stay active.
+__host__ __device__ __forceinline__ uint32_t probe_law_act(uint32_t act_raw, int64_t q,
+                                                           int64_t dense_from) {
+  uint32_t act = raw_to_natural(act_raw);
+  const int64_t from = dense_from - 32LL * q;  // first dense coordinate inside the run
+  if (from <= 0)
+    act = 0xFFFFFFFFu;
+  else if (from < 32)
+    act |= 0xFFFFFFFFu << from;
+  return act;
+}
+
 }  // namespace soma

@@ -26,6 +26,8 @@
 // by res_supported(); other experts use the persistent kernel.
 #include <cuda_fp16.h>
 
+#define SOMA_CHECK_FILE 2
+#include "checked.cuh"
 #include "soma_api.h"
 #include "soma_device.cuh"
 #include "soma_launch.h"
@@ -98,6 +100,7 @@ struct ResArgs {
   float* coef_out;    // [N][n] or null
   float* coef_ws;     // [N][n] or null
   int* status;
+  size_t n_params, n_bytes;  // extents for the index checks of the checked build
 };
 
 // z of flat parameter p as an fp16 +-1 / 0 (sparse) value.
@@ -158,6 +161,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
     }
     ProbeBits zb = {0u, 0u};
     if (kmax > 0 && do_z) zb = probe_bits(pk, p0, s.sparse);
+    if (kmax > 0 && !SOMA_CHECK((size_t)(e * L.P + p0 + kmax) <= a.n_params, a.status)) kmax = 0;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const bool ok = j < kmax;
@@ -165,15 +169,18 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       z[j] = ok ? z_half(zb, j) : __float2half_rn(0.f);
     }
     const uint32_t off = m * (128u * g.K * 2) + kmajor_offset(r, k0, g.K);
-    *reinterpret_cast<uint4*>(smem + g.wg + off) = *reinterpret_cast<const uint4*>(w);
-    *reinterpret_cast<uint4*>(smem + g.zg + off) = *reinterpret_cast<const uint4*>(z);
+    if (SOMA_CHECK(off + 16 <= g.MTg * 128u * g.K * 2 && g.zg + off + 16 <= g.bytes, a.status)) {
+      *reinterpret_cast<uint4*>(smem + g.wg + off) = *reinterpret_cast<const uint4*>(w);
+      *reinterpret_cast<uint4*>(smem + g.zg + off) = *reinterpret_cast<const uint4*>(z);
+    }
   }
   const int head_chunks = 2 * 128 * (g.Hk / 8);
   for (int c = tid; c < head_chunks; c += kResThreads) {
     const int h = c / (128 * (g.Hk / 8)), rem = c % (128 * (g.Hk / 8));
     const int r = rem / (g.Hk / 8), k0 = 8 * (rem % (g.Hk / 8));
     const int64_t p0 = L.w_out + (int64_t)(128 * h + r) * g.H + k0;
-    const int kmax = min(8, g.H - k0);
+    int kmax = min(8, g.H - k0);
+    if (kmax > 0 && !SOMA_CHECK((size_t)(e * L.P + p0 + kmax) <= a.n_params, a.status)) kmax = 0;
     ProbeBits zb = {0u, 0u};
     if (kmax > 0 && do_z) zb = probe_bits(pk, p0, s.sparse);
     __align__(16) __half w[8], z[8];
@@ -184,8 +191,10 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       z[j] = ok ? z_half(zb, j) : __float2half_rn(0.f);
     }
     const uint32_t off = h * (128u * g.Hk * 2) + kmajor_offset(r, k0, g.Hk);
-    *reinterpret_cast<uint4*>(smem + g.wo + off) = *reinterpret_cast<const uint4*>(w);
-    *reinterpret_cast<uint4*>(smem + g.zo + off) = *reinterpret_cast<const uint4*>(z);
+    if (SOMA_CHECK(off + 16 <= 2u * 128u * g.Hk * 2 && g.zo + off + 16 <= g.bytes, a.status)) {
+      *reinterpret_cast<uint4*>(smem + g.wo + off) = *reinterpret_cast<const uint4*>(w);
+      *reinterpret_cast<uint4*>(smem + g.zo + off) = *reinterpret_cast<const uint4*>(z);
+    }
   }
   for (int c = tid; c < 2 * (2 * g.Bp * g.K / 8); c += kResThreads)
     reinterpret_cast<uint4*>(smem + g.op)[c] = make_uint4(0u, 0u, 0u, 0u);
@@ -298,7 +307,10 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
       if (lane == 0) {
         tc_fence_after();
         const uint32_t ob = op_lo + cur * (g.opsz >> 4);  // operand buffer t % 2
-        if (t < g.T) {  // gate of t: [x_t | h_{t-1}]
+        if (!SOMA_CHECK(hcol0 + 8u * g.Bp <= g.tmem_cols && gcol0 + g.MTg * 4u * g.Bp <= hcol0,
+                        a.status)) {
+          // columns outside the allocation: no MMA; the epilogue waits time out
+        } else if (t < g.T) {  // gate of t: [x_t | h_{t-1}]
 #pragma unroll 1
           for (int m = 0; m < g.MTg; ++m) {
             const uint32_t d = tmem + gcol0 + (uint32_t)m * 2 * n2;
@@ -377,7 +389,8 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
             const float hp = actp[3] * fmaf(sigm_res(2.f * cp), 2.f, -1.f);
             const float hm = actm[3] * fmaf(sigm_res(2.f * cm), 2.f, -1.f);
             const int b = b0 + 4 * h + bq;
-            if (unit_ok && b < g.B) {
+            if (unit_ok && b < g.B &&
+                SOMA_CHECK(kmajor_offset(g.Bp + b, g.Ek + U, g.K) + 2 <= g.opsz, a.status)) {
               *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(b, g.Ek + U, g.K)) =
                   __float2half_rn(0.5f * (hp + hm));
               *reinterpret_cast<__half*>(smem + g.op + nxt * g.opsz + kmajor_offset(g.Bp + b, g.Ek + U, g.K)) =
@@ -453,7 +466,7 @@ __global__ void __launch_bounds__(kResThreads, 1) res_kernel(const ResArgs a) {
           red[((half * 4 + q4) * 2 + 0) * g.Bp + b] = make_float2(mp, sp);
           red[((half * 4 + q4) * 2 + 1) * g.Bp + b] = make_float2(mm, sm_);
         }
-        if (b < g.B) {
+        if (b < g.B && SOMA_CHECK((size_t)seq_offset(s, e, i, b) + t < a.n_bytes, a.status)) {
           const int y = s.bytes[seq_offset(s, e, i, b) + t] - vq - r4;  // target of t - 1
           if (y >= 0 && y < 32 && (y & 7) == 0) {
             const int k = y >> 3;
@@ -535,6 +548,9 @@ cudaError_t launch_forward_res(const Sweep& s, int n_sign, float* losses_out, fl
   a.coef_out = coef_out;
   a.coef_ws = coef_ws;
   a.status = status;
+  a.n_params = (size_t)s.n_experts * s.lay.P;
+  a.n_bytes = (size_t)(s.batch_per_probe ? s.n_experts * s.n_pert : s.n_experts) * s.B_mem *
+              (size_t)(s.T + 1);
   cudaError_t e = cudaFuncSetAttribute(res_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)a.g.bytes);
   if (e != cudaSuccess) return e;

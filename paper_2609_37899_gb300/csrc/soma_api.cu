@@ -7,15 +7,19 @@
 #include <cstring>
 #include <vector>
 
+#define SOMA_CHECK_FILE 7
+#include "checked.cuh"
 #include "soma_api.h"
 #include "body_device.cuh"
 #include "soma_launch.h"
 
 using namespace soma;
 
-// Per-device status word (see soma_get_status).  Kernels get its address as
-// an argument; it is read and cleared only by soma_get_status.
-__device__ int g_soma_status = 0;
+// Per-device status word (see soma_get_status) and, after it, the position of
+// the first failed index check of the checked build (soma_debug_check_line).
+// Kernels get the address of the pair as their status argument; only
+// soma_get_status and soma_debug_check_line read and clear it.
+__device__ int g_soma_status[2] = {0, 0};
 
 namespace {
 
@@ -44,88 +48,161 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 constexpr size_t kAlign = 256;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Workspace of one sweep with `n_pert` probes and `n_sign` signs.  Batches of
-// up to 64 sequences run on the tensor cores (both signs always); larger
-// batches on the fp32 CUDA-core kernels.
-struct WsPlan {
-  bool res;  // the resident small-expert kernel: no scratch but the coefficients
-  bool tc;
-  TcGeom g;
-  TcSizes z;
-  int Tc;
-  size_t hist, cst, nll, coef, total;
+// Workspace layout: regions in order, each rounded up to 256 bytes.  The
+// checked build puts a 256-byte canary gap before every region and after
+// the last; the gaps are filled before a step and checked after it.
+#ifdef SOMA_CHECKED
+constexpr size_t kGuard = 256;
+#else
+constexpr size_t kGuard = 0;
+#endif
+constexpr int kMaxRegions = 12;
+constexpr uint32_t kCanaryWord = 0x5A17C0DEu;
+
+struct Regions {
+  int n;
+  size_t off[kMaxRegions];
+  size_t end;
+  size_t add(size_t bytes) {
+    off[n] = end + kGuard;
+    end = off[n] + round_up(bytes);
+    return off[n++];
+  }
+  size_t total() const { return end + kGuard; }
 };
+
+#ifdef SOMA_CHECKED
+// The canary gaps of a workspace: before each region and after the last.
+struct Gaps {
+  int n;
+  size_t off[kMaxRegions + 1];
+};
+
+Gaps gaps_of(const Regions& r) {
+  Gaps g;
+  g.n = r.n + 1;
+  for (int i = 0; i < r.n; ++i) g.off[i] = r.off[i] - kGuard;
+  g.off[r.n] = r.end;
+  return g;
+}
+
+__global__ void canary_fill_kernel(uint32_t* ws, Gaps g) {
+  for (int j = threadIdx.x; j < g.n * (int)(kGuard / 4); j += blockDim.x) {
+    const int k = j / (int)(kGuard / 4), w = j % (int)(kGuard / 4);
+    ws[g.off[k] / 4 + w] = kCanaryWord;
+  }
+}
+
+// A canary word that changed means a kernel wrote outside its region:
+// SOMA_ERR_BOUNDS, position 90000 + the gap index.
+__global__ void canary_check_kernel(const uint32_t* ws, Gaps g, int* status) {
+  for (int j = threadIdx.x; j < g.n * (int)(kGuard / 4); j += blockDim.x) {
+    const int k = j / (int)(kGuard / 4), w = j % (int)(kGuard / 4);
+    if (ws[g.off[k] / 4 + w] != kCanaryWord) {
+      atomicCAS(status, 0, kStatusBounds);
+      atomicCAS(status + 1, 0, 90000 + k);
+    }
+  }
+}
+#endif
+
+cudaError_t canary_fill(const Regions& r, void* ws, cudaStream_t st) {
+#ifdef SOMA_CHECKED
+  canary_fill_kernel<<<1, 256, 0, st>>>(static_cast<uint32_t*>(ws), gaps_of(r));
+  return cudaGetLastError();
+#else
+  (void)r, (void)ws, (void)st;
+  return cudaSuccess;
+#endif
+}
+
+cudaError_t canary_check(const Regions& r, const void* ws, int* status, cudaStream_t st) {
+#ifdef SOMA_CHECKED
+  canary_check_kernel<<<1, 256, 0, st>>>(static_cast<const uint32_t*>(ws), gaps_of(r), status);
+  return cudaGetLastError();
+#else
+  (void)r, (void)ws, (void)status, (void)st;
+  return cudaSuccess;
+#endif
+}
+
+// Workspace of one sweep with `n_pert` probes and `n_sign` signs.  Small
+// experts run on the resident kernel (only the coefficients need scratch);
+// every other batch runs on the persistent tensor-core kernel (both signs
+// always), in chunks of at most kTcMaxBatch sequences that share the
+// operand and cell buffers and write their loss partials into buffers of
+// the whole batch.
+struct WsPlan {
+  bool res;    // the resident small-expert kernel: no scratch but the coefficients
+  TcGeom g;    // geometry of the largest chunk
+  TcSizes z;   // buffer sizes: the largest chunk's operand and cell buffers
+  Regions r;   // w16, wo16, op[0], op[1], cst, pm, ps, ply, coef; or coef alone
+  size_t total;
+};
+
+int chunk_size(int B, int b0) { return B - b0 < kTcMaxBatch ? B - b0 : kTcMaxBatch; }
 
 WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T,
                   bool allow_res = true) {
+  (void)n_sign;
   WsPlan w;
   std::memset(&w, 0, sizeof(w));
   const Layout lay = make_layout(d.embed, d.hidden);
-  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
+  const size_t coef = (size_t)n_experts * n_pert * sizeof(float);
   if (allow_res && res_supported(lay, B)) {
     w.res = true;
-    w.total = w.coef;
+    w.r.add(coef);
+    w.total = w.r.total();
     return w;
   }
-  if (tc_supported(B)) {
-    w.tc = true;
-    w.g = make_tc_geom(lay, n_experts, n_pert, B, T);
-    w.z = tc_sizes(w.g);
-    w.total = round_up(w.z.w16) + round_up(w.z.wo16) + 2 * round_up(w.z.op) + round_up(w.z.cst) +
-              2 * round_up(w.z.pm) + round_up(w.z.ply) + w.coef;
-    return w;
-  }
-  Sweep s;
-  std::memset(&s, 0, sizeof(s));
-  s.lay = lay;
-  s.n_experts = n_experts;
-  s.n_pert = n_pert;
-  s.n_sign = n_sign;
-  s.B = B;
-  s.T = T;
-  w.Tc = forward_hist_slots(s);
-  const size_t lanes = (size_t)s.lanes();
-  w.hist = round_up(lanes * w.Tc * B * (size_t)d.hidden * sizeof(float));
-  w.cst = round_up(lanes * B * (size_t)d.hidden * sizeof(float));
-  w.nll = round_up(lanes * B * (size_t)T * sizeof(float));
-  w.total = w.hist + w.cst + w.nll + w.coef;
+  // the operand and cell buffers of every chunk fit those of the first one
+  // or of the last (smaller Bp packs two probes per group)
+  w.g = make_tc_geom(lay, n_experts, n_pert, chunk_size(B, 0), T, B);
+  w.z = tc_sizes(w.g);
+  const int last = chunk_size(B, (B - 1) / kTcMaxBatch * kTcMaxBatch);
+  const TcSizes zl = tc_sizes(make_tc_geom(lay, n_experts, n_pert, last, T, B));
+  if (zl.op > w.z.op) w.z.op = zl.op;
+  if (zl.cst > w.z.cst) w.z.cst = zl.cst;
+  for (size_t bytes : {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, coef})
+    w.r.add(bytes);
+  w.total = w.r.total();
   return w;
-}
-
-ForwardBuffers carve(const WsPlan& w, void* ws) {
-  char* base = static_cast<char*>(ws);
-  ForwardBuffers fb;
-  fb.Tc = w.Tc;
-  fb.hist = reinterpret_cast<float*>(base);
-  fb.cst = reinterpret_cast<float*>(base + w.hist);
-  fb.nll = reinterpret_cast<float*>(base + w.hist + w.cst);
-  return fb;
 }
 
 TcBuffers carve_tc(const WsPlan& w, void* ws) {
   uint8_t* p = static_cast<uint8_t*>(ws);
   TcBuffers tb;
-  tb.w16 = p;
-  p += round_up(w.z.w16);
-  tb.wo16 = p;
-  p += round_up(w.z.wo16);
-  tb.op[0] = p;
-  p += round_up(w.z.op);
-  tb.op[1] = p;
-  p += round_up(w.z.op);
-  tb.cst = reinterpret_cast<float*>(p);
-  p += round_up(w.z.cst);
-  tb.pm = reinterpret_cast<float*>(p);
-  p += round_up(w.z.pm);
-  tb.ps = reinterpret_cast<float*>(p);
-  p += round_up(w.z.pm);
-  tb.ply = reinterpret_cast<float*>(p);
+  tb.w16 = p + w.r.off[0];
+  tb.wo16 = p + w.r.off[1];
+  tb.op[0] = p + w.r.off[2];
+  tb.op[1] = p + w.r.off[3];
+  tb.cst = reinterpret_cast<float*>(p + w.r.off[4]);
+  tb.pm = reinterpret_cast<float*>(p + w.r.off[5]);
+  tb.ps = reinterpret_cast<float*>(p + w.r.off[6]);
+  tb.ply = reinterpret_cast<float*>(p + w.r.off[7]);
   return tb;
+}
+
+// The tensor-core forward of a whole batch: one sweep per chunk of at most
+// kTcMaxBatch sequences (each with its own geometry), all writing the loss
+// partials of the batch.
+cudaError_t forward_tc_chunks(Sweep s, const Layout& lay, const TcBuffers& tb, int* status,
+                              cudaStream_t st) {
+  const int B = s.B;
+  s.B_mem = B;
+  cudaError_t e = cudaSuccess;
+  for (int b0 = 0; b0 < B && e == cudaSuccess; b0 += kTcMaxBatch) {
+    s.b0 = b0;
+    s.B = chunk_size(B, b0);
+    const TcGeom g = make_tc_geom(lay, s.n_experts, s.n_pert, s.B, s.T, B);
+    e = launch_forward_tc(s, g, tb, status, st);
+  }
+  return e;
 }
 
 // the coefficient scratch is the last region of both layouts
 float* coef_scratch(const WsPlan& w, void* ws) {
-  return reinterpret_cast<float*>(static_cast<char*>(ws) + (w.total - w.coef));
+  return reinterpret_cast<float*>(static_cast<char*>(ws) + w.r.off[w.r.n - 1]);
 }
 
 bool sizes_ok(int n_experts, int n_pert, int batch, int seq_len) {
@@ -191,33 +268,31 @@ static int spsa_forward(float* params, int n_experts, soma_dims d, int n_pert, i
   s.n_sign = 2;
   s.B = batch;
   s.T = seq_len;
+  s.b0 = 0;
+  s.B_mem = batch;
   s.eps = eps;
   s.sparse = sparse;
   s.batch_per_probe = batch_per_probe;
   s.seed = seed;
   s.step = step;
   float* coef_ws = coef_scratch(w, workspace);
-  cudaError_t e;
-  if (w.res) {
+  cudaError_t e = canary_fill(w.r, workspace, st);
+  if (e != cudaSuccess) {
+  } else if (w.res) {
     e = launch_forward_res(s, 2, losses_out, coef_out, coef_ws, status, st);
-  } else if (w.tc) {
+  } else {
     const TcBuffers tb = carve_tc(w, workspace);
-    e = launch_forward_tc(s, w.g, tb, status, st);
+    e = forward_tc_chunks(s, s.lay, tb, status, st);
     if (e == cudaSuccess)
       e = launch_reduce_tc(tb, n_experts * n_pert, 2, batch, seq_len, eps, losses_out, coef_out,
                            coef_ws, status, st);
-  } else {
-    const ForwardBuffers fb = carve(w, workspace);
-    e = launch_forward_simt(s, fb, st);
-    if (e == cudaSuccess)
-      e = launch_reduce_losses(fb.nll, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
-                               coef_out, coef_ws, status, st);
   }
   if (summed_loss && e == cudaSuccess) e = launch_sum_over_experts(coef_out, n_experts, n_pert, st);
   // eps == 0 makes every coefficient 0 and lr == 0 every step 0: theta stays
   // bit-identical, so the update is not launched at all.
   if (update && e == cudaSuccess && eps != 0.f && lr != 0.f)
     e = launch_spsa_update(params, s.lay, n_experts, n_pert, lr, seed, step, coef_ws, st);
+  if (e == cudaSuccess) e = canary_check(w.r, workspace, status, st);
   return cuda_status(e);
 }
 
@@ -307,27 +382,25 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
   s.n_sign = 1;
   s.B = batch;
   s.T = seq_len;
+  s.b0 = 0;
+  s.B_mem = batch;
   s.eps = 0.f;
   s.sparse = 0;
   s.batch_per_probe = 0;
   s.seed = 0;
   s.step = 0;
-  cudaError_t e;
-  if (w.res) {
+  cudaError_t e = canary_fill(w.r, workspace, st);
+  if (e != cudaSuccess) {
+  } else if (w.res) {
     e = launch_forward_res(s, 1, loss_out, nullptr, nullptr, status, st);
-  } else if (w.tc) {
+  } else {
     const TcBuffers tb = carve_tc(w, workspace);
-    e = launch_forward_tc(s, w.g, tb, status, st);
+    e = forward_tc_chunks(s, s.lay, tb, status, st);
     if (e == cudaSuccess)
       e = launch_reduce_tc(tb, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr, nullptr,
                            status, st);
-  } else {
-    const ForwardBuffers fb = carve(w, workspace);
-    e = launch_forward_simt(s, fb, st);
-    if (e == cudaSuccess)
-      e = launch_reduce_losses(fb.nll, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
-                               nullptr, status, st);
   }
+  if (e == cudaSuccess) e = canary_check(w.r, workspace, status, st);
   return cuda_status(e);
 }
 
@@ -341,6 +414,25 @@ int soma_spsa_update(float* params, int n_experts, soma_dims d, int n_pert, floa
   const Layout lay = make_layout(d.embed, d.hidden);
   return cuda_status(
       launch_spsa_update(params, lay, n_experts, n_pert, lr, seed, step, coef, (cudaStream_t)stream));
+}
+
+int soma_checked_build(void) {
+#ifdef SOMA_CHECKED
+  return 1;
+#else
+  return 0;
+#endif
+}
+
+int soma_debug_check_line(void* stream) {
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return -1;
+  int* p = status_ptr();
+  if (!p) return -1;
+  int v = 0;
+  if (cudaMemcpy(&v, p + 1, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+  const int zero = 0;
+  if (cudaMemcpy(p + 1, &zero, sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess) return -1;
+  return v;
 }
 
 int soma_get_status(void* stream) {
@@ -364,6 +456,7 @@ const char* soma_status_string(int code) {
     case SOMA_ERR_CUDA: return "CUDA error";
     case SOMA_ERR_TIMEOUT: return "device-side wait timed out";
     case SOMA_ERR_NONFINITE: return "non-finite loss or coefficient";
+    case SOMA_ERR_BOUNDS: return "an index check of the checked build failed";
     default: return "unknown status";
   }
 }
@@ -393,6 +486,12 @@ int soma_debug_tc_gemm(const uint16_t* a, const uint16_t* b, float* d, int n, in
 int soma_debug_tc_gemm_ts(const uint16_t* a, const uint16_t* b, float* d, int n, int k,
                           void* stream) {
   return debug_tc_gemm(a, b, d, n, k, 1, stream);
+}
+
+int soma_debug_check_fail(void* stream) {
+  int* status = status_ptr();
+  if (!status) return SOMA_ERR_CUDA;
+  return cuda_status(launch_debug_check_fail(status, (cudaStream_t)stream));
 }
 
 int soma_debug_wait_timeout(uint32_t max_polls, void* stream) {
@@ -428,7 +527,7 @@ int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int pro
 namespace {
 
 constexpr int kMaxRoutes = 16;
-constexpr int kMixChunk = 64;  // sequences per expert and sweep (the tensor path's limit)
+constexpr int kMixChunk = kTcMaxBatch;  // sequences per expert and sweep
 
 struct MixPlan {
   int b_max, Bc, chunks;
@@ -457,7 +556,7 @@ bool plan_mixture(const soma_dims& d, int N, const int32_t* routes, int R, int k
       m.gather_h[(size_t)routes[(size_t)r * k + j] * m.b_max + m.slot_h[(size_t)r * k + j]] = r;
   m.Bc = m.b_max < kMixChunk ? m.b_max : kMixChunk;
   m.chunks = (m.b_max + m.Bc - 1) / m.Bc;
-  // the mixture reads per-target NLL, which only the per-timestep kernels keep
+  // the mixture reads per-target NLL, which the persistent kernel keeps
   m.sweep = plan_sweep(d, N, 1, 1, m.Bc, T, false);
   m.gather = round_up((size_t)N * m.b_max * sizeof(int32_t));
   m.route = round_up((size_t)R * k * sizeof(int32_t));
@@ -523,6 +622,8 @@ int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint
   s.n_sign = 1;
   s.B = m.Bc;
   s.T = seq_len;
+  s.b0 = 0;
+  s.B_mem = m.Bc;
   s.eps = 0.f;
   s.sparse = 0;
   s.batch_per_probe = 0;
@@ -533,17 +634,10 @@ int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint
     e = launch_gather_requests(requests, gather, n_experts, m.b_max, b0, m.Bc, seq_len + 1,
                                grouped, st);
     if (e != cudaSuccess) break;
-    if (m.sweep.tc) {
-      const TcBuffers tb = carve_tc(m.sweep, sweep_ws);
-      e = launch_forward_tc(s, m.sweep.g, tb, status, st);
-      if (e == cudaSuccess)
-        e = launch_token_nll_tc(tb, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
-    } else {
-      const ForwardBuffers fb = carve(m.sweep, sweep_ws);
-      e = launch_forward_simt(s, fb, st);
-      if (e == cudaSuccess)
-        e = launch_token_nll_copy(fb.nll, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
-    }
+    const TcBuffers tb = carve_tc(m.sweep, sweep_ws);
+    e = launch_forward_tc(s, m.sweep.g, tb, status, st);
+    if (e == cudaSuccess)
+      e = launch_token_nll_tc(tb, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
   }
   if (e == cudaSuccess)
     e = launch_mixture(nll, route, slot, R, k, seq_len, t0, m.b_max, nll_out, st);
@@ -561,15 +655,17 @@ bool body_dims_ok(const soma_body_dims& d) {
 
 // fp64 NLL sums [N * n * n_sign][chunks], then the coefficients [N][n].
 struct BodyWs {
-  size_t partial, coef, total;
+  Regions r;  // partial, coef
+  size_t total;
 };
 
 BodyWs plan_body(int n_experts, int n_pert, int n_sign, int B) {
   BodyWs w;
+  std::memset(&w, 0, sizeof(w));
   const int chunks = (B + body_rows_per_cta() - 1) / body_rows_per_cta();
-  w.partial = round_up((size_t)n_experts * n_pert * n_sign * chunks * sizeof(double));
-  w.coef = round_up((size_t)n_experts * n_pert * sizeof(float));
-  w.total = w.partial + w.coef;
+  w.r.add((size_t)n_experts * n_pert * n_sign * chunks * sizeof(double));
+  w.r.add((size_t)n_experts * n_pert * sizeof(float));
+  w.total = w.r.total();
   return w;
 }
 
@@ -594,10 +690,12 @@ int body_forward(float* params, int n_experts, soma_body_dims d, const float* he
   int* status = status_ptr();
   if (!status) return SOMA_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)stream;
-  double* partial = static_cast<double*>(workspace);
-  float* coef_ws = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + w.partial);
-  cudaError_t e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, n_pert, 2, batch,
-                                 seq_len, eps, probe_kind, seed, step, partial, status, st);
+  double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(workspace) + w.r.off[0]);
+  float* coef_ws = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + w.r.off[1]);
+  cudaError_t e = canary_fill(w.r, workspace, st);
+  if (e == cudaSuccess)
+    e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, n_pert, 2, batch, seq_len,
+                       eps, probe_kind, seed, step, partial, status, st);
   if (e == cudaSuccess)
     e = launch_body_reduce(partial, n_experts * n_pert, 2, batch, seq_len, eps, losses_out,
                            coef_out, coef_ws, status, st);
@@ -605,6 +703,7 @@ int body_forward(float* params, int n_experts, soma_body_dims d, const float* he
   if (update && e == cudaSuccess && eps != 0.f && lr != 0.f)
     e = launch_body_sgd(params, n_experts, d.blocks, n_pert, probe_kind, lr, seed, step, coef_ws,
                         st);
+  if (e == cudaSuccess) e = canary_check(w.r, workspace, status, st);
   return cuda_status(e);
 }
 
@@ -656,12 +755,15 @@ int soma_body_eval_loss(const float* params, int n_experts, soma_body_dims d, co
   int* status = status_ptr();
   if (!status) return SOMA_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)stream;
-  double* partial = static_cast<double*>(workspace);
-  cudaError_t e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, 1, 1, batch,
-                                 seq_len, 0.f, 0, 0, 0, partial, status, st);
+  double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(workspace) + w.r.off[0]);
+  cudaError_t e = canary_fill(w.r, workspace, st);
+  if (e == cudaSuccess)
+    e = launch_body_tc(params, head, byte_batch, n_experts, d.blocks, 1, 1, batch, seq_len, 0.f,
+                       0, 0, 0, partial, status, st);
   if (e == cudaSuccess)
     e = launch_body_reduce(partial, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr,
                            nullptr, status, st);
+  if (e == cudaSuccess) e = canary_check(w.r, workspace, status, st);
   return cuda_status(e);
 }
 

@@ -178,16 +178,19 @@ struct Sweep {
   int B, T;
   float eps;
   int sparse;              // probe kind: 0 dense Rademacher, 1 sparse (App. E)
-  int batch_per_probe;     // 0: bytes [N][B][T+1] shared by every probe (Sec. 4);
-                           // 1: bytes [N][n_pert][B][T+1], one batch per probe (App. D)
+  int batch_per_probe;     // 0: bytes [N][B_mem][T+1] shared by every probe (Sec. 4);
+                           // 1: bytes [N][n_pert][B_mem][T+1], one batch per probe (App. D)
+  int b0, B_mem;           // the sweep covers sequences b0 .. b0 + B - 1 of each batch of
+                           // B_mem sequences (a batch of more than 64 runs in chunks)
   uint64_t seed, step;
   __host__ __device__ int lanes() const { return n_experts * n_pert * n_sign; }
 };
 
-// Offset of the first byte of sequence b seen by probe i of expert e.
+// Offset of the first byte of sequence b (of the sweep) seen by probe i of
+// expert e.
 __host__ __device__ __forceinline__ int64_t seq_offset(const Sweep& s, int e, int i, int b) {
   const int64_t blk = s.batch_per_probe ? (int64_t)e * s.n_pert + i : (int64_t)e;
-  return (blk * s.B + b) * (int64_t)(s.T + 1);
+  return (blk * s.B_mem + s.b0 + b) * (int64_t)(s.T + 1);
 }
 
 __host__ __device__ __forceinline__ void lane_parts(const Sweep& s, int lane, int& e, int& i,

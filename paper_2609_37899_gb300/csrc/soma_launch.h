@@ -11,20 +11,10 @@
 
 namespace soma {
 
-// Scratch of one forward sweep, carved out of the caller's workspace.
-struct ForwardBuffers {
-  int Tc;        // ring length of the h_t history
-  float* hist;   // [lanes][Tc][B][H]
-  float* cst;    // [lanes][B][H]
-  float* nll;    // [lanes][B][T] per-target NLL
-};
-
 // Tracing hooks: bracket one kernel launch of class `kind` (SOMA_TRACE_*).
 void trace_begin(int kind, cudaStream_t stream);
 void trace_end(int kind, cudaStream_t stream);
 
-int forward_hist_slots(const Sweep& s);
-cudaError_t launch_forward_simt(const Sweep& s, const ForwardBuffers& fb, cudaStream_t stream);
 
 // ---- tensor-core path ------------------------------------------------------
 // Geometry of one sweep on the tensor cores.  K of the gate GEMM is
@@ -36,6 +26,7 @@ struct TcGeom {
   int E, H, Ep, Hp, S, Sx, Sh, MT, Bp, P, G, rowsB;
   uint32_t tileB;  // bytes of one operand group tile of one stage
   int n_experts, n_pert, B, T;
+  int Bm;          // sequences of the whole batch (the loss partials); B <= 64 of them per sweep
 };
 
 struct TcSizes {
@@ -52,8 +43,9 @@ struct TcBuffers {
   float* ply;      // target logits
 };
 
-TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T);
-bool tc_supported(int B);
+TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem);
+// Sequences of one tensor-core sweep; a larger batch runs in chunks of this many.
+constexpr int kTcMaxBatch = 64;
 TcSizes tc_sizes(const TcGeom& g);
 cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
                               cudaStream_t stream);
@@ -63,10 +55,6 @@ cudaError_t launch_reduce_tc(const TcBuffers& tb, int pairs, int n_sign, int B, 
 cudaError_t launch_debug_tc_gemm(const void* A, const void* B, float* D, int N, int K,
                                  int a_in_tmem, int* status, cudaStream_t stream);
 
-// losses_out [pairs][n_sign]; coef_out / coef_ws [pairs] (either may be null).
-cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B, int T, float eps,
-                                 float* losses_out, float* coef_out, float* coef_ws, int* status,
-                                 cudaStream_t stream);
 cudaError_t launch_spsa_update(float* params, const Layout& lay, int n_experts, int n_pert,
                                float lr, uint64_t seed, uint64_t step, const float* coef,
                                cudaStream_t stream);
@@ -78,6 +66,7 @@ cudaError_t launch_sgd_update(float* params, int64_t P, int64_t dense_from, int 
 cudaError_t launch_init(float* params, const Layout& lay, int n_experts, uint64_t seed, float std,
                         cudaStream_t stream);
 cudaError_t launch_debug_wait_timeout(uint32_t max_polls, int* status, cudaStream_t stream);
+cudaError_t launch_debug_check_fail(int* status, cudaStream_t stream);
 cudaError_t launch_debug_philox(uint64_t seed, const uint32_t* ctr4, uint32_t* out4, int count,
                                 cudaStream_t stream);
 cudaError_t launch_debug_rademacher(uint64_t seed, uint64_t step, int expert, int pert, int sparse,
@@ -108,8 +97,6 @@ cudaError_t launch_gather_requests(const uint8_t* requests, const int32_t* gathe
                                    cudaStream_t stream);
 cudaError_t launch_token_nll_tc(const TcBuffers& tb, int N, int Bc, int T, int b_max, int b0,
                                 float* nll, cudaStream_t stream);
-cudaError_t launch_token_nll_copy(const float* src, int N, int Bc, int T, int b_max, int b0,
-                                  float* nll, cudaStream_t stream);
 cudaError_t launch_mixture(const float* nll, const int32_t* route, const int32_t* slot, int R,
                            int k, int T, int t0, int b_max, float* out, cudaStream_t stream);
 cudaError_t launch_sum_over_experts(float* coef, int n_experts, int n_pert, cudaStream_t stream);

@@ -1,5 +1,7 @@
-// spsa_misc.cu -- the loss reduction, the SPSA update, the parameter
-// initialisation and the generator test kernels.
+// spsa_misc.cu -- the SPSA and Adam updates, the summed-loss arm, the
+// parameter initialisation and the generator test kernels.
+#define SOMA_CHECK_FILE 4
+#include "checked.cuh"
 #include "soma_api.h"
 #include "probe_law.cuh"
 #include "soma_launch.h"
@@ -9,69 +11,72 @@ namespace soma {
 
 namespace {
 
-constexpr int kRedThreads = 256;
+constexpr int kUpdThreads = 128;
+constexpr int kUpdParams = kUpdThreads * 32;  // parameters of one block
 
-// One block per (expert, probe) pair: L+, L- = mean NLL of each sign (fp64
-// sums in a fixed order), the pairwise mean D = mean(nll+ - nll-) and the
-// coefficient D / (2 eps) (Eq. main-spsa).  nll: [pairs][n_sign][B*T].
-__global__ void __launch_bounds__(kRedThreads)
-reduce_losses_kernel(const float* __restrict__ nll, int n_sign, int BT, float eps,
-                     float* losses_out, float* coef_out, float* coef_ws, int* status) {
-  __shared__ double red[3][kRedThreads];
-  const int pair = blockIdx.x;
-  const float* np = nll + (int64_t)pair * n_sign * BT;
-  double sp = 0.0, sm = 0.0, sd = 0.0;
-  for (int j = threadIdx.x; j < BT; j += kRedThreads) {
-    const float a = np[j];
-    sp += (double)a;
-    if (n_sign == 2) {
-      const float b = np[BT + j];
-      sm += (double)b;
-      sd += (double)a - (double)b;  // exact in fp64 for any two fp32 values
-    }
+// Adds the probe terms c_i z_i of probes i0 .. i0 + 3 to the 32 parameters of
+// run q (32q .. 32q + 31) owned by this thread.  One Philox block covers the
+// 128 parameters of four consecutive runs, i.e. of a group of four
+// consecutive lanes (q % 4 == lane % 4), so lane j of the group draws the
+// block of probe i0 + j (and its activity block for sparse probes) and the
+// four lanes pass words round: in round k every lane sends word (j - k) % 4
+// of its block and receives, from lane (j + k) % 4 of the group, the word of
+// its own run for probe i0 + (j + k) % 4.  One Philox block per 128
+// parameters and probe, one shuffle per probe and word kind.  All 32 lanes
+// of the warp take part.
+__device__ __forceinline__ void accumulate_x4(float (&acc)[32], const float* cf, int n_pert,
+                                              int i0, const ProbeKey& pk0, int64_t q, int sparse,
+                                              int64_t dense_from) {
+  const int lane = threadIdx.x & 31;
+  const int j = lane & 3, base = lane & ~3;
+  uint4 wn = make_uint4(0u, 0u, 0u, 0u), wa = make_uint4(0u, 0u, 0u, 0u);
+  if (i0 + j < n_pert) {
+    ProbeKey pk = pk0;
+    pk.probe = (uint32_t)(i0 + j);
+    const uint32_t blk = (uint32_t)(q >> 2);
+    wn = probe_block(pk, blk);
+    if (sparse) wa = probe_block(activity_key(pk), blk);
   }
-  red[0][threadIdx.x] = sp;
-  red[1][threadIdx.x] = sm;
-  red[2][threadIdx.x] = sd;
-  __syncthreads();
-  for (int w = kRedThreads / 2; w > 0; w >>= 1) {
-    if (threadIdx.x < w) {
-      red[0][threadIdx.x] += red[0][threadIdx.x + w];
-      red[1][threadIdx.x] += red[1][threadIdx.x + w];
-      red[2][threadIdx.x] += red[2][threadIdx.x + w];
-    }
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) {
-    const double inv = 1.0 / (double)BT;
-    const double Lp = red[0][0] * inv;
-    bool finite = isfinite(Lp);
-    if (losses_out) losses_out[(int64_t)pair * n_sign] = (float)Lp;
-    if (n_sign == 2) {
-      const double Lm = red[1][0] * inv;
-      const double D = red[2][0] * inv;
-      const double c = (eps == 0.f) ? 0.0 : D / (2.0 * (double)eps);
-      finite = finite && isfinite(Lm) && isfinite(c);
-      if (losses_out) losses_out[(int64_t)pair * 2 + 1] = (float)Lm;
-      if (coef_out) coef_out[pair] = (float)c;
-      if (coef_ws) coef_ws[pair] = (float)c;
-    }
-    if (!finite && status) atomicCAS(status, 0, kStatusNonFinite);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int send = (j - k) & 3, from = (j + k) & 3;
+    const uint32_t rn =
+        __shfl_sync(0xffffffffu, word_of(wn, send), base | from);
+    uint32_t act = 0xFFFFFFFFu;
+    if (sparse) act = probe_law_act(__shfl_sync(0xffffffffu, word_of(wa, send), base | from), q,
+                                    dense_from);
+    const int i = i0 + from;
+    if (i >= n_pert) continue;
+    const uint32_t neg = raw_to_natural(rn);
+    const float c = cf[i];
+#pragma unroll
+    for (int b = 0; b < 32; ++b)
+      if ((act >> b) & 1u) acc[b] += ((neg >> b) & 1u) ? -c : c;
   }
 }
 
-constexpr int kUpdThreads = 128;
+// Writes the block's 32 x kUpdThreads accumulators to shared memory in
+// parameter order (thread t: parameters 32t .. 32t + 31 of the block).
+__device__ __forceinline__ void stage_acc(float* sacc, const float (&acc)[32], float scale) {
+  float4* dst = reinterpret_cast<float4*>(sacc + 32 * threadIdx.x);
+#pragma unroll
+  for (int j4 = 0; j4 < 8; ++j4)
+    dst[j4] = make_float4(scale * acc[4 * j4], scale * acc[4 * j4 + 1], scale * acc[4 * j4 + 2],
+                          scale * acc[4 * j4 + 3]);
+}
 
 // theta[e][p] -= lr * (1/n) * sum_i coef[e][i] z_{e,i}[p] (Eq. main-spsa).
-// Thread q of expert e owns the 32 parameters 32q .. 32q + 31, whose probe
-// bits are one Philox word per probe (two for sparse probes), under the probe
-// law of probe_law_words.  An expert whose coefficients are not all finite is
-// left unchanged.
+// Thread q of expert e accumulates the 32 parameters 32q .. 32q + 31 under
+// the probe law of probe_law_words (accumulate_x4); the block then stages its
+// 4096 steps in shared memory and reads and writes theta as consecutive
+// float4s, so a warp's access covers 512 contiguous bytes.  An expert whose
+// coefficients are not all finite is left unchanged.
 __global__ void __launch_bounds__(kUpdThreads)
 sgd_update_kernel(float* __restrict__ params, int64_t P, int64_t dense_from, int n_pert,
                   int sparse, float lr, uint64_t seed, uint64_t step,
                   const float* __restrict__ coef) {
   extern __shared__ float cf[];  // [n_pert]
+  __shared__ __align__(16) float sacc[kUpdParams];
   __shared__ int all_finite;
   const int e = blockIdx.y;
   if (threadIdx.x == 0) all_finite = 1;
@@ -84,35 +89,34 @@ sgd_update_kernel(float* __restrict__ params, int64_t P, int64_t dense_from, int
   __syncthreads();
   if (!all_finite) return;
   const int64_t q = (int64_t)blockIdx.x * kUpdThreads + threadIdx.x;
-  const int64_t p0 = q * 32;
-  if (p0 >= P) return;
   float acc[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-  for (int i = 0; i < n_pert; ++i) {
-    uint32_t neg, act;
-    probe_law_words(make_probe_key(seed, step, (uint32_t)e, (uint32_t)i), (int)q, sparse,
-                    dense_from, neg, act);
-    const float c = cf[i];
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
-  }
-  const float scale = lr / (float)n_pert;
+  const ProbeKey pk0 = make_probe_key(seed, step, (uint32_t)e, 0u);
+  // runs past the end draw probe words too (their Philox counters exist) and
+  // are simply not written back
+  for (int i0 = 0; i0 < n_pert; i0 += 4) accumulate_x4(acc, cf, n_pert, i0, pk0, q, sparse,
+                                                       dense_from);
+  stage_acc(sacc, acc, lr / (float)n_pert);
+  __syncthreads();
+  const int64_t p0 = (int64_t)blockIdx.x * kUpdParams;
   float* th = params + (int64_t)e * P + p0;
-  if (p0 + 32 <= P && (P & 3) == 0) {
-    // P a multiple of 4 and p0 of 32: 16-byte aligned
-#pragma unroll
-    for (int j4 = 0; j4 < 8; ++j4) {
-      float4 v = reinterpret_cast<float4*>(th)[j4];
-      v.x -= scale * acc[4 * j4 + 0];
-      v.y -= scale * acc[4 * j4 + 1];
-      v.z -= scale * acc[4 * j4 + 2];
-      v.w -= scale * acc[4 * j4 + 3];
-      reinterpret_cast<float4*>(th)[j4] = v;
+  const int64_t left = P - p0;
+  for (int k = threadIdx.x; k < kUpdParams / 4; k += kUpdThreads) {
+    const int64_t p = 4LL * k;
+    if (p >= left) break;
+    if (p + 4 <= left && (P & 3) == 0) {
+      // P a multiple of 4: theta + p is 16-byte aligned
+      float4 v = reinterpret_cast<float4*>(th)[k];
+      const float4 d = reinterpret_cast<const float4*>(sacc)[k];
+      v.x -= d.x;
+      v.y -= d.y;
+      v.z -= d.z;
+      v.w -= d.w;
+      reinterpret_cast<float4*>(th)[k] = v;
+    } else {
+      for (int64_t pp = p; pp < p + 4 && pp < left; ++pp) th[pp] -= sacc[pp];
     }
-  } else {
-    for (int j = 0; j < 32 && p0 + j < P; ++j) th[j] -= scale * acc[j];
   }
 }
 
@@ -121,13 +125,16 @@ sgd_update_kernel(float* __restrict__ params, int64_t P, int64_t dense_from, int
 //   m = b1 m + (1 - b1) g,  v = b2 v + (1 - b2) g^2,
 //   theta -= lr * (m / bc1) / (sqrt(v / bc2) + delta),
 // with z^{(a)} drawn with step counter steps[a] under the probe law of
-// probe_law_words.  Thread q owns the 32 parameters 32q .. 32q + 31.  An
-// expert whose coefficients are not all finite is left unchanged, moments
-// included.
+// probe_law_words.  Thread q accumulates the 32 parameters 32q .. 32q + 31;
+// the block stages the averaged estimate in shared memory and updates
+// theta, m and v as consecutive float4s.  An expert whose coefficients are
+// not all finite is left unchanged, moments included.
 __global__ void __launch_bounds__(kUpdThreads)
 adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __restrict__ v,
                    int64_t P, int64_t dense_from, int n_experts, int n_pert, int sparse,
                    uint64_t seed, AdamSteps steps, const float* __restrict__ coef, AdamArgs h) {
+  extern __shared__ float cf[];  // [n_pert]: the coefficients of one accumulation batch
+  __shared__ __align__(16) float sacc[kUpdParams];
   __shared__ int all_finite;
   const int e = blockIdx.y;
   if (threadIdx.x == 0) all_finite = 1;
@@ -139,34 +146,56 @@ adam_update_kernel(float* __restrict__ params, float* __restrict__ m, float* __r
   __syncthreads();
   if (!all_finite) return;
   const int64_t q = (int64_t)blockIdx.x * kUpdThreads + threadIdx.x;
-  const int64_t p0 = q * 32;
-  if (p0 >= P) return;
   float acc[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) acc[j] = 0.f;
   for (int a = 0; a < steps.n_acc; ++a) {
-    const float* ca = coef + ((int64_t)a * n_experts + e) * n_pert;
-    for (int i = 0; i < n_pert; ++i) {
-      uint32_t neg, act;
-      probe_law_words(make_probe_key(seed, steps.step[a], (uint32_t)e, (uint32_t)i), (int)q,
-                      sparse, dense_from, neg, act);
-      const float c = ca[i];
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if ((act >> j) & 1u) acc[j] += ((neg >> j) & 1u) ? -c : c;
-    }
+    for (int i = threadIdx.x; i < n_pert; i += kUpdThreads)
+      cf[i] = coef[((int64_t)a * n_experts + e) * n_pert + i];
+    __syncthreads();
+    const ProbeKey pk0 = make_probe_key(seed, steps.step[a], (uint32_t)e, 0u);
+    for (int i0 = 0; i0 < n_pert; i0 += 4)
+      accumulate_x4(acc, cf, n_pert, i0, pk0, q, sparse, dense_from);
+    __syncthreads();  // cf is refilled for the next batch
   }
-  const float inv = 1.f / ((float)steps.n_acc * (float)n_pert);
+  stage_acc(sacc, acc, 1.f / ((float)steps.n_acc * (float)n_pert));
+  __syncthreads();
+  const int64_t p0 = (int64_t)blockIdx.x * kUpdParams;
   const int64_t base = (int64_t)e * P + p0;
-  const int cnt = P - p0 < 32 ? (int)(P - p0) : 32;
-  for (int j = 0; j < cnt; ++j) {
-    const float th = params[base + j];
-    const float g = fmaf(h.wd, th, acc[j] * inv);
-    const float mj = fmaf(h.b1, m[base + j], (1.f - h.b1) * g);
-    const float vj = fmaf(h.b2, v[base + j], (1.f - h.b2) * g * g);
-    m[base + j] = mj;
-    v[base + j] = vj;
-    params[base + j] = th - h.lr * (mj * h.inv_bc1) / (sqrtf(vj * h.inv_bc2) + h.delta);
+  const int64_t left = P - p0;
+  for (int k = threadIdx.x; k < kUpdParams / 4; k += kUpdThreads) {
+    const int64_t p = 4LL * k;
+    if (p >= left) break;
+    if (p + 4 <= left && (P & 3) == 0) {
+      float4 t4 = reinterpret_cast<float4*>(params + base)[k];
+      float4 m4 = reinterpret_cast<float4*>(m + base)[k];
+      float4 v4 = reinterpret_cast<float4*>(v + base)[k];
+      const float4 g4 = reinterpret_cast<const float4*>(sacc)[k];
+      float* tt = &t4.x;
+      float* mm = &m4.x;
+      float* vv = &v4.x;
+      const float* gg = &g4.x;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float g = fmaf(h.wd, tt[c], gg[c]);
+        mm[c] = fmaf(h.b1, mm[c], (1.f - h.b1) * g);
+        vv[c] = fmaf(h.b2, vv[c], (1.f - h.b2) * g * g);
+        tt[c] = tt[c] - h.lr * (mm[c] * h.inv_bc1) / (sqrtf(vv[c] * h.inv_bc2) + h.delta);
+      }
+      reinterpret_cast<float4*>(params + base)[k] = t4;
+      reinterpret_cast<float4*>(m + base)[k] = m4;
+      reinterpret_cast<float4*>(v + base)[k] = v4;
+    } else {
+      for (int64_t pp = p; pp < p + 4 && pp < left; ++pp) {
+        const float th = params[base + pp];
+        const float g = fmaf(h.wd, th, sacc[pp]);
+        const float mj = fmaf(h.b1, m[base + pp], (1.f - h.b1) * g);
+        const float vj = fmaf(h.b2, v[base + pp], (1.f - h.b2) * g * g);
+        m[base + pp] = mj;
+        v[base + pp] = vj;
+        params[base + pp] = th - h.lr * (mj * h.inv_bc1) / (sqrtf(vj * h.inv_bc2) + h.delta);
+      }
+    }
   }
 }
 
@@ -253,26 +282,26 @@ __global__ void debug_wait_timeout_kernel(uint32_t max_polls, int* status) {
   if (threadIdx.x == 0 && !tc::mbar_wait(&bar, 0u, max_polls))
     atomicCAS(status, 0, kStatusTimeout);
 }
-}  // namespace
 
-cudaError_t launch_reduce_losses(const float* nll, int pairs, int n_sign, int B, int T, float eps,
-                                 float* losses_out, float* coef_out, float* coef_ws, int* status,
-                                 cudaStream_t stream) {
-  trace_begin(SOMA_TRACE_REDUCE, stream);
-  reduce_losses_kernel<<<pairs, kRedThreads, 0, stream>>>(nll, n_sign, B * T, eps, losses_out,
-                                                          coef_out, coef_ws, status);
-  trace_end(SOMA_TRACE_REDUCE, stream);
-  return cudaGetLastError();
+// An index check whose condition is false and that guards no access: the
+// reporting path of the checked build (nothing happens in the default one).
+__global__ void debug_check_fail_kernel(int* status) {
+  if (threadIdx.x == 0) (void)SOMA_CHECK(blockDim.x == 0, status);
 }
+}  // namespace
 
 cudaError_t launch_sgd_update(float* params, int64_t P, int64_t dense_from, int n_experts,
                               int n_pert, int sparse, float lr, uint64_t seed, uint64_t step,
                               const float* coef, cudaStream_t stream) {
   const int64_t words = (P + 31) / 32;
   dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
+  const size_t smem = (size_t)n_pert * sizeof(float);  // plus the 16 KB staging array
+  cudaError_t e = cudaFuncSetAttribute(sgd_update_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   trace_begin(SOMA_TRACE_UPDATE, stream);
-  sgd_update_kernel<<<grid, kUpdThreads, n_pert * sizeof(float), stream>>>(
-      params, P, dense_from, n_pert, sparse, lr, seed, step, coef);
+  sgd_update_kernel<<<grid, kUpdThreads, smem, stream>>>(params, P, dense_from, n_pert, sparse,
+                                                          lr, seed, step, coef);
   trace_end(SOMA_TRACE_UPDATE, stream);
   return cudaGetLastError();
 }
@@ -320,9 +349,13 @@ cudaError_t launch_probe_adam(float* params, float* m, float* v, int64_t P, int6
                               cudaStream_t stream) {
   const int64_t words = (P + 31) / 32;
   dim3 grid((unsigned)((words + kUpdThreads - 1) / kUpdThreads), n_experts);
+  const size_t smem = (size_t)n_pert * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(adam_update_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   trace_begin(SOMA_TRACE_UPDATE, stream);
-  adam_update_kernel<<<grid, kUpdThreads, 0, stream>>>(params, m, v, P, dense_from, n_experts,
-                                                       n_pert, sparse, seed, steps, coef, h);
+  adam_update_kernel<<<grid, kUpdThreads, smem, stream>>>(params, m, v, P, dense_from, n_experts,
+                                                          n_pert, sparse, seed, steps, coef, h);
   trace_end(SOMA_TRACE_UPDATE, stream);
   return cudaGetLastError();
 }
@@ -332,6 +365,11 @@ cudaError_t launch_adam_update(float* params, float* m, float* v, const Layout& 
                                const float* coef, const AdamArgs& h, cudaStream_t stream) {
   return launch_probe_adam(params, m, v, lay.P, lay.P, n_experts, n_pert, sparse, seed, steps,
                            coef, h, stream);
+}
+
+cudaError_t launch_debug_check_fail(int* status, cudaStream_t stream) {
+  debug_check_fail_kernel<<<1, 32, 0, stream>>>(status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_debug_wait_timeout(uint32_t max_polls, int* status, cudaStream_t stream) {

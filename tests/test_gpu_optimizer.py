@@ -3,7 +3,7 @@
 The step is split into two parts, each compared with the fp64 oracle on the
 same seeded inputs:
 - soma_spsa_estimate, with sparse and dense probes. Checked: L+, L- and the
-  coefficients (tiny, ragged and a CUDA-core shape in full; SOMA N=2 at
+  coefficients (tiny, ragged and a batch of 70 in two chunks in full; SOMA N=2 at
   sampled probes).
 - soma_adam_update, given coefficients. Checked: theta', m' and v' against
   the oracle's Adam update of the same coefficients.
@@ -55,7 +55,7 @@ def _batch(N, B, T, seed):
 @pytest.mark.parametrize("E,H,N,n,B,T", [
     (32, 64, 1, 8, 4, 64),     # the tiny workload (tensor path)
     (40, 72, 2, 5, 5, 9),      # ragged: every tile dimension padded
-    (16, 32, 1, 3, 70, 4),     # B > 64: the CUDA-core path
+    (16, 32, 1, 3, 70, 4),     # B > 64: two tensor-core chunks (64 + 6)
 ])
 def test_sparse_estimate_full(oracle_mod, E, H, N, n, B, T):
     theta = inputs.init_params(N, E, H, seed=21, std=0.1)

@@ -220,9 +220,12 @@ def test_init_experts():
     assert q.std().item() == pytest.approx(0.5, rel=0.02)
 
 
-def test_large_batch_uses_the_cuda_core_path(oracle_mod):
-    # more than 64 sequences per expert: the fp32 CUDA-core kernels
-    N, E, H, B, T, n = 1, 3, 5, 130, 4, 2
+@pytest.mark.parametrize("B", [65, 130, 192])
+def test_large_batch_runs_in_chunks(oracle_mod, B):
+    # more than 64 sequences per expert: tensor-core sweeps over chunks of at
+    # most 64 sequences (65 = 64 + 1, 130 = 64 + 64 + 2, 192 = 3 x 64), each
+    # writing its part of the loss partials of the whole batch
+    N, E, H, T, n = 2, 3, 70, 4, 3
     theta = inputs.init_params(N, E, H, seed=21, std=0.3)
     bx = inputs.expert_batch(N, B, T, 1, seed=22, step=0)
     _full_parity(oracle_mod, theta, bx, E, H, n, 1e-3, 1e-2, 3, 1)

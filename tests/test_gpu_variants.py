@@ -1,6 +1,6 @@
 """Parity of the two mechanism variants on the GPU (App. D): per-probe batches
 and the summed-loss control arm, through soma_spsa_estimate_opts, against the
-fp64 oracle on the same seeded inputs (tensor-core and CUDA-core shapes)."""
+fp64 oracle on the same seeded inputs (resident, persistent and chunked shapes)."""
 import numpy as np
 import pytest
 import torch
@@ -33,7 +33,7 @@ def _estimate(theta, bx, E, H, n, kind, eps, seed, step, batch_per_probe, summed
 @pytest.mark.parametrize("E,H,N,n,B,T", [
     (32, 64, 3, 8, 4, 24),     # tensor path
     (40, 72, 2, 5, 5, 9),      # ragged
-    (16, 32, 2, 3, 70, 4),     # B > 64: the CUDA-core path
+    (16, 32, 2, 3, 70, 4),     # B > 64: two tensor-core chunks (64 + 6)
 ])
 def test_variant_estimate(oracle_mod, kind, batch_per_probe, summed_loss, E, H, N, n, B, T):
     theta = inputs.init_params(N, E, H, seed=31, std=0.1)

@@ -3,7 +3,7 @@ device memory, with its scratch in a fixed array inside the library.
 
 Through the C ABI, on every path whose scratch lives in that array (the
 resident small-expert kernel, the persistent tensor-core kernel with one and
-two probes per operand group, the CUDA-core kernels for batches above 64):
+two probes per operand group, and a batch above 64 that runs in chunks):
  - two calls in a row (the second continues from the first's parameters)
    give bit for bit the losses, coefficients and updated parameters of
    soma_spsa_step with a caller workspace;
@@ -36,7 +36,7 @@ SHAPES = {
     "resident_n256_cut": "n256",                           # 3 experts of the N=256 shape
     "persistent_p2": (2, 64, 96, 8, 32, 16, 1e-3, 1e-2),   # two probes per operand group
     "persistent_p1": (1, 40, 130, 40, 12, 5, 1e-3, 1e-2),  # B = 40: one probe per group
-    "cuda_core": (1, 6, 20, 70, 6, 3, 1e-3, 1e-2),         # B = 70 > 64
+    "chunked": (1, 6, 20, 70, 6, 3, 1e-3, 1e-2),           # B = 70 > 64: chunks of 64 and 6
 }
 
 
@@ -147,7 +147,7 @@ def test_static_step_large_then_small():
     theta_b = inputs.init_params(N, E, H, seed=5, std=None)
     bx_b = torch.from_numpy(inputs.expert_batch(N, B, T, 2, seed=8, step=0)).cuda()
     _static_call(f, torch.from_numpy(theta_b).cuda(), bx_b, big, 1, 0)
-    for name in ("persistent_p2", "persistent_p1", "cuda_core", "resident_tiny"):
+    for name in ("persistent_p2", "persistent_p1", "chunked", "resident_tiny"):
         theta, batch, sizes = _shape(name)
         bx = torch.from_numpy(batch(0)).cuda()
         p_ref = torch.from_numpy(theta).cuda()
