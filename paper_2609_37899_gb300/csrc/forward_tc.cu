@@ -310,6 +310,8 @@ struct TcArgs {
   float* pm;             // [N*n*2][B_mem][T][2] head max partials
   float* ps;             // sum-exp partials
   float* ply;            // [N*n*2][B_mem][T] target logits
+  const uint2* zb;       // probe-word table (zbits_kernel), n_zrows rows, then activity words
+  size_t n_zrows;
   int* status;
   // extents for the index checks of the checked build (bytes of w16, wo16,
   // each op buffer and the byte batch; floats of cst, pm / ps, ply, params;
@@ -357,6 +359,23 @@ __device__ __forceinline__ int64_t z_param(const TcArgs& a, const Task& T, int r
   const int64_t R = (int64_t)tile_gate(r) * a.g.H + 32 * T.m + tile_unit(r);  // W row of tile row r
   return st < a.g.Sx ? L.w_ih + R * a.g.E + (int64_t)kKt * st
                      : L.w_hh + R * a.g.H + (int64_t)kKt * (st - a.g.Sx);
+}
+
+// Probe-word table: for every (expert, probe, tile, stage) the raw words of
+// the stage's 64 parameters of each of the 128 tile rows, one uint2 per row
+// (runs 0 and 1 of the stage); the activity words of sparse probes follow in
+// a second table of the same shape.  Tiles: the MT gate tiles of S stages,
+// then the two head tiles of Sh stages.
+constexpr int kZRows = 128;
+
+__host__ __device__ __forceinline__ int zbits_stages(const TcGeom& g) {
+  return g.MT * g.S + 2 * g.Sh;
+}
+
+__host__ __device__ __forceinline__ size_t zbits_row(const TcGeom& g, int e, int probe, bool head,
+                                                     int m) {
+  const int ts = head ? g.MT * g.S + m * g.Sh : m * g.S;
+  return (((size_t)e * g.n_pert + probe) * zbits_stages(g) + ts) * kZRows;
 }
 
 // Gate epilogue of one task for one warp of TMEM lane quarter q4 (units
@@ -791,9 +810,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     __syncwarp();
   } else if (warp >= kZWarp0 && warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
-    // Thread (probe gtid / 128, row gtid % 128 = TMEM lane).  The raw words
-    // of the next stage are drawn before waiting for its slot, so the Philox
-    // rounds overlap the wait instead of following it.
+    // Thread (probe gtid / 128, row gtid % 128 = TMEM lane).  The raw probe
+    // words of a stage come from the table zbits_kernel wrote before the
+    // sweep, loaded two stages ahead.  A stage's fp16 row is expanded while
+    // the previous stage's slot is still busy; once its slot is free it is
+    // stored, and the next stage is expanded while that store completes.
     if (do_z) {
       const int gtid = tid - kZWarp0 * 32;
       const int r = gtid & 127, pz = gtid >> 7;
@@ -802,23 +823,29 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       bool alive = true;
       for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
         const Task T = make_task(a, task);
-        const bool active = pz < T.p_valid;  // uniform over the warp
-        const ProbeKey pk =
-            make_probe_key(s.seed, s.step, (uint32_t)T.e, (uint32_t)(T.grp * g.P + pz));
-        const ProbeKey pka = activity_key(pk);
-        ZSlot cache, cache_a;
-        cache.blk = 0xFFFFFFFFu;
-        cache_a.blk = 0xFFFFFFFFu;
-        const int split = T.head ? T.nst : g.Sx;
-        const int64_t seg0 = z_param(a, T, r, 0);
-        const int64_t seg1 = z_param(a, T, r, split) - (int64_t)kKt * split;
-        uint32_t raw[kKt / 32] = {}, act[kKt / 32] = {};
+        const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
+        // uniform over the warp
+        const bool active = pz < T.p_valid &&
+                            SOMA_CHECK(row0 + (size_t)kZRows * (T.nst - 1) < a.n_zrows, status);
+        const uint2* zn = a.zb + row0;
+        const uint2* za = a.zb + a.n_zrows + row0;
+        const uint2 none = make_uint2(0u, 0u);
+        // raw words (and activity words) of stages st + 1 and st + 2
+        uint2 n1 = none, n2 = none, a1 = none, a2 = none;
+        uint32_t zw[kKt / 2];
         if (active) {
-#pragma unroll
-          for (int w = 0; w < kKt / 32; ++w) {
-            raw[w] = z_run_raw(pk, seg0 + 32 * w, cache);
-            if (SPARSE) act[w] = z_run_raw(pka, seg0 + 32 * w, cache_a);
+          const uint2 n0 = __ldg(zn);
+          const uint2 a0 = SPARSE ? __ldg(za) : none;
+          if (T.nst > 1) {
+            n1 = __ldg(zn + kZRows);
+            if (SPARSE) a1 = __ldg(za + kZRows);
           }
+          if (T.nst > 2) {
+            n2 = __ldg(zn + 2 * kZRows);
+            if (SPARSE) a2 = __ldg(za + 2 * kZRows);
+          }
+          z_run_pairs<SPARSE>(n0.x, a0.x, zw);
+          z_run_pairs<SPARSE>(n0.y, a0.y, zw + 16);
         }
         for (int st = 0; st < T.nst; ++st, ++gs) {
           const int q = gs % kStages;
@@ -832,23 +859,22 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           tc_fence_after();
           if (active &&
               SOMA_CHECK(kZCol0 + 64u * (uint32_t)q + 32u * pz + 32u <= kTmemCols, status)) {
-            uint32_t zw[kKt / 2];
-#pragma unroll
-            for (int w = 0; w < kKt / 32; ++w) z_run_pairs<SPARSE>(raw[w], act[w], zw + 16 * w);
             tmem_st32(trow + 64u * (uint32_t)q, zw);
+            if (st + 1 < T.nst) {
+              z_run_pairs<SPARSE>(n1.x, a1.x, zw);
+              z_run_pairs<SPARSE>(n1.y, a1.y, zw + 16);
+              n1 = n2;
+              a1 = a2;
+              if (st + 3 < T.nst) {
+                n2 = __ldg(zn + (size_t)kZRows * (st + 3));
+                if (SPARSE) a2 = __ldg(za + (size_t)kZRows * (st + 3));
+              }
+            }
             tmem_wait_st();
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->full[q]);
-          if (active && st + 1 < T.nst) {
-            const int64_t p1 = (st + 1 < split ? seg0 : seg1) + (int64_t)kKt * (st + 1);
-#pragma unroll
-            for (int w = 0; w < kKt / 32; ++w) {
-              raw[w] = z_run_raw(pk, p1 + 32 * w, cache);
-              if (SPARSE) act[w] = z_run_raw(pka, p1 + 32 * w, cache_a);
-            }
-          }
         }
       }
     }
@@ -930,6 +956,43 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
 
 __global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
   xpart_block(a, op, t, blockIdx.x);
+}
+
+// The probe-word table of one sweep (zbits_row): block b writes the 128 rows
+// of (expert, probe, tile stage) b, thread r the raw words of the stage's
+// 64 parameters of tile row r (and their activity words for sparse probes).
+template <bool SPARSE>
+__global__ void zbits_kernel(const TcArgs a, uint2* __restrict__ out) {
+  const TcGeom& g = a.g;
+  const Sweep& s = a.sw;
+  const int TS = zbits_stages(g);
+  const size_t b = blockIdx.x;
+  const int ts = (int)(b % TS), i = (int)((b / TS) % g.n_pert), e = (int)(b / TS / g.n_pert);
+  const int r = threadIdx.x;
+  Task T;
+  T.head = ts >= g.MT * g.S;
+  T.e = e;
+  const int tj = T.head ? ts - g.MT * g.S : ts;
+  const int per = T.head ? g.Sh : g.S;
+  T.m = tj / per;
+  const int st = tj % per;
+  const int64_t p0 = z_param(a, T, r, st);
+  const ProbeKey pk = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
+  const size_t row = b * kZRows + (size_t)r;
+  if (!SOMA_CHECK(row < a.n_zrows, a.status)) return;
+  ZSlot c;
+  c.blk = 0xFFFFFFFFu;
+  uint2 w;
+  w.x = z_run_raw(pk, p0, c);
+  w.y = z_run_raw(pk, p0 + 32, c);
+  out[row] = w;
+  if (SPARSE) {
+    const ProbeKey pka = activity_key(pk);
+    c.blk = 0xFFFFFFFFu;
+    w.x = z_run_raw(pka, p0, c);
+    w.y = z_run_raw(pka, p0 + 32, c);
+    out[a.n_zrows + row] = w;
+  }
 }
 
 // fp16 A tiles of the gate weights ([x part | h part], gate-major rows) and
@@ -1180,6 +1243,8 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.cst = N * n * 2 * (size_t)g.Hp * g.Bp * sizeof(float);
   z.pm = N * n * 2 * g.Bm * (size_t)g.T * 2 * sizeof(float);
   z.ply = N * n * 2 * g.Bm * (size_t)g.T * sizeof(float);
+  // raw words and activity words
+  z.zb = 2 * N * n * (size_t)zbits_stages(g) * kZRows * sizeof(uint2);
   return z;
 }
 
@@ -1200,6 +1265,8 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.pm = tb.pm;
   a.ps = tb.ps;
   a.ply = tb.ply;
+  a.zb = tb.zbits;
+  a.n_zrows = (size_t)g.n_experts * g.n_pert * zbits_stages(g) * kZRows;
   a.status = status;
   a.t_gate = -1;
   a.t_head = -1;
@@ -1224,6 +1291,13 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   cudaMemsetAsync(tb.op[1], 0, z.op, stream);
   const int xblocks = g.n_experts * g.Sx * g.G;
   xpart_kernel<<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
+  if (s.eps != 0.f) {
+    const unsigned zblocks = (unsigned)(a.n_zrows / kZRows);
+    if (s.sparse)
+      zbits_kernel<true><<<zblocks, kZRows, 0, stream>>>(a, tb.zbits);
+    else
+      zbits_kernel<false><<<zblocks, kZRows, 0, stream>>>(a, tb.zbits);
+  }
   trace_end(SOMA_TRACE_PREP, stream);
 
   const int sms = sm_count();

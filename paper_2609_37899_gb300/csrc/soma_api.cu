@@ -57,7 +57,6 @@ constexpr size_t kGuard = 256;
 constexpr size_t kGuard = 0;
 #endif
 constexpr int kMaxRegions = 12;
-constexpr uint32_t kCanaryWord = 0x5A17C0DEu;
 
 struct Regions {
   int n;
@@ -72,6 +71,8 @@ struct Regions {
 };
 
 #ifdef SOMA_CHECKED
+constexpr uint32_t kCanaryWord = 0x5A17C0DEu;
+
 // The canary gaps of a workspace: before each region and after the last.
 struct Gaps {
   int n;
@@ -136,7 +137,7 @@ struct WsPlan {
   bool res;    // the resident small-expert kernel: no scratch but the coefficients
   TcGeom g;    // geometry of the largest chunk
   TcSizes z;   // buffer sizes: the largest chunk's operand and cell buffers
-  Regions r;   // w16, wo16, op[0], op[1], cst, pm, ps, ply, coef; or coef alone
+  Regions r;   // w16, wo16, op[0], op[1], cst, pm, ps, ply, zbits, coef; or coef alone
   size_t total;
 };
 
@@ -163,7 +164,8 @@ WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int
   const TcSizes zl = tc_sizes(make_tc_geom(lay, n_experts, n_pert, last, T, B));
   if (zl.op > w.z.op) w.z.op = zl.op;
   if (zl.cst > w.z.cst) w.z.cst = zl.cst;
-  for (size_t bytes : {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, coef})
+  for (size_t bytes :
+       {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, coef})
     w.r.add(bytes);
   w.total = w.r.total();
   return w;
@@ -180,6 +182,7 @@ TcBuffers carve_tc(const WsPlan& w, void* ws) {
   tb.pm = reinterpret_cast<float*>(p + w.r.off[5]);
   tb.ps = reinterpret_cast<float*>(p + w.r.off[6]);
   tb.ply = reinterpret_cast<float*>(p + w.r.off[7]);
+  tb.zbits = reinterpret_cast<uint2*>(p + w.r.off[8]);
   return tb;
 }
 

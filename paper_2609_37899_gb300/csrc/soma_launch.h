@@ -30,7 +30,7 @@ struct TcGeom {
 };
 
 struct TcSizes {
-  size_t w16, wo16, op, cst, pm, ply;
+  size_t w16, wo16, op, cst, pm, ply, zb;
 };
 
 struct TcBuffers {
@@ -41,6 +41,7 @@ struct TcBuffers {
   float* pm;       // head partial max
   float* ps;       // head partial sum-exp
   float* ply;      // target logits
+  uint2* zbits;    // probe-word table of the sweep
 };
 
 TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem);
