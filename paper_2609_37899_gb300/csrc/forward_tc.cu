@@ -139,12 +139,21 @@ __device__ __forceinline__ uint32_t z_run_raw(const ProbeKey& pk, int64_t p0, ZS
   return natural_to_raw(probe_bits32(pk, p0));
 }
 
+// 2^(15 - J): moves raw bits J and J + 16 to the sign bits 15 and 31 of a
+// pair word.  Read from the constant bank, so the move is an integer
+// multiply-add (the FMA pipe) instead of a shift and a logic op (both on the
+// integer pipe, which the rest of the pair-word work already loads).
+__constant__ uint32_t kPairShift[16] = {32768u, 16384u, 8192u, 4096u, 2048u, 1024u, 512u, 256u,
+                                        128u,   64u,    32u,   16u,   8u,    4u,    2u,   1u};
+
 // fp16 pair word J of a run: +-1 for dense probes; for sparse probes the
 // magnitude is kept only where the activity bit (same position in `act`) is
 // set, so inactive coordinates are +-0.
 template <bool SPARSE, int J>
 __device__ __forceinline__ uint32_t z_pair(uint32_t raw, uint32_t act) {
-  if (!SPARSE) return pm_pair<J>(raw, 0x3C003C00u);
+  // dense: the two sign bits isolated, moved into place, ORed with 1.0 | 1.0
+  // (an addition: the moved bits and 0x3C003C00 do not overlap)
+  if (!SPARSE) return (raw & (0x00010001u << J)) * kPairShift[J] + 0x3C003C00u;
   // activity bits at the sign positions (bits 15 and 31), each spread over
   // its 16-bit half by a byte permute that replicates the top bit of bytes 1
   // and 3: a mask of 1.0 magnitudes where the coordinate is active
