@@ -106,6 +106,20 @@ __host__ __device__ __forceinline__ int row_e2(int p) { return p == 0 ? 0 : 5; }
 __host__ __device__ __forceinline__ int col_c(int p) { return row_mean(p) - 1; }
 __host__ __device__ __forceinline__ int col_d(int p) { return row_dhat(p) - 1; }
 
+// The unperturbed layout: accumulator column block j (and operand row block
+// j + 1) holds sequences (4 grp + j) Bp .. + Bp - 1 of the expert's batch.
+// "Probe" p of a group then stands for the two blocks col_c(p) (its + lane)
+// and col_d(p) (its - lane), and its cell states sit where a probe's two
+// signs sit in the perturbed layout.
+__host__ __device__ __forceinline__ int inf_seq(const TcGeom& g, int grp, int blk, int b) {
+  return (4 * grp + blk) * g.Bp + b;
+}
+
+// Probe slots of the cell-state buffer per expert.
+__host__ __device__ __forceinline__ int cst_lanes(const TcGeom& g) {
+  return g.inf ? 2 * g.G : g.n_pert;
+}
+
 // Shared-memory carve-up of one ring slot.
 struct StageLayout {
   uint32_t a_off, b_off, bytes;
@@ -348,7 +362,7 @@ __device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
   const int rows = T.head ? 2 : g.MT;
   T.m = (j / g.G) % rows;
   T.e = j / (g.G * rows);
-  T.p_valid = min(g.P, a.sw.n_pert - T.grp * g.P);
+  T.p_valid = g.inf ? g.P : min(g.P, a.sw.n_pert - T.grp * g.P);
   if (T.head) {
     T.nst = g.Sh;
     T.a = a.wo16 + (((size_t)T.e * 2 + T.m) * g.Sh) * kTileA;
@@ -447,7 +461,7 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   }
   const int U = 32 * T.m + 8 * q4 + u8;
   const float2* cell = reinterpret_cast<const float2*>(a.cst) +
-                       (((int64_t)T.e * s.n_pert + i) * g.Hp + U) * (int64_t)g.Bp;
+                       (((int64_t)T.e * cst_lanes(g) + i) * g.Hp + U) * (int64_t)g.Bp;
   const bool load = U < H && a.t_gate > 0;
 #pragma unroll
   for (int j = 0; j < kEpiMaxChunks; ++j) {
@@ -482,7 +496,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
   const int kk = 32 * T.m % kKt + 8 * q4 + u8;
   const int i = T.grp * g.P + p;
   float2* cell = reinterpret_cast<float2*>(a.cst) +
-                 (((int64_t)T.e * s.n_pert + i) * g.Hp + U) * (int64_t)g.Bp;
+                 (((int64_t)T.e * cst_lanes(g) + i) * g.Hp + U) * (int64_t)g.Bp;
   const uint32_t tq = tacc + ((uint32_t)(32 * q4) << 16);  // gates 0, 1
   const uint32_t tq2 = tq + (16u << 16);                    // gates 2, 3
   const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
@@ -506,16 +520,32 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       float actp[4], actm[4];
+      if (g.inf) {
+        // unperturbed: the + and - lanes are two blocks' own pre-activations
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const float C = __uint_as_float(vc[h][k]) + G.bias[k];
-        const float D = fmaf(eps, __uint_as_float(vd[h][k]), G.dbias[k]);
-        if (k == 2) {  // g: tanh(x) = 2 sigmoid(2x) - 1
-          actp[k] = fmaf(sigm(2.f * (C + D)), 2.f, -1.f);
-          actm[k] = fmaf(sigm(2.f * (C - D)), 2.f, -1.f);
-        } else {
-          actp[k] = sigm(C + D);
-          actm[k] = sigm(C - D);
+        for (int k = 0; k < 4; ++k) {
+          const float ap = __uint_as_float(vc[h][k]) + G.bias[k];
+          const float am = __uint_as_float(vd[h][k]) + G.bias[k];
+          if (k == 2) {
+            actp[k] = fmaf(sigm(2.f * ap), 2.f, -1.f);
+            actm[k] = fmaf(sigm(2.f * am), 2.f, -1.f);
+          } else {
+            actp[k] = sigm(ap);
+            actm[k] = sigm(am);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float C = __uint_as_float(vc[h][k]) + G.bias[k];
+          const float D = fmaf(eps, __uint_as_float(vd[h][k]), G.dbias[k]);
+          if (k == 2) {  // g: tanh(x) = 2 sigmoid(2x) - 1
+            actp[k] = fmaf(sigm(2.f * (C + D)), 2.f, -1.f);
+            actm[k] = fmaf(sigm(2.f * (C - D)), 2.f, -1.f);
+          } else {
+            actp[k] = sigm(C + D);
+            actm[k] = sigm(C - D);
+          }
         }
       }
       const float cp = fmaf(actp[1], G.cprev[j][h].x, actp[0] * actp[2]);
@@ -530,7 +560,15 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
                          rM + b < g.rowsB && kk < kKt,
                      a.status)) {
         cell[b] = make_float2(cp, cm);
-        if (b < s.B) {
+        if (g.inf) {
+          // h of the two blocks into their own rows (the W product's rows)
+          if (inf_seq(g, T.grp, col_c(p), b) < s.B)
+            *reinterpret_cast<__half*>(out_tile + kmajor_offset(rM + b, kk, kKt)) =
+                __float2half_rn(hp);
+          if (inf_seq(g, T.grp, col_d(p), b) < s.B)
+            *reinterpret_cast<__half*>(out_tile + kmajor_offset(rD + b, kk, kKt)) =
+                __float2half_rn(hm);
+        } else if (b < s.B) {
           const float dh = hp - hm;
           *reinterpret_cast<__half*>(out_tile + kmajor_offset(rM + b, kk, kKt)) =
               __float2half_rn(0.5f * (hp + hm));
@@ -585,7 +623,9 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
 #pragma unroll
       for (int k = 0; k < 4; ++k) dbo[k] = __shfl_sync(0xffffffffu, dbo_r, r4 + 8 * k);
     }
-    const int64_t lane_plus = ((int64_t)T.e * s.n_pert + i) * 2;
+    // perturbed: lanes (e, i, +) and (e, i, -) for sequence b; unperturbed:
+    // lane (e, 0, +) for the sequences of blocks col_c(p) and col_d(p)
+    const int64_t lane_plus = g.inf ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2;
     const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
     for (int b0 = 0; b0 < g.Bp; b0 += 4) {
       // [k]: C and D of row r4 + 8 k, sequence b0 + bq
@@ -599,10 +639,15 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
       float lp[4], lm[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const float C = __uint_as_float(vc[k]) + bo[k];
-        const float D = fmaf(eps, __uint_as_float(vd[k]), dbo[k]);
-        lp[k] = C + D;
-        lm[k] = C - D;
+        if (g.inf) {
+          lp[k] = __uint_as_float(vc[k]) + bo[k];
+          lm[k] = __uint_as_float(vd[k]) + bo[k];
+        } else {
+          const float C = __uint_as_float(vc[k]) + bo[k];
+          const float D = fmaf(eps, __uint_as_float(vd[k]), dbo[k]);
+          lp[k] = C + D;
+          lm[k] = C - D;
+        }
       }
       float mp = fmaxf(fmaxf(lp[0], lp[1]), fmaxf(lp[2], lp[3]));
       float mm = fmaxf(fmaxf(lm[0], lm[1]), fmaxf(lm[2], lm[3]));
@@ -627,11 +672,30 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
         red[((p * g.Bp + b) * 2 + 0) * 4 + q4] = make_float2(mp, sp);
         red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
       }
-      if (b < s.B &&
-          SOMA_CHECK((size_t)(seq_offset(s, T.e, i, b) + t + 1) < a.n_bytes &&
-                         (size_t)(((lane_plus + 1) * s.B_mem + s.b0 + b) * (int64_t)s.T + t) <
-                             a.n_ply,
-                     a.status)) {
+      if (g.inf) {
+        // the target logit of each block's sequence, into lane (e, 0, +)
+#pragma unroll
+        for (int sg = 0; sg < 2; ++sg) {
+          const int q = inf_seq(g, T.grp, sg ? col_d(p) : col_c(p), b);
+          if (q >= s.B ||
+              !SOMA_CHECK((size_t)(seq_offset(s, T.e, 0, q) + t + 1) < a.n_bytes &&
+                              (size_t)((lane_plus * s.B_mem + s.b0 + q) * (int64_t)s.T + t) <
+                                  a.n_ply,
+                          a.status))
+            continue;
+          const int y = s.bytes[seq_offset(s, T.e, 0, q) + t + 1] - vq - r4;
+          if (y >= 0 && y < 32 && (y & 7) == 0) {
+            const int k = y >> 3;
+            const float* l = sg ? lm : lp;
+            a.ply[(lane_plus * s.B_mem + s.b0 + q) * (int64_t)s.T + t] =
+                k == 0 ? l[0] : k == 1 ? l[1] : k == 2 ? l[2] : l[3];
+          }
+        }
+      } else if (b < s.B &&
+                 SOMA_CHECK((size_t)(seq_offset(s, T.e, i, b) + t + 1) < a.n_bytes &&
+                                (size_t)(((lane_plus + 1) * s.B_mem + s.b0 + b) * (int64_t)s.T +
+                                         t) < a.n_ply,
+                            a.status)) {
         const int y = s.bytes[seq_offset(s, T.e, i, b) + t + 1] - vq - r4;
         // y = 8 k for the thread that holds the target row
         if (y >= 0 && y < 32 && (y & 7) == 0) {
@@ -652,15 +716,17 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     const int sgn = idx & 1;
     const int pb = idx >> 1;
     const int pp = pb / g.Bp, b = pb % g.Bp;
-    if (b >= s.B) continue;
+    // the partials' lane and sequence (see the target logits above)
+    const int qs = g.inf ? inf_seq(g, T.grp, sgn ? col_d(pp) : col_c(pp), b) : b;
+    if (qs >= s.B) continue;
     const float2* q = red + (size_t)idx * 4;
     const float M = fmaxf(fmaxf(q[0].x, q[1].x), fmaxf(q[2].x, q[3].x));
     float S = 0.f;
 #pragma unroll
     for (int k = 0; k < 4; ++k) S += q[k].y * __expf(q[k].x - M);
     const int i = T.grp * g.P + pp;
-    const int64_t ln = ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
-    const int64_t o = ((ln * s.B_mem + s.b0 + b) * (int64_t)s.T + t) * 2 + T.m;
+    const int64_t ln = g.inf ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
+    const int64_t o = ((ln * s.B_mem + s.b0 + qs) * (int64_t)s.T + t) * 2 + T.m;
     if (!SOMA_CHECK((size_t)o < a.n_pm, a.status)) continue;
     a.pm[o] = M;
     a.ps[o] = S;
@@ -935,7 +1001,23 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
     const int i = grp * g.P + p;
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
-    if (i < s.n_pert && b < s.B &&
+    if (g.inf) {
+      // row blocks 1..4: the embeddings of four blocks of sequences; 0, 5: zero
+      const int q = blkr >= 1 && blkr <= 4 ? inf_seq(g, grp, blkr - 1, b) : s.B;
+      float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (q < s.B && SOMA_CHECK((size_t)seq_offset(s, e, 0, q) + t < a.n_bytes, a.status)) {
+        const int y = s.bytes[seq_offset(s, e, 0, q) + t];
+        const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
+        if (SOMA_CHECK(k0 >= g.E || (size_t)(e * L.P + p0 + min(8, g.E - k0)) <= a.n_params,
+                       a.status)) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (k0 + j < g.E) x[j] = th[p0 + j];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = __float2half_rn(x[j]);
+    } else if (i < s.n_pert && b < s.B &&
         SOMA_CHECK((size_t)seq_offset(s, e, i, b) + t < a.n_bytes, a.status)) {
       const int y = s.bytes[seq_offset(s, e, i, b) + t];
       const int64_t p0 = L.emb + (int64_t)y * g.E + k0;
@@ -1240,6 +1322,18 @@ TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, 
   g.B = B;
   g.Bm = B_mem;
   g.T = T;
+  g.inf = 0;
+  return g;
+}
+
+TcGeom make_tc_geom_inf(const Layout& lay, int n_experts, int B, int T) {
+  TcGeom g = make_tc_geom(lay, n_experts, 1, 32, T, B);
+  g.P = 2;
+  g.G = (B + kInfGroupSeqs - 1) / kInfGroupSeqs;
+  g.rowsB = 3 * g.Bp * g.P;
+  g.tileB = (uint32_t)g.rowsB * kKt * 2;
+  g.B = B;
+  g.inf = 1;
   return g;
 }
 
@@ -1249,7 +1343,7 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.w16 = N * g.MT * g.S * kTileA;
   z.wo16 = N * 2 * g.Sh * kTileA;
   z.op = N * g.S * g.G * g.tileB;
-  z.cst = N * n * 2 * (size_t)g.Hp * g.Bp * sizeof(float);
+  z.cst = N * (size_t)cst_lanes(g) * 2 * (size_t)g.Hp * g.Bp * sizeof(float);
   z.pm = N * n * 2 * g.Bm * (size_t)g.T * 2 * sizeof(float);
   z.ply = N * n * 2 * g.Bm * (size_t)g.T * sizeof(float);
   // raw words and activity words

@@ -143,9 +143,11 @@ struct WsPlan {
 
 int chunk_size(int B, int b0) { return B - b0 < kTcMaxBatch ? B - b0 : kTcMaxBatch; }
 
+// A sweep of n_pert probes and n_sign signs.  With n_sign == 1 (eps = 0:
+// evaluation and routed inference) the tensor path takes the unperturbed
+// layout, every sequence of the batch in one sweep.
 WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int B, int T,
                   bool allow_res = true) {
-  (void)n_sign;
   WsPlan w;
   std::memset(&w, 0, sizeof(w));
   const Layout lay = make_layout(d.embed, d.hidden);
@@ -156,14 +158,19 @@ WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int
     w.total = w.r.total();
     return w;
   }
-  // the operand and cell buffers of every chunk fit those of the first one
-  // or of the last (smaller Bp packs two probes per group)
-  w.g = make_tc_geom(lay, n_experts, n_pert, chunk_size(B, 0), T, B);
-  w.z = tc_sizes(w.g);
-  const int last = chunk_size(B, (B - 1) / kTcMaxBatch * kTcMaxBatch);
-  const TcSizes zl = tc_sizes(make_tc_geom(lay, n_experts, n_pert, last, T, B));
-  if (zl.op > w.z.op) w.z.op = zl.op;
-  if (zl.cst > w.z.cst) w.z.cst = zl.cst;
+  if (n_sign == 1) {
+    w.g = make_tc_geom_inf(lay, n_experts, B, T);
+    w.z = tc_sizes(w.g);
+  } else {
+    // the operand and cell buffers of every chunk fit those of the first one
+    // or of the last (smaller Bp packs two probes per group)
+    w.g = make_tc_geom(lay, n_experts, n_pert, chunk_size(B, 0), T, B);
+    w.z = tc_sizes(w.g);
+    const int last = chunk_size(B, (B - 1) / kTcMaxBatch * kTcMaxBatch);
+    const TcSizes zl = tc_sizes(make_tc_geom(lay, n_experts, n_pert, last, T, B));
+    if (zl.op > w.z.op) w.z.op = zl.op;
+    if (zl.cst > w.z.cst) w.z.cst = zl.cst;
+  }
   for (size_t bytes :
        {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, coef})
     w.r.add(bytes);
@@ -398,7 +405,7 @@ int soma_eval_loss(const float* params, int n_experts, soma_dims d, const uint8_
     e = launch_forward_res(s, 1, loss_out, nullptr, nullptr, status, st);
   } else {
     const TcBuffers tb = carve_tc(w, workspace);
-    e = forward_tc_chunks(s, s.lay, tb, status, st);
+    e = launch_forward_tc(s, w.g, tb, status, st);
     if (e == cudaSuccess)
       e = launch_reduce_tc(tb, n_experts, 1, batch, seq_len, 0.f, loss_out, nullptr, nullptr,
                            status, st);
@@ -530,10 +537,9 @@ int soma_debug_probe(uint64_t seed, uint64_t step, int expert, int pert, int pro
 namespace {
 
 constexpr int kMaxRoutes = 16;
-constexpr int kMixChunk = kTcMaxBatch;  // sequences per expert and sweep
 
 struct MixPlan {
-  int b_max, Bc, chunks;
+  int b_max;
   WsPlan sweep;
   size_t gather, route, slot, grouped, nll, total;
   std::vector<int32_t> gather_h, slot_h;
@@ -557,14 +563,13 @@ bool plan_mixture(const soma_dims& d, int N, const int32_t* routes, int R, int k
   for (int r = 0; r < R; ++r)
     for (int j = 0; j < k; ++j)
       m.gather_h[(size_t)routes[(size_t)r * k + j] * m.b_max + m.slot_h[(size_t)r * k + j]] = r;
-  m.Bc = m.b_max < kMixChunk ? m.b_max : kMixChunk;
-  m.chunks = (m.b_max + m.Bc - 1) / m.Bc;
-  // the mixture reads per-target NLL, which the persistent kernel keeps
-  m.sweep = plan_sweep(d, N, 1, 1, m.Bc, T, false);
+  // one unperturbed sweep over every expert's group of requests; the
+  // mixture reads per-target NLL, which the persistent kernel keeps
+  m.sweep = plan_sweep(d, N, 1, 1, m.b_max, T, false);
   m.gather = round_up((size_t)N * m.b_max * sizeof(int32_t));
   m.route = round_up((size_t)R * k * sizeof(int32_t));
   m.slot = m.route;
-  m.grouped = round_up((size_t)N * m.Bc * (T + 1));
+  m.grouped = round_up((size_t)N * m.b_max * (T + 1));
   m.nll = round_up((size_t)N * m.b_max * T * sizeof(float));
   m.total = m.sweep.total + m.gather + m.route + m.slot + m.grouped + m.nll;
   return true;
@@ -623,24 +628,23 @@ int soma_mixture_nll(const float* params, int n_experts, soma_dims d, const uint
   s.n_experts = n_experts;
   s.n_pert = 1;
   s.n_sign = 1;
-  s.B = m.Bc;
+  s.B = m.b_max;
   s.T = seq_len;
   s.b0 = 0;
-  s.B_mem = m.Bc;
+  s.B_mem = m.b_max;
   s.eps = 0.f;
   s.sparse = 0;
   s.batch_per_probe = 0;
   s.seed = 0;
   s.step = 0;
-  for (int c = 0; c < m.chunks && e == cudaSuccess; ++c) {
-    const int b0 = c * m.Bc;
-    e = launch_gather_requests(requests, gather, n_experts, m.b_max, b0, m.Bc, seq_len + 1,
+  if (e == cudaSuccess)
+    e = launch_gather_requests(requests, gather, n_experts, m.b_max, 0, m.b_max, seq_len + 1,
                                grouped, st);
-    if (e != cudaSuccess) break;
+  if (e == cudaSuccess) {
     const TcBuffers tb = carve_tc(m.sweep, sweep_ws);
     e = launch_forward_tc(s, m.sweep.g, tb, status, st);
     if (e == cudaSuccess)
-      e = launch_token_nll_tc(tb, n_experts, m.Bc, seq_len, m.b_max, b0, nll, st);
+      e = launch_token_nll_tc(tb, n_experts, m.b_max, seq_len, m.b_max, 0, nll, st);
   }
   if (e == cudaSuccess)
     e = launch_mixture(nll, route, slot, R, k, seq_len, t0, m.b_max, nll_out, st);

@@ -22,12 +22,22 @@ void trace_end(int kind, cudaStream_t stream);
 // 32-unit tiles of 4 gates; sequences are padded to Bp and P <= 2 probes
 // share one operand group tile of rowsB = 3 Bp P rows (vbar, dhat and
 // eps^2 dhat per probe, forward_tc.cu).
+//
+// The unperturbed layout (inf = 1: evaluation and routed inference, eps = 0,
+// one sign) uses the same tile shape, but the four row blocks that the W
+// product reads hold four blocks of Bp = 32 different sequences, so a group
+// is 128 sequences and every MMA column does useful work; G groups cover
+// the whole batch in one sweep.
 struct TcGeom {
   int E, H, Ep, Hp, S, Sx, Sh, MT, Bp, P, G, rowsB;
   uint32_t tileB;  // bytes of one operand group tile of one stage
   int n_experts, n_pert, B, T;
   int Bm;          // sequences of the whole batch (the loss partials); B <= 64 of them per sweep
+  int inf;         // the unperturbed layout
 };
+
+// Sequences of one group of the unperturbed layout.
+constexpr int kInfGroupSeqs = 128;
 
 struct TcSizes {
   size_t w16, wo16, op, cst, pm, ply, zb;
@@ -45,6 +55,8 @@ struct TcBuffers {
 };
 
 TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem);
+// The unperturbed layout for B sequences per expert (all in one sweep).
+TcGeom make_tc_geom_inf(const Layout& lay, int n_experts, int B, int T);
 // Sequences of one tensor-core sweep; a larger batch runs in chunks of this many.
 constexpr int kTcMaxBatch = 64;
 TcSizes tc_sizes(const TcGeom& g);

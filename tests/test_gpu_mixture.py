@@ -1,6 +1,7 @@
 """Parity of routed inference on the GPU (Sec. 3, Eq. main-mixture) with the
 fp64 oracle: per-target NLL of the mixture of the routed experts, including
-repeated routes, ragged shapes and groups larger than one sweep (64)."""
+repeated routes, ragged shapes and expert groups of more than 128 requests
+(several 128-sequence groups of the unperturbed layout in one sweep)."""
 import numpy as np
 import pytest
 import torch
@@ -34,7 +35,8 @@ def _run(theta, rq, routes, E, H, t0):
 @pytest.mark.parametrize("E,H,N,R,T,k,t0", [
     (32, 64, 8, 40, 20, 3, 5),     # tensor path, one sweep
     (40, 72, 3, 17, 11, 2, 0),     # ragged
-    (16, 48, 2, 100, 6, 2, 2),     # groups of 100: two sweeps per expert
+    (16, 48, 2, 100, 6, 2, 2),     # 100 requests per expert: one partly filled group
+    (16, 80, 2, 300, 7, 2, 3),     # about 300 per expert: three groups, the last ragged
     (32, 48, 256, 64, 12, 4, 4),   # the N=256 expert shape, sparse routing
 ])
 def test_mixture_matches_oracle(oracle_mod, E, H, N, R, T, k, t0):
