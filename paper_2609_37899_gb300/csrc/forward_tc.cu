@@ -119,6 +119,10 @@ __host__ __device__ __forceinline__ int inf_seq(const TcGeom& g, int grp, int bl
 __host__ __device__ __forceinline__ int cst_lanes(const TcGeom& g) {
   return g.inf ? 2 * g.G : g.n_pert;
 }
+template <bool INF>
+__device__ __forceinline__ int cst_lanes_of(const TcGeom& g) {
+  return INF ? 2 * g.G : g.n_pert;
+}
 
 // Shared-memory carve-up of one ring slot.
 struct StageLayout {
@@ -353,6 +357,7 @@ struct Task {
   const uint8_t* b;  // operand group tile of stage 0
 };
 
+template <bool INF>
 __device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
   const TcGeom& g = a.g;
   Task T;
@@ -362,7 +367,7 @@ __device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
   const int rows = T.head ? 2 : g.MT;
   T.m = (j / g.G) % rows;
   T.e = j / (g.G * rows);
-  T.p_valid = g.inf ? g.P : min(g.P, a.sw.n_pert - T.grp * g.P);
+  T.p_valid = INF ? g.P : min(g.P, a.sw.n_pert - T.grp * g.P);
   if (T.head) {
     T.nst = g.Sh;
     T.a = a.wo16 + (((size_t)T.e * 2 + T.m) * g.Sh) * kTileA;
@@ -423,6 +428,7 @@ struct GatePre {
   bool on;
 };
 
+template <bool INF>
 __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int q4, int eg,
                                              GatePre& G) {
   const TcGeom& g = a.g;
@@ -461,7 +467,7 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   }
   const int U = 32 * T.m + 8 * q4 + u8;
   const float2* cell = reinterpret_cast<const float2*>(a.cst) +
-                       (((int64_t)T.e * cst_lanes(g) + i) * g.Hp + U) * (int64_t)g.Bp;
+                       (((int64_t)T.e * cst_lanes_of<INF>(g) + i) * g.Hp + U) * (int64_t)g.Bp;
   const bool load = U < H && a.t_gate > 0;
 #pragma unroll
   for (int j = 0; j < kEpiMaxChunks; ++j) {
@@ -476,6 +482,7 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   }
 }
 
+template <bool INF>
 __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q4,
                             const GatePre& G) {
   if (!G.on) return;
@@ -496,7 +503,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
   const int kk = 32 * T.m % kKt + 8 * q4 + u8;
   const int i = T.grp * g.P + p;
   float2* cell = reinterpret_cast<float2*>(a.cst) +
-                 (((int64_t)T.e * cst_lanes(g) + i) * g.Hp + U) * (int64_t)g.Bp;
+                 (((int64_t)T.e * cst_lanes_of<INF>(g) + i) * g.Hp + U) * (int64_t)g.Bp;
   const uint32_t tq = tacc + ((uint32_t)(32 * q4) << 16);  // gates 0, 1
   const uint32_t tq2 = tq + (16u << 16);                    // gates 2, 3
   const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
@@ -520,7 +527,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       float actp[4], actm[4];
-      if (g.inf) {
+      if constexpr (INF) {
         // unperturbed: the + and - lanes are two blocks' own pre-activations
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -560,7 +567,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
                          rM + b < g.rowsB && kk < kKt,
                      a.status)) {
         cell[b] = make_float2(cp, cm);
-        if (g.inf) {
+        if constexpr (INF) {
           // h of the two blocks into their own rows (the W product's rows)
           if (inf_seq(g, T.grp, col_c(p), b) < s.B)
             *reinterpret_cast<__half*>(out_tile + kmajor_offset(rM + b, kk, kKt)) =
@@ -590,6 +597,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
 // shuffle rounds).  The four quarters of the half merge through shared
 // memory (`red`, [P][Bp][2][4]); the thread holding the target byte's row
 // writes the target logit.
+template <bool INF>
 __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int q4, int ew,
                               float2* red) {
   const TcGeom& g = a.g;
@@ -625,7 +633,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     }
     // perturbed: lanes (e, i, +) and (e, i, -) for sequence b; unperturbed:
     // lane (e, 0, +) for the sequences of blocks col_c(p) and col_d(p)
-    const int64_t lane_plus = g.inf ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2;
+    const int64_t lane_plus = INF ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2;
     const uint32_t cC = (uint32_t)(col_c(p) * g.Bp), cD = (uint32_t)(col_d(p) * g.Bp);
     for (int b0 = 0; b0 < g.Bp; b0 += 4) {
       // [k]: C and D of row r4 + 8 k, sequence b0 + bq
@@ -639,7 +647,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
       float lp[4], lm[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        if (g.inf) {
+        if constexpr (INF) {
           lp[k] = __uint_as_float(vc[k]) + bo[k];
           lm[k] = __uint_as_float(vd[k]) + bo[k];
         } else {
@@ -672,7 +680,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
         red[((p * g.Bp + b) * 2 + 0) * 4 + q4] = make_float2(mp, sp);
         red[((p * g.Bp + b) * 2 + 1) * 4 + q4] = make_float2(mm, sm_);
       }
-      if (g.inf) {
+      if constexpr (INF) {
         // the target logit of each block's sequence, into lane (e, 0, +)
 #pragma unroll
         for (int sg = 0; sg < 2; ++sg) {
@@ -717,7 +725,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     const int pb = idx >> 1;
     const int pp = pb / g.Bp, b = pb % g.Bp;
     // the partials' lane and sequence (see the target logits above)
-    const int qs = g.inf ? inf_seq(g, T.grp, sgn ? col_d(pp) : col_c(pp), b) : b;
+    const int qs = INF ? inf_seq(g, T.grp, sgn ? col_d(pp) : col_c(pp), b) : b;
     if (qs >= s.B) continue;
     const float2* q = red + (size_t)idx * 4;
     const float M = fmaxf(fmaxf(q[0].x, q[1].x), fmaxf(q[2].x, q[3].x));
@@ -725,7 +733,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
 #pragma unroll
     for (int k = 0; k < 4; ++k) S += q[k].y * __expf(q[k].x - M);
     const int i = T.grp * g.P + pp;
-    const int64_t ln = g.inf ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
+    const int64_t ln = INF ? (int64_t)T.e * 2 : ((int64_t)T.e * s.n_pert + i) * 2 + sgn;
     const int64_t o = ((ln * s.B_mem + s.b0 + qs) * (int64_t)s.T + t) * 2 + T.m;
     if (!SOMA_CHECK((size_t)o < a.n_pm, a.status)) continue;
     a.pm[o] = M;
@@ -739,11 +747,13 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
+template <bool INF>
 __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk);
 
 // grid: min(tasks, SMs) persistent CTAs plus the embedding-part blocks of the
 // next timestep's operand, kThreads threads.
-template <bool SPARSE>
+// SPARSE: sparse probes; INF: the unperturbed layout (eps = 0, one sign).
+template <bool SPARSE, bool INF>
 __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
   extern __shared__ uint8_t dyn_smem[];
   const TcGeom& g = a.g;
@@ -751,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   if ((int)blockIdx.x >= n_ctas) {
     // the embedding part of timestep t + 1's operand (the gate tasks write
     // its h part)
-    xpart_block(a, a.op_out, a.t_gate + 1, blockIdx.x - n_ctas);
+    xpart_block<INF>(a, a.op_out, a.t_gate + 1, blockIdx.x - n_ctas);
     return;
   }
   const int n_tasks = a.n_gate + a.n_head;
@@ -793,7 +803,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     uint32_t gs = 0;
     bool done = true;
     for (int task = blockIdx.x; task < n_tasks && done; task += n_ctas) {
-      const Task T = make_task(a, task);
+      const Task T = make_task<INF>(a, task);
       for (int st = 0; st < T.nst; ++st, ++gs) {
         if ((int)(gs % kLoaders) != li) continue;
         const int q = gs % kStages;
@@ -854,7 +864,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       RingPos rp = {0u, 0u};
       int k = 0;
       for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-        const Task T = make_task(a, task);
+        const Task T = make_task<INF>(a, task);
         const int buf = k & 1;
         if (k >= 2 &&
             !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
@@ -897,7 +907,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       uint32_t gs = 0;
       bool alive = true;
       for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
-        const Task T = make_task(a, task);
+        const Task T = make_task<INF>(a, task);
         const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
         // uniform over the warp
         const bool active = pz < T.p_valid &&
@@ -959,17 +969,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     const int q4 = warp & 3;
     int k = 0;
     for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-      const Task T = make_task(a, task);
+      const Task T = make_task<INF>(a, task);
       const int buf = k & 1;
       GatePre G;
       if (!wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status)) break;
-      if (!T.head) gate_prepare(a, T, q4, ew >> 2, G);
+      if (!T.head) gate_prepare<INF>(a, T, q4, ew >> 2, G);
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)buf * kAccCols;
       if (T.head)
-        head_epilogue(a, T, tacc, q4, ew, red);
+        head_epilogue<INF>(a, T, tacc, q4, ew, red);
       else
-        gate_finish(a, T, tacc, q4, G);
+        gate_finish<INF>(a, T, tacc, q4, G);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
@@ -983,6 +993,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
 // Embedding part of the operand of timestep t: per probe p of the group the
 // rows vbar = Emb[byte_t], dhat = z_emb[byte_t] (+-1, or 0) and eps^2 dhat.
 // Block `blk` of Sx * G * N writes one (expert, stage, group) tile.
+template <bool INF>
 __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
@@ -1001,7 +1012,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
     const int i = grp * g.P + p;
     __align__(16) __half v[8];
     const int k0 = kKt * st + 8 * kc;
-    if (g.inf) {
+    if constexpr (INF) {
       // row blocks 1..4: the embeddings of four blocks of sequences; 0, 5: zero
       const int q = blkr >= 1 && blkr <= 4 ? inf_seq(g, grp, blkr - 1, b) : s.B;
       float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -1045,8 +1056,9 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   }
 }
 
+template <bool INF>
 __global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
-  xpart_block(a, op, t, blockIdx.x);
+  xpart_block<INF>(a, op, t, blockIdx.x);
 }
 
 // The probe-word table of one sweep (zbits_row): block b writes the 128 rows
@@ -1354,7 +1366,8 @@ TcSizes tc_sizes(const TcGeom& g) {
 cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& tb, int* status,
                               cudaStream_t stream) {
   const size_t smem = kernel_smem_bytes(g);
-  auto kernel = s.sparse ? tc_persistent_kernel<true> : tc_persistent_kernel<false>;
+  auto kernel = g.inf ? tc_persistent_kernel<false, true>
+                      : s.sparse ? tc_persistent_kernel<true, false> : tc_persistent_kernel<false, false>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
@@ -1393,7 +1406,10 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   cudaMemsetAsync(tb.op[0], 0, z.op, stream);
   cudaMemsetAsync(tb.op[1], 0, z.op, stream);
   const int xblocks = g.n_experts * g.Sx * g.G;
-  xpart_kernel<<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
+  if (g.inf)
+    xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
+  else
+    xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
   if (s.eps != 0.f) {
     const unsigned zblocks = (unsigned)(a.n_zrows / kZRows);
     if (s.sparse)
