@@ -43,11 +43,11 @@ UNIT = "perturbed tokens/s"
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel
 # source it was taken on.
 TRAFFIC = {
-    # profiles/tc_persistent_kernel_soma_n2.md: the gate launch, captured on
-    # the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
-    "soma_n2": {"bytes_per_launch": 64.062720e6 + 5.382400e6,
+    # profiles/tc_persistent_kernel_soma_n2.md: one persistent launch, captured
+    # on the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
+    "soma_n2": {"bytes_per_launch": 148.339968e6 + 35.523072e6,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "91304d8250931a36"},
+                "source_hash": "93404859b197ada1"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
     "soma_n256": {"bytes_per_launch": 39.559168e6 + 2304,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
@@ -467,7 +467,8 @@ def our_arm(args):
             "launches": gate_n,
             "kernel_ms_per_launch": gate_ms / gate_n if gate_n else None,
             "share_of_step": gate_ms / ms if ms else None,
-            "step_frac_burst": (flops_total / K / (ms / 1e3) / 1e12 / peaks["bf16_tflops"])
+            # all K steps' algorithmic flops over the K untraced steps' time
+            "step_frac_burst": (flops_total / (ms / 1e3) / 1e12 / peaks["bf16_tflops"])
                                if ms else None,
         },
         "kernel_ms": {k: v[0] / K for k, v in traced.items()},

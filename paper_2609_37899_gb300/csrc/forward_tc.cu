@@ -58,11 +58,10 @@ using namespace tc;
 namespace {
 
 constexpr int kStages = 4;       // ring slots: shared-memory operands and TMEM probe tiles
-// The bulk-copy instructions of one warp complete one after another (~750
-// cycles each, whatever the size up to 48 KB), while the lanes of one
-// instruction and different warps copy in parallel.  So each stage's two
-// copies are one instruction of two lanes, and the stages rotate over three
-// loader warps.
+// Each stage's two copies (W tile, operand tile) are one 2-lane bulk-copy
+// instruction.  The copies of one warp complete one after another, but
+// more loader warps (stage gs to loader gs % kLoaders) measured no faster:
+// the copies are not what bounds the launch.
 constexpr int kLoaders = 1;
 constexpr int kMmaWarp = 1;
 constexpr int kZWarp0 = 4;       // Z generators: a multiple of 4 (TMEM lane quarters)
@@ -235,16 +234,17 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // tasks (blockIdx.x, blockIdx.x + n_ctas, ...): the gate tasks of timestep
 // t, then the head tasks of t - 1.  Extra blocks (blockIdx.x >= n_ctas)
 // write the embedding part of the next operand.  Roles:
-//   warps 0, 2, 3 loaders: stage gs belongs to loader gs % 3, whose lanes 0
-//                 and 1 bulk-copy its A tile and its operand group tile in
-//                 one instruction;
+//   warp 0        loader (with kLoaders > 1, warps 0, 2, 3, ... take stage
+//                 gs % kLoaders): lanes 0 and 1 bulk-copy the stage's A
+//                 tile and operand group tile in one instruction;
 //   warp 1        MMA issuer (lane 0 alone, so no warp-wide step sits
 //                 between consecutive stages): W x operand (shared memory)
 //                 and Z_p x operand (Z_p in tensor memory) per stage into one
 //                 of two TMEM accumulator buffers;
-//   warps 4..11   Z generators: thread (probe, row) expands Philox words into
-//                 the fp16 +-1 row of its probe tile and stores it into the
-//                 slot's TMEM columns (lane = row);
+//   warps 4..11   Z generators: thread (probe, row) expands the raw probe
+//                 words of the sweep's table into the fp16 +-1 row of its
+//                 probe tile and stores it into the slot's TMEM columns
+//                 (lane = row);
 //   warps 12..19  epilogue: reads a finished accumulator buffer while the
 //                 MMAs of the next task fill the other one; warp w reads the
 //                 TMEM lanes of quarter w % 4 for probe group (w - 12) / 4.
