@@ -49,14 +49,14 @@ TRAFFIC = {
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
                 "source_hash": "93404859b197ada1"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
-    "soma_n256": {"bytes_per_launch": 39.559168e6 + 2304,
+    "soma_n256": {"bytes_per_launch": 39.452672e6 + 2048,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                  "source_hash": "81adb1efd931ba90"},
+                  "source_hash": "7cc9de59fd25da8c"},
     # profiles/body_tc_kernel_body_n256.md: one full-size launch (T=512)
-    "body_n256": {"bytes_per_launch": 36.277248e6,
+    "body_n256": {"bytes_per_launch": 36.546304e6,
                   "files": ["body_tc.cu", "body_device.cuh", "tc_primitives.cuh",
                             "soma_device.cuh"],
-                  "source_hash": "0600bd36a9c58263"},
+                  "source_hash": "aed1fa16ae461890"},
 }
 
 
