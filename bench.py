@@ -116,8 +116,8 @@ def gate_kernel_name(B, resident):
     if resident:
         return ("res_kernel (tcgen05, the whole recurrence of a probe pair resident in one CTA: "
                 "gate GEMM + cell + head + loss)")
-    return ("tc_persistent_kernel (tcgen05; launch t = gate GEMM + fused cell of timestep t "
-            "and output head + softmax partials of t - 1)")
+    return ("tc_persistent_kernel (tcgen05; one cooperative launch per sweep, phase t = "
+            "gate GEMM + fused cell of timestep t and output head + softmax partials of t - 1)")
 
 
 def gate_flops_per_timestep(c):
@@ -426,7 +426,7 @@ def our_arm(args):
     # kernel's traced time: K steps x A estimates x T timesteps, whether a
     # launch covers one timestep (persistent kernel, the head of the previous
     # timestep inside) or all of them (resident kernel)
-    one_launch = traced["head"][1] == 0 and gate_n == K * A  # the resident kernel
+    one_launch = traced["prep"][1] == 0  # the resident kernel: no tile preparation
     flops_total = (gate_flops_per_timestep(c) + head_flops_per_timestep(c)) * T * K * A
     achieved = flops_total / (gate_ms / 1e3) / 1e12 if gate_n else None
     tr = TRAFFIC.get(args.config)

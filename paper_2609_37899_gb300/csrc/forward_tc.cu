@@ -59,10 +59,9 @@ namespace {
 
 constexpr int kStages = 4;       // ring slots: shared-memory operands and TMEM probe tiles
 // Each stage's two copies (W tile, operand tile) are one 2-lane bulk-copy
-// instruction.  The copies of one warp complete one after another, but
-// more loader warps (stage gs to loader gs % kLoaders) measured no faster:
-// the copies are not what bounds the launch.
-constexpr int kLoaders = 1;
+// instruction of one loader warp.  The copies of one warp complete one after
+// another, but more loader warps measured no faster: the copies are not
+// what bounds the launch.
 constexpr int kMmaWarp = 1;
 constexpr int kZWarp0 = 4;       // Z generators: a multiple of 4 (TMEM lane quarters)
 constexpr int kZWarps = 8;       // (probe, lane quarter)
@@ -230,13 +229,14 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 }
 
 // ---------------------------------------------------------------------------
-// Persistent warp-specialised kernel.  One CTA per SM walks a static list of
-// tasks (blockIdx.x, blockIdx.x + n_ctas, ...): the gate tasks of timestep
-// t, then the head tasks of t - 1.  Extra blocks (blockIdx.x >= n_ctas)
-// write the embedding part of the next operand.  Roles:
-//   warp 0        loader (with kLoaders > 1, warps 0, 2, 3, ... take stage
-//                 gs % kLoaders): lanes 0 and 1 bulk-copy the stage's A
-//                 tile and operand group tile in one instruction;
+// Persistent warp-specialised kernel.  One launch runs every phase of a
+// sweep (phase t: the head tasks of timestep t - 1 and the gate tasks of
+// timestep t, see make_task); one CTA per SM walks the phases and, in each,
+// a static list of tasks (blockIdx.x, blockIdx.x + n_ctas, ...).  Phase
+// counters in global memory replace a barrier between phases.  Roles:
+//   warp 0        loader: lanes 0 and 1 bulk-copy the stage's A tile and
+//                 operand group tile in one instruction;
+//   warps 2, 3    the embedding part of the next timestep's operand;
 //   warp 1        MMA issuer (lane 0 alone, so no warp-wide step sits
 //                 between consecutive stages): W x operand (shared memory)
 //                 and Z_p x operand (Z_p in tensor memory) per stage into one
@@ -259,6 +259,7 @@ struct Ctl {
   uint64_t slot_free[kStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
+  uint64_t red_bar;                // the head epilogue's rendezvous
   uint64_t mma_done;
   uint32_t tmem_slot;
   volatile int abort;
@@ -326,13 +327,13 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
 struct TcArgs {
   Sweep sw;
   TcGeom g;
-  int t_gate;            // timestep of the gate tasks, -1: none
-  int t_head;            // timestep of the head tasks, -1: none
-  int n_gate, n_head;    // task counts
+  int t_first, t_last;   // the phases of this launch (phase t: the gate of t, the head of t - 1)
+  int gate_tasks, head_tasks, x_tiles;  // per phase
   const uint8_t* w16;    // [N][MT][S] A tiles
   const uint8_t* wo16;   // [N][2][Sh] A tiles
-  const uint8_t* op_in;  // [N][S][G] operand group tiles: [x_t | h_{t-1}]
-  uint8_t* op_out;       // operand of t + 1
+  uint8_t* op[2];        // [N][S][G] operand group tiles; phase t reads op[t % 2] = [x_t | h_{t-1}]
+  int* prod;             // [N][G] writes finished into a group's operand (see the phase counters)
+  int* hd;               // [N][G] head tasks finished reading a group's operand
   float* cst;            // [N*n][Hp][Bp] cell state (float2: sign +, -)
   float* pm;             // [N*n*2][B_mem][T][2] head max partials
   float* ps;             // sum-exp partials
@@ -347,6 +348,82 @@ struct TcArgs {
   uint32_t smem_bytes;
 };
 
+// One phase t of the sweep: the gate tasks of timestep t (t < T) and the
+// head tasks of timestep t - 1 (t >= 1), both reading op[t % 2], and the
+// embedding-part tiles of timestep t + 1 (t + 1 < T), written into
+// op[(t + 1) % 2] with the gate tasks' h part.
+struct Phase {
+  int t_gate, t_head;    // timesteps, -1: none
+  int n_gate, n_head, n_x;
+  const uint8_t* op_in;
+  uint8_t* op_out;
+};
+
+__device__ __forceinline__ Phase make_phase(const TcArgs& a, int t) {
+  Phase ph;
+  const int T = a.sw.T;
+  ph.t_gate = t < T ? t : -1;
+  ph.t_head = t - 1;
+  ph.n_gate = t < T ? a.gate_tasks : 0;
+  ph.n_head = t >= 1 ? a.head_tasks : 0;
+  ph.n_x = t + 1 < T ? a.x_tiles : 0;
+  ph.op_in = a.op[t & 1];
+  ph.op_out = a.op[(t + 1) & 1];
+  return ph;
+}
+
+// Phase counters.  A launch may run several phases; tasks of phase t + 1
+// start on the groups that phase t has finished, without a grid-wide
+// barrier.  Per (expert, group): prod counts the writes finished into the
+// group's operand (one per epilogue warp of a gate task, one per
+// embedding-part tile), hd the head tasks finished (one per epilogue warp).
+// Through phase t (inclusive):
+__device__ __forceinline__ int prod_target(const TcArgs& a, int t) {
+  if (t < 0) return 0;
+  const int T = a.sw.T;
+  const int gate_phases = min(t, T - 1) + 1;
+  const int x_phases = max(0, min(t, T - 2) + 1);
+  return kEpiWarps * a.g.MT * gate_phases + a.g.Sx * x_phases;
+}
+__device__ __forceinline__ int hd_target(const TcArgs& a, int t) {
+  return t < 1 ? 0 : kEpiWarps * 2 * t;
+}
+
+// Waits (bounded) until *ctr >= target; lane 0 polls for the warp.  The
+// acquire and the cross-proxy fence order the operand data written by other
+// CTAs before this warp's later reads, bulk copies included.
+__device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatile int* abort,
+                                             int* status) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) {
+    uint32_t n = 0;
+    for (;;) {
+      int v;
+      asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+      if (v >= target) break;
+      if (++n >= (1u << 22) || ((n & 63u) == 0 && *abort)) {
+        ok = 0;
+        break;
+      }
+      __nanosleep(64);
+    }
+    if (!ok && n >= (1u << 22)) {
+      *abort = 1;
+      atomicCAS(status, 0, kStatusTimeout);
+    }
+  }
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  return ok != 0;
+}
+
+// The warp's writes so far are visible before the counter moves.
+__device__ __forceinline__ void release_count(int* ctr) {
+  __threadfence();
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) atomicAdd(ctr, 1);
+}
+
 // One task: (expert, row tile, probe group).  For the gate the row tile is
 // 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
 // half.
@@ -357,25 +434,29 @@ struct Task {
   const uint8_t* b;  // operand group tile of stage 0
 };
 
+// A phase's task list: the head tasks first (their operand is complete when
+// the phase starts), then the gate tasks group by group, row tiles fastest,
+// so that the groups of a phase finish one after another and the next
+// phase can start on them while this one completes.
 template <bool INF>
-__device__ __forceinline__ Task make_task(const TcArgs& a, int task) {
+__device__ __forceinline__ Task make_task(const TcArgs& a, const Phase& ph, int task) {
   const TcGeom& g = a.g;
   Task T;
-  T.head = task >= a.n_gate;
-  const int j = T.head ? task - a.n_gate : task;
-  T.grp = j % g.G;
+  T.head = task < ph.n_head;
+  const int j = T.head ? task : task - ph.n_head;
   const int rows = T.head ? 2 : g.MT;
-  T.m = (j / g.G) % rows;
+  T.m = j % rows;
+  T.grp = (j / rows) % g.G;
   T.e = j / (g.G * rows);
   T.p_valid = INF ? g.P : min(g.P, a.sw.n_pert - T.grp * g.P);
   if (T.head) {
     T.nst = g.Sh;
     T.a = a.wo16 + (((size_t)T.e * 2 + T.m) * g.Sh) * kTileA;
-    T.b = a.op_in + (((size_t)T.e * g.S + g.Sx) * g.G + T.grp) * g.tileB;
+    T.b = ph.op_in + (((size_t)T.e * g.S + g.Sx) * g.G + T.grp) * g.tileB;
   } else {
     T.nst = g.S;
     T.a = a.w16 + (((size_t)T.e * g.MT + T.m) * g.S) * kTileA;
-    T.b = a.op_in + (((size_t)T.e * g.S) * g.G + T.grp) * g.tileB;
+    T.b = ph.op_in + (((size_t)T.e * g.S) * g.G + T.grp) * g.tileB;
   }
   return T;
 }
@@ -429,8 +510,8 @@ struct GatePre {
 };
 
 template <bool INF>
-__device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int q4, int eg,
-                                             GatePre& G) {
+__device__ __forceinline__ void gate_prepare(const TcArgs& a, const Phase& ph, const Task& T,
+                                             int q4, int eg, GatePre& G) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
@@ -468,7 +549,7 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
   const int U = 32 * T.m + 8 * q4 + u8;
   const float2* cell = reinterpret_cast<const float2*>(a.cst) +
                        (((int64_t)T.e * cst_lanes_of<INF>(g) + i) * g.Hp + U) * (int64_t)g.Bp;
-  const bool load = U < H && a.t_gate > 0;
+  const bool load = U < H && ph.t_gate > 0;
 #pragma unroll
   for (int j = 0; j < kEpiMaxChunks; ++j) {
     const int b0 = 8 * (G.c0 + j * G.cstep);
@@ -483,8 +564,8 @@ __device__ __forceinline__ void gate_prepare(const TcArgs& a, const Task& T, int
 }
 
 template <bool INF>
-__device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q4,
-                            const GatePre& G) {
+__device__ void gate_finish(const TcArgs& a, const Phase& ph, const Task& T, uint32_t tacc,
+                            int q4, const GatePre& G) {
   if (!G.on) return;
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
@@ -499,7 +580,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
   const bool unit_ok = U < H;
   // a stage of the next operand holds kKt / 32 of the 32-unit row tiles
   uint8_t* out_tile =
-      a.op_out + (((size_t)T.e * g.S + g.Sx + 32 * T.m / kKt) * g.G + T.grp) * g.tileB;
+      ph.op_out + (((size_t)T.e * g.S + g.Sx + 32 * T.m / kKt) * g.G + T.grp) * g.tileB;
   const int kk = 32 * T.m % kKt + 8 * q4 + u8;
   const int i = T.grp * g.P + p;
   float2* cell = reinterpret_cast<float2*>(a.cst) +
@@ -560,7 +641,7 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
       const float hp = actp[3] * fmaf(sigm(2.f * cp), 2.f, -1.f);
       const float hm = actm[3] * fmaf(sigm(2.f * cm), 2.f, -1.f);
       const int b = b0 + 4 * h + bq;
-      const size_t tile_off = (size_t)(out_tile - a.op_out);
+      const size_t tile_off = (size_t)(out_tile - ph.op_out);
       if (unit_ok &&
           SOMA_CHECK((size_t)(cell - reinterpret_cast<float2*>(a.cst) + b + 1) * 2 <= a.n_cst &&
                          tile_off + g.tileB <= a.n_op && rE + b < g.rowsB && rD + b < g.rowsB &&
@@ -597,9 +678,24 @@ __device__ void gate_finish(const TcArgs& a, const Task& T, uint32_t tacc, int q
 // shuffle rounds).  The four quarters of the half merge through shared
 // memory (`red`, [P][Bp][2][4]); the thread holding the target byte's row
 // writes the target logit.
+// Rendezvous of the epilogue warps around the head's reduction buffer: a
+// bounded wait on an mbarrier (count: one arrival per epilogue warp), so a
+// warp that has left after an abort makes the others time out instead of
+// blocking.  *use counts this warp's rendezvous so far.
+__device__ __forceinline__ bool epi_rendezvous(uint64_t* bar, uint32_t* use, volatile int* abort,
+                                               int* status) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+  const bool ok = wait_or_abort(bar, *use & 1u, abort, status);
+  ++*use;
+  __syncwarp();
+  return ok;
+}
+
 template <bool INF>
-__device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int q4, int ew,
-                              float2* red) {
+__device__ bool head_epilogue(const TcArgs& a, const Phase& ph, const Task& T, uint32_t tacc,
+                              int q4, int ew, float2* red, uint64_t* red_bar, uint32_t* red_use,
+                              volatile int* abort) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
@@ -612,7 +708,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
       SOMA_CHECK((size_t)(T.e * L.P + L.b_out + vq + lane) < a.n_params, a.status)
           ? th[L.b_out + vq + lane]
           : 0.f;
-  const int t = a.t_head;
+  const int t = ph.t_head;
   const int bq = lane & 3, r4 = lane >> 2;
   // rows of this thread: vq + r4 + 8 k, k = 0..3 (k = 2 h + reg)
   float bo[4];
@@ -717,7 +813,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     }
   }
   // all epilogue warps: partials of this task are in `red`
-  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+  if (!epi_rendezvous(red_bar, red_use, abort, a.status)) return false;
   const int et = threadIdx.x - kEpiWarp0 * 32;
   const int n_red = T.p_valid * g.Bp * 2;
   for (int idx = et; idx < n_red; idx += kEpiWarps * 32) {
@@ -740,7 +836,7 @@ __device__ void head_epilogue(const TcArgs& a, const Task& T, uint32_t tacc, int
     a.ps[o] = S;
   }
   // `red` is reused by the next task
-  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+  return epi_rendezvous(red_bar, red_use, abort, a.status);
 }
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -748,23 +844,17 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 }
 
 template <bool INF>
-__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk);
+__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int first, int stride);
 
-// grid: min(tasks, SMs) persistent CTAs plus the embedding-part blocks of the
-// next timestep's operand, kThreads threads.
+// grid: n_ctas persistent CTAs (at most one per SM, all resident: the launch
+// is cooperative), kThreads threads.  The CTA runs phases t_first ..
+// t_last; within a phase, CTA b takes tasks b, b + n_ctas, ...
 // SPARSE: sparse probes; INF: the unperturbed layout (eps = 0, one sign).
 template <bool SPARSE, bool INF>
 __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
   extern __shared__ uint8_t dyn_smem[];
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  if ((int)blockIdx.x >= n_ctas) {
-    // the embedding part of timestep t + 1's operand (the gate tasks write
-    // its h part)
-    xpart_block<INF>(a, a.op_out, a.t_gate + 1, blockIdx.x - n_ctas);
-    return;
-  }
-  const int n_tasks = a.n_gate + a.n_head;
   uint8_t* smem = align1024(dyn_smem);
   const StageLayout SL = stage_layout(g);
   Ctl* ctl = reinterpret_cast<Ctl*>(smem + kStages * SL.bytes);
@@ -786,6 +876,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       mbar_init(&ctl->acc_full[q], 1);
       mbar_init(&ctl->acc_empty[q], kEpiWarps);
     }
+    mbar_init(&ctl->red_bar, kEpiWarps);
     mbar_init(&ctl->mma_done, 1);
     mbar_fence_init();
   }
@@ -795,52 +886,65 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   tc_fence_after();
   const uint32_t tmem = ctl->tmem_slot;
 
-  if (warp < kLoaders + (kLoaders > 1 ? 1 : 0) && warp != kMmaWarp) {
-    // --------------------------------------------------------------- loaders
-    // the whole warp walks the stages in order and waits for the slots of
-    // its own stages; lanes 0 and 1 issue the stage's two copies together
-    const int li = warp == 0 ? 0 : warp - 1;  // loader index: warps 0, 2, 3, ...
+  if (warp == 0) {
+    // ---------------------------------------------------------------- loader
+    // the whole warp walks the stages in order and waits for their slots;
+    // lanes 0 and 1 issue the stage's two copies together.  A task of phase
+    // t >= 1 first waits until phase t - 1 has finished writing its group's
+    // operand.
     uint32_t gs = 0;
     bool done = true;
-    for (int task = blockIdx.x; task < n_tasks && done; task += n_ctas) {
-      const Task T = make_task<INF>(a, task);
-      for (int st = 0; st < T.nst; ++st, ++gs) {
-        if ((int)(gs % kLoaders) != li) continue;
-        const int q = gs % kStages;
-        const uint32_t use = gs / kStages;
-        if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
-          done = false;
-          break;
+    for (int t = a.t_first; t <= a.t_last && done; ++t) {
+      const Phase ph = make_phase(a, t);
+      const int n_tasks = ph.n_head + ph.n_gate;
+      for (int task = blockIdx.x; task < n_tasks && done; task += n_ctas) {
+        const Task T = make_task<INF>(a, ph, task);
+        if (t >= 1) {
+          const size_t c = (size_t)T.e * g.G + T.grp;
+          if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
+              !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status)) {
+            done = false;
+            break;
+          }
         }
-        uint8_t* slot = smem + q * SL.bytes;
-        if (lane == 0) mbar_arrive_expect_tx(&ctl->full[q], kTileA + g.tileB);
-        __syncwarp();
-        if (lane < 2) {
-          uint8_t* dst = lane == 0 ? slot + SL.a_off : slot + SL.b_off;
-          const uint8_t* src =
-              lane == 0 ? T.a + (size_t)st * kTileA : T.b + (size_t)st * g.G * g.tileB;
-          const uint32_t nb = lane == 0 ? kTileA : g.tileB;
-          const uint8_t* gbase = lane == 1 ? a.op_in : (T.head ? a.wo16 : a.w16);
-          const size_t gsize = lane == 1 ? a.n_op : (T.head ? a.n_wo16 : a.n_w16);
-          if (SOMA_CHECK((size_t)(dst - dyn_smem) + nb <= a.smem_bytes &&
-                             src >= gbase && (size_t)(src - gbase) + nb <= gsize,
-                         status))
-            bulk_g2s(dst, src, nb, &ctl->full[q]);
+        for (int st = 0; st < T.nst; ++st, ++gs) {
+          const int q = gs % kStages;
+          const uint32_t use = gs / kStages;
+          if (gs >= kStages &&
+              !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
+            done = false;
+            break;
+          }
+          uint8_t* slot = smem + q * SL.bytes;
+          if (lane == 0) mbar_arrive_expect_tx(&ctl->full[q], kTileA + g.tileB);
+          __syncwarp();
+          if (lane < 2) {
+            uint8_t* dst = lane == 0 ? slot + SL.a_off : slot + SL.b_off;
+            const uint8_t* src =
+                lane == 0 ? T.a + (size_t)st * kTileA : T.b + (size_t)st * g.G * g.tileB;
+            const uint32_t nb = lane == 0 ? kTileA : g.tileB;
+            const uint8_t* gbase = lane == 1 ? ph.op_in : (T.head ? a.wo16 : a.w16);
+            const size_t gsize = lane == 1 ? a.n_op : (T.head ? a.n_wo16 : a.n_w16);
+            if (SOMA_CHECK((size_t)(dst - dyn_smem) + nb <= a.smem_bytes &&
+                               src >= gbase && (size_t)(src - gbase) + nb <= gsize,
+                           status))
+              bulk_g2s(dst, src, nb, &ctl->full[q]);
+          }
+          __syncwarp();
         }
-        __syncwarp();
       }
     }
-    // The copies of the last stage of each slot land before the CTA exits;
-    // the loader that issued that stage waits for them (earlier phases of a
-    // slot completed before its later copies were issued).  After an abort
-    // the copies issued so far are not tracked: the slot waits that failed
-    // above were bounded, and copies take microseconds against that bound.
+    // The copies of the last stage of each slot land before the CTA exits
+    // (earlier phases of a slot completed before its later copies were
+    // issued).  After an abort the copies issued so far are not tracked: the
+    // slot waits that failed above were bounded, and copies take
+    // microseconds against that bound.
     if (done) {
 #pragma unroll
       for (int q = 0; q < kStages; ++q) {
         if ((int)gs <= q) continue;
         const uint32_t last = gs - 1 - ((gs - 1 - (uint32_t)q) % kStages);  // last stage of slot q
-        if ((int)(last % kLoaders) == li) mbar_wait(&ctl->full[q], (last / kStages) & 1u);
+        mbar_wait(&ctl->full[q], (last / kStages) & 1u);
       }
     }
   } else if (warp == kMmaWarp) {
@@ -863,36 +967,64 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const uint32_t dz1 = (uint32_t)(2 * g.Bp);
       RingPos rp = {0u, 0u};
       int k = 0;
-      for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-        const Task T = make_task<INF>(a, task);
-        const int buf = k & 1;
-        if (k >= 2 &&
-            !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
-          break;
-        tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)buf * kAccCols;
-        const int np = do_z ? T.p_valid : 0;
-        bool ok;
-        if (np == 2)
-          ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
-                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
-                           status);
-        else if (np == 1)
-          ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
-                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
-                           status);
-        else
-          ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0,
-                           b_lo0, slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort,
-                           status);
-        if (!ok) break;
-        mma_commit(&ctl->acc_full[buf]);
+      bool ok = true;
+      for (int t = a.t_first; t <= a.t_last && ok; ++t) {
+        const Phase ph = make_phase(a, t);
+        const int n_tasks = ph.n_head + ph.n_gate;
+        for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
+          const Task T = make_task<INF>(a, ph, task);
+          const int buf = k & 1;
+          if (k >= 2 &&
+              !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort,
+                             status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)buf * kAccCols;
+          const int np = do_z ? T.p_valid : 0;
+          if (np == 2)
+            ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+          else if (np == 1)
+            ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+          else
+            ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+          if (!ok) break;
+          mma_commit(&ctl->acc_full[buf]);
+        }
       }
       // every MMA of this CTA completes before its tensor memory is freed
       mma_commit(&ctl->mma_done);
       mbar_wait(&ctl->mma_done, 0);
     }
     __syncwarp();
+  } else if (warp == 2 || warp == 3) {
+    // ------------------------------------------------- embedding-part tiles
+    // Tile j of phase t (the x part of op[(t + 1) % 2] for one (expert,
+    // stage, group)) belongs to CTA j % n_ctas, warp 2 + (j / n_ctas) % 2.
+    // It overwrites what phase t - 1 read: it waits until that phase's gate
+    // and head tasks of the group have finished.
+    bool alive = true;
+    for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+      const Phase ph = make_phase(a, t);
+      int i = 0;
+      for (int j = blockIdx.x; j < ph.n_x; j += n_ctas, ++i) {
+        if ((i & 1) != warp - 2) continue;
+        const int grp = j % g.G, e = j / (g.G * g.Sx);
+        const size_t c = (size_t)e * g.G + grp;
+        if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
+            !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
+            !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status)) {
+          alive = false;
+          break;
+        }
+        xpart_block<INF>(a, ph.op_out, t + 1, j, lane, 32);
+        release_count(a.prod + c);
+      }
+    }
   } else if (warp >= kZWarp0 && warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
     // Thread (probe gtid / 128, row gtid % 128 = TMEM lane).  The raw probe
@@ -906,83 +1038,108 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kZCol0 + 32u * pz;
       uint32_t gs = 0;
       bool alive = true;
-      for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
-        const Task T = make_task<INF>(a, task);
-        const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
-        // uniform over the warp
-        const bool active = pz < T.p_valid &&
-                            SOMA_CHECK(row0 + (size_t)kZRows * (T.nst - 1) < a.n_zrows, status);
-        const uint2* zn = a.zb + row0;
-        const uint2* za = a.zb + a.n_zrows + row0;
-        const uint2 none = make_uint2(0u, 0u);
-        // raw words (and activity words) of stages st + 1 and st + 2
-        uint2 n1 = none, n2 = none, a1 = none, a2 = none;
-        uint32_t zw[kKt / 2];
-        if (active) {
-          const uint2 n0 = __ldg(zn);
-          const uint2 a0 = SPARSE ? __ldg(za) : none;
-          if (T.nst > 1) {
-            n1 = __ldg(zn + kZRows);
-            if (SPARSE) a1 = __ldg(za + kZRows);
-          }
-          if (T.nst > 2) {
-            n2 = __ldg(zn + 2 * kZRows);
-            if (SPARSE) a2 = __ldg(za + 2 * kZRows);
-          }
-          z_run_pairs<SPARSE>(n0.x, a0.x, zw);
-          z_run_pairs<SPARSE>(n0.y, a0.y, zw + 16);
-        }
-        for (int st = 0; st < T.nst; ++st, ++gs) {
-          const int q = gs % kStages;
-          const uint32_t use = gs / kStages;
-          // after an abort the generators stop: an arrival on a phase that
-          // can no longer complete would overfill it
-          if (gs >= kStages && !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
-            alive = false;
-            break;
-          }
-          tc_fence_after();
-          if (active &&
-              SOMA_CHECK(kZCol0 + 64u * (uint32_t)q + 32u * pz + 32u <= kTmemCols, status)) {
-            tmem_st32(trow + 64u * (uint32_t)q, zw);
-            if (st + 1 < T.nst) {
-              z_run_pairs<SPARSE>(n1.x, a1.x, zw);
-              z_run_pairs<SPARSE>(n1.y, a1.y, zw + 16);
-              n1 = n2;
-              a1 = a2;
-              if (st + 3 < T.nst) {
-                n2 = __ldg(zn + (size_t)kZRows * (st + 3));
-                if (SPARSE) a2 = __ldg(za + (size_t)kZRows * (st + 3));
-              }
+      for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+        const Phase ph = make_phase(a, t);
+        const int n_tasks = ph.n_head + ph.n_gate;
+        for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
+          const Task T = make_task<INF>(a, ph, task);
+          const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
+          // uniform over the warp
+          const bool active =
+              pz < T.p_valid &&
+              SOMA_CHECK(row0 + (size_t)kZRows * (T.nst - 1) < a.n_zrows, status);
+          const uint2* zn = a.zb + row0;
+          const uint2* za = a.zb + a.n_zrows + row0;
+          const uint2 none = make_uint2(0u, 0u);
+          // raw words (and activity words) of stages st + 1 and st + 2
+          uint2 n1 = none, n2 = none, a1 = none, a2 = none;
+          uint32_t zw[kKt / 2];
+          if (active) {
+            const uint2 n0 = __ldg(zn);
+            const uint2 a0 = SPARSE ? __ldg(za) : none;
+            if (T.nst > 1) {
+              n1 = __ldg(zn + kZRows);
+              if (SPARSE) a1 = __ldg(za + kZRows);
             }
-            tmem_wait_st();
+            if (T.nst > 2) {
+              n2 = __ldg(zn + 2 * kZRows);
+              if (SPARSE) a2 = __ldg(za + 2 * kZRows);
+            }
+            z_run_pairs<SPARSE>(n0.x, a0.x, zw);
+            z_run_pairs<SPARSE>(n0.y, a0.y, zw + 16);
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&ctl->full[q]);
+          for (int st = 0; st < T.nst; ++st, ++gs) {
+            const int q = gs % kStages;
+            const uint32_t use = gs / kStages;
+            // after an abort the generators stop: an arrival on a phase that
+            // can no longer complete would overfill it
+            if (gs >= kStages &&
+                !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
+              alive = false;
+              break;
+            }
+            tc_fence_after();
+            if (active &&
+                SOMA_CHECK(kZCol0 + 64u * (uint32_t)q + 32u * pz + 32u <= kTmemCols, status)) {
+              tmem_st32(trow + 64u * (uint32_t)q, zw);
+              if (st + 1 < T.nst) {
+                z_run_pairs<SPARSE>(n1.x, a1.x, zw);
+                z_run_pairs<SPARSE>(n1.y, a1.y, zw + 16);
+                n1 = n2;
+                a1 = a2;
+                if (st + 3 < T.nst) {
+                  n2 = __ldg(zn + (size_t)kZRows * (st + 3));
+                  if (SPARSE) a2 = __ldg(za + (size_t)kZRows * (st + 3));
+                }
+              }
+              tmem_wait_st();
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctl->full[q]);
+          }
         }
       }
     }
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
+    // A gate task of phase t overwrites what the head tasks of phase t - 1
+    // read (op[(t + 1) % 2]): it waits for them before its first write.
+    // After each task the warp publishes its writes on the group's counter.
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
     int k = 0;
-    for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-      const Task T = make_task<INF>(a, task);
-      const int buf = k & 1;
-      GatePre G;
-      if (!wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status)) break;
-      if (!T.head) gate_prepare<INF>(a, T, q4, ew >> 2, G);
-      tc_fence_after();
-      const uint32_t tacc = tmem + (uint32_t)buf * kAccCols;
-      if (T.head)
-        head_epilogue<INF>(a, T, tacc, q4, ew, red);
-      else
-        gate_finish<INF>(a, T, tacc, q4, G);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
+    uint32_t red_use = 0;
+    bool alive = true;
+    for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+      const Phase ph = make_phase(a, t);
+      const int n_tasks = ph.n_head + ph.n_gate;
+      for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
+        const Task T = make_task<INF>(a, ph, task);
+        const int buf = k & 1;
+        const size_t c = (size_t)T.e * g.G + T.grp;
+        GatePre G;
+        if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
+            !wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status) ||
+            (!T.head && !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status))) {
+          alive = false;
+          break;
+        }
+        if (!T.head) gate_prepare<INF>(a, ph, T, q4, ew >> 2, G);
+        tc_fence_after();
+        const uint32_t tacc = tmem + (uint32_t)buf * kAccCols;
+        if (T.head) {
+          if (!head_epilogue<INF>(a, ph, T, tacc, q4, ew, red, &ctl->red_bar, &red_use, abort)) {
+            alive = false;
+            break;
+          }
+        } else {
+          gate_finish<INF>(a, ph, T, tacc, q4, G);
+        }
+        tc_fence_before();
+        release_count(T.head ? a.hd + c : a.prod + c);
+        if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
+      }
     }
   }
   tc_fence_before();
@@ -994,7 +1151,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
 // rows vbar = Emb[byte_t], dhat = z_emb[byte_t] (+-1, or 0) and eps^2 dhat.
 // Block `blk` of Sx * G * N writes one (expert, stage, group) tile.
 template <bool INF>
-__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
+__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int first, int stride) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const int st = (blk / g.G) % g.Sx, grp = blk % g.G;
@@ -1004,7 +1161,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
   const float eps2 = s.eps * s.eps;
   uint8_t* tile = op + (((size_t)e * g.S + st) * g.G + grp) * g.tileB;
   const int chunks = g.rowsB * (kKt / 8);
-  for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+  for (int c = first; c < chunks; c += stride) {
     const int row = c / (kKt / 8), kc = c % (kKt / 8);
     const int blkr = row / g.Bp, b = row % g.Bp;  // row block 0..3P-1, sequence
     const int p = blkr < 3 ? 0 : 1;
@@ -1058,7 +1215,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk) {
 
 template <bool INF>
 __global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
-  xpart_block<INF>(a, op, t, blockIdx.x);
+  xpart_block<INF>(a, op, t, blockIdx.x, threadIdx.x, blockDim.x);
 }
 
 // The probe-word table of one sweep (zbits_row): block b writes the 128 rows
@@ -1360,6 +1517,8 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.ply = N * n * 2 * g.Bm * (size_t)g.T * sizeof(float);
   // raw words and activity words
   z.zb = 2 * N * n * (size_t)zbits_stages(g) * kZRows * sizeof(uint2);
+  // phase counters: prod and hd per (expert, group)
+  z.cnt = 2 * N * (size_t)g.G * sizeof(int);
   return z;
 }
 
@@ -1384,10 +1543,6 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.zb = tb.zbits;
   a.n_zrows = (size_t)g.n_experts * g.n_pert * zbits_stages(g) * kZRows;
   a.status = status;
-  a.t_gate = -1;
-  a.t_head = -1;
-  a.n_gate = 0;
-  a.n_head = 0;
   a.n_w16 = z.w16;
   a.n_wo16 = z.wo16;
   a.n_op = z.op;
@@ -1398,13 +1553,21 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.n_ply = z.ply / sizeof(float);
   a.n_params = (size_t)s.n_experts * s.lay.P;
   a.smem_bytes = (uint32_t)smem;
-  a.op_in = tb.op[0];
-  a.op_out = tb.op[0];
+  a.op[0] = tb.op[0];
+  a.op[1] = tb.op[1];
+  a.prod = tb.cnt;
+  a.hd = tb.cnt + (size_t)g.n_experts * g.G;
+  a.gate_tasks = g.n_experts * g.MT * g.G;
+  a.head_tasks = g.n_experts * 2 * g.G;
+  a.x_tiles = g.n_experts * g.Sx * g.G;
+  a.t_first = 0;
+  a.t_last = s.T;
 
   trace_begin(SOMA_TRACE_PREP, stream);
   prep_tiles_kernel<<<dim3(g.MT * g.S + 2 * g.Sh, g.n_experts), 128, 0, stream>>>(a);
   cudaMemsetAsync(tb.op[0], 0, z.op, stream);
   cudaMemsetAsync(tb.op[1], 0, z.op, stream);
+  cudaMemsetAsync(tb.cnt, 0, z.cnt, stream);
   const int xblocks = g.n_experts * g.Sx * g.G;
   if (g.inf)
     xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
@@ -1419,25 +1582,29 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   }
   trace_end(SOMA_TRACE_PREP, stream);
 
+  // every phase of the sweep in one cooperative launch: its CTAs wait on
+  // each other's phase counters, so all of them must be resident together
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) return cudaErrorLaunchOutOfResources;
   const int sms = sm_count();
-  const int gate_tasks = g.n_experts * g.MT * g.G;
-  const int head_tasks = g.n_experts * 2 * g.G;
-  // launch t: the gate of t (t < T) and the head of t - 1 (t >= 1), both
-  // reading the operand [x_t | h_{t-1}]
-  for (int t = 0; t <= s.T; ++t) {
-    a.t_gate = t < s.T ? t : -1;
-    a.t_head = t - 1;
-    a.n_gate = t < s.T ? gate_tasks : 0;
-    a.n_head = t >= 1 ? head_tasks : 0;
-    a.op_in = tb.op[t & 1];
-    a.op_out = tb.op[(t + 1) & 1];
-    const int tasks = a.n_gate + a.n_head;
-    const int ctas = tasks < sms ? tasks : sms;
-    const int extra = t + 1 < s.T ? xblocks : 0;
-    trace_begin(SOMA_TRACE_GATE, stream);
-    kernel<<<ctas + extra, kThreads, smem, stream>>>(a, ctas);
-    trace_end(SOMA_TRACE_GATE, stream);
-  }
+  const int tasks = a.gate_tasks + a.head_tasks;
+  const int ctas = tasks < sms ? tasks : sms;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  trace_begin(SOMA_TRACE_GATE, stream);
+  e = cudaLaunchKernelEx(&cfg, kernel, a, ctas);
+  trace_end(SOMA_TRACE_GATE, stream);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -137,7 +137,7 @@ struct WsPlan {
   bool res;    // the resident small-expert kernel: no scratch but the coefficients
   TcGeom g;    // geometry of the largest chunk
   TcSizes z;   // buffer sizes: the largest chunk's operand and cell buffers
-  Regions r;   // w16, wo16, op[0], op[1], cst, pm, ps, ply, zbits, coef; or coef alone
+  Regions r;   // w16, wo16, op[0], op[1], cst, pm, ps, ply, zbits, cnt, coef; or coef alone
   size_t total;
 };
 
@@ -170,9 +170,10 @@ WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int
     const TcSizes zl = tc_sizes(make_tc_geom(lay, n_experts, n_pert, last, T, B));
     if (zl.op > w.z.op) w.z.op = zl.op;
     if (zl.cst > w.z.cst) w.z.cst = zl.cst;
+    if (zl.cnt > w.z.cnt) w.z.cnt = zl.cnt;
   }
   for (size_t bytes :
-       {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, coef})
+       {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, w.z.cnt, coef})
     w.r.add(bytes);
   w.total = w.r.total();
   return w;
@@ -190,6 +191,7 @@ TcBuffers carve_tc(const WsPlan& w, void* ws) {
   tb.ps = reinterpret_cast<float*>(p + w.r.off[6]);
   tb.ply = reinterpret_cast<float*>(p + w.r.off[7]);
   tb.zbits = reinterpret_cast<uint2*>(p + w.r.off[8]);
+  tb.cnt = reinterpret_cast<int*>(p + w.r.off[9]);
   return tb;
 }
 

@@ -40,7 +40,7 @@ struct TcGeom {
 constexpr int kInfGroupSeqs = 128;
 
 struct TcSizes {
-  size_t w16, wo16, op, cst, pm, ply, zb;
+  size_t w16, wo16, op, cst, pm, ply, zb, cnt;
 };
 
 struct TcBuffers {
@@ -52,6 +52,7 @@ struct TcBuffers {
   float* ps;       // head partial sum-exp
   float* ply;      // target logits
   uint2* zbits;    // probe-word table of the sweep
+  int* cnt;        // phase counters of the persistent kernel
 };
 
 TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem);
