@@ -1103,9 +1103,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     }
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
-    // A gate task of phase t overwrites what the head tasks of phase t - 1
-    // read (op[(t + 1) % 2]): it waits for them before its first write.
-    // After each task the warp publishes its writes on the group's counter.
+    // A gate task of phase t overwrites what phase t - 1 read (op[(t + 1) %
+    // 2]) and reads the cell states that phase t - 1 wrote, possibly in
+    // another CTA (the task lists of phase 0 and the later phases differ):
+    // it waits for that phase's group before its first access.  After each
+    // task the warp publishes its writes on the group's counter.
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
     int k = 0;
@@ -1119,9 +1121,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         const int buf = k & 1;
         const size_t c = (size_t)T.e * g.G + T.grp;
         GatePre G;
+        // a gate task reads cell states and overwrites operand rows that
+        // other CTAs wrote or read in phase t - 1: the warp acquires both
+        // of the group's counters itself (the loader already waited for the
+        // first, so that wait is one load)
         if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
             !wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status) ||
-            (!T.head && !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status))) {
+            (!T.head && (!wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
+                         !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status)))) {
           alive = false;
           break;
         }
