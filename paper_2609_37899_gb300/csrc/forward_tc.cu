@@ -70,6 +70,7 @@ constexpr int kEpiWarps = 8;     // (probe, lane quarter)
 constexpr int kEpiProbeStep = kEpiWarps / 4;  // head: warp group eg runs probes eg, eg + 2, ...
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 static_assert(kZWarp0 % 4 == 0 && kEpiWarp0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
+constexpr int kTaskSlots = 4;               // tasks a CTA's loader publishes ahead of the others
 constexpr int kKt = 64;                     // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
 constexpr uint32_t kSbo = kKt * 16;         // bytes between 8-row groups
@@ -231,9 +232,12 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // ---------------------------------------------------------------------------
 // Persistent warp-specialised kernel.  One launch runs every phase of a
 // sweep (phase t: the head tasks of timestep t - 1 and the gate tasks of
-// timestep t, see make_task); one CTA per SM walks the phases and, in each,
-// a static list of tasks (blockIdx.x, blockIdx.x + n_ctas, ...).  Phase
-// counters in global memory replace a barrier between phases.  Roles:
+// timestep t, see make_task); one CTA per SM takes tasks in global order
+// (phase by phase, decode_task) from a counter in global memory, so the
+// tasks whose inputs are ready first run first wherever an SM is free.  Its
+// loader publishes each task to the CTA's other roles through a small ring
+// of slots.  Phase counters in global memory replace a barrier between
+// phases.  Roles:
 //   warp 0        loader: lanes 0 and 1 bulk-copy the stage's A tile and
 //                 operand group tile in one instruction;
 //   warps 2, 3    the embedding part of the next timestep's operand;
@@ -261,6 +265,9 @@ struct Ctl {
   uint64_t acc_empty[2];
   uint64_t red_bar;                // the head epilogue's rendezvous
   uint64_t mma_done;
+  uint64_t task_full[kTaskSlots];  // the loader published the slot's task
+  uint64_t task_empty[kTaskSlots]; // every other role has read it
+  int task_gid[kTaskSlots];        // global task index, -1: no more tasks
   uint32_t tmem_slot;
   volatile int abort;
 };
@@ -334,6 +341,8 @@ struct TcArgs {
   uint8_t* op[2];        // [N][S][G] operand group tiles; phase t reads op[t % 2] = [x_t | h_{t-1}]
   int* prod;             // [N][G] writes finished into a group's operand (see the phase counters)
   int* hd;               // [N][G] head tasks finished reading a group's operand
+  int* next_task;        // the next global task index to hand out
+  int total_tasks;       // over all phases
   float* cst;            // [N*n][Hp][Bp] cell state (float2: sign +, -)
   float* pm;             // [N*n*2][B_mem][T][2] head max partials
   float* ps;             // sum-exp partials
@@ -370,6 +379,40 @@ __device__ __forceinline__ Phase make_phase(const TcArgs& a, int t) {
   ph.op_in = a.op[t & 1];
   ph.op_out = a.op[(t + 1) & 1];
   return ph;
+}
+
+// Global task index -> (phase, task of the phase): phase 0 has the gate
+// tasks only, phases 1 .. T - 1 both kinds, phase T the head tasks only.
+__device__ __forceinline__ void decode_task(const TcArgs& a, int gid, int& t, int& task) {
+  const int both = a.gate_tasks + a.head_tasks;
+  if (gid < a.gate_tasks) {
+    t = 0;
+    task = gid;
+    return;
+  }
+  gid -= a.gate_tasks;
+  const int mid = (a.sw.T - 1) * both;
+  if (gid < mid) {
+    t = 1 + gid / both;
+    task = gid % both;
+  } else {
+    t = a.sw.T;
+    task = gid - mid;
+  }
+}
+
+// The consumer side of the task ring: waits for the next published task,
+// reads it and releases the slot (one arrival per warp).  Returns the global
+// task index, -1 at the end, -2 after an abort.
+__device__ __forceinline__ int next_task(uint64_t* full, uint64_t* empty, const int* gids,
+                                         uint32_t& kt, volatile int* abort, int* status) {
+  const int sl = (int)(kt % kTaskSlots);
+  if (!wait_or_abort(&full[sl], (kt / kTaskSlots) & 1u, abort, status)) return -2;
+  const int gid = *reinterpret_cast<const volatile int*>(&gids[sl]);
+  __syncwarp(__activemask());
+  if ((threadIdx.x & 31) == 0) mbar_arrive(&empty[sl]);
+  ++kt;
+  return gid;
 }
 
 // Phase counters.  A launch may run several phases; tasks of phase t + 1
@@ -434,20 +477,22 @@ struct Task {
   const uint8_t* b;  // operand group tile of stage 0
 };
 
-// A phase's task list: the head tasks first (their operand is complete when
-// the phase starts), then the gate tasks group by group, row tiles fastest,
-// so that the groups of a phase finish one after another and the next
-// phase can start on them while this one completes.
+// A phase's task list runs group by group ((expert, probe group), in
+// order): the group's two head tasks, then its gate tasks (row tiles
+// fastest).  The CTAs take tasks in global order (phase by phase, see
+// decode_task), so the groups of a phase finish one after another and the
+// next phase's tasks of a group become ready in the same order.
 template <bool INF>
 __device__ __forceinline__ Task make_task(const TcArgs& a, const Phase& ph, int task) {
   const TcGeom& g = a.g;
   Task T;
-  T.head = task < ph.n_head;
-  const int j = T.head ? task : task - ph.n_head;
-  const int rows = T.head ? 2 : g.MT;
-  T.m = j % rows;
-  T.grp = (j / rows) % g.G;
-  T.e = j / (g.G * rows);
+  const int hb = ph.n_head > 0 ? 2 : 0;
+  const int per = hb + (ph.n_gate > 0 ? g.MT : 0);
+  const int block = task / per, w = task % per;
+  T.head = w < hb;
+  T.m = T.head ? w : w - hb;
+  T.grp = block % g.G;
+  T.e = block / g.G;
   T.p_valid = INF ? g.P : min(g.P, a.sw.n_pert - T.grp * g.P);
   if (T.head) {
     T.nst = g.Sh;
@@ -847,8 +892,9 @@ template <bool INF>
 __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int first, int stride);
 
 // grid: n_ctas persistent CTAs (at most one per SM, all resident: the launch
-// is cooperative), kThreads threads.  The CTA runs phases t_first ..
-// t_last; within a phase, CTA b takes tasks b, b + n_ctas, ...
+// is cooperative), kThreads threads.  The CTAs share the tasks of phases
+// 0 .. T through the task counter; the embedding-part tiles of phases
+// t_first .. t_last are dealt statically.
 // SPARSE: sparse probes; INF: the unperturbed layout (eps = 0, one sign).
 template <bool SPARSE, bool INF>
 __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
@@ -878,6 +924,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     }
     mbar_init(&ctl->red_bar, kEpiWarps);
     mbar_init(&ctl->mma_done, 1);
+    for (int q = 0; q < kTaskSlots; ++q) {
+      mbar_init(&ctl->task_full[q], 1);
+      // the MMA issuer, the Z warps (when probes are generated) and the
+      // epilogue warps read every task
+      mbar_init(&ctl->task_empty[q], 1 + (do_z ? kZWarps : 0) + kEpiWarps);
+    }
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(&ctl->tmem_slot, kTmemCols);
@@ -892,12 +944,30 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // lanes 0 and 1 issue the stage's two copies together.  A task of phase
     // t >= 1 first waits until phase t - 1 has finished writing its group's
     // operand.
-    uint32_t gs = 0;
+    uint32_t gs = 0, kt = 0;
     bool done = true;
-    for (int t = a.t_first; t <= a.t_last && done; ++t) {
+    for (;;) {
+      // take the next task in global order and publish it to the other roles
+      const int sl = (int)(kt % kTaskSlots);
+      if (kt >= kTaskSlots &&
+          !wait_or_abort(&ctl->task_empty[sl], ((kt / kTaskSlots) - 1) & 1u, abort, status)) {
+        done = false;
+        break;
+      }
+      int gid = 0;
+      if (lane == 0) gid = atomicAdd(a.next_task, 1);
+      gid = __shfl_sync(0xffffffffu, gid, 0);
+      const bool end = gid >= a.total_tasks;
+      if (lane == 0) {
+        ctl->task_gid[sl] = end ? -1 : gid;
+        mbar_arrive(&ctl->task_full[sl]);
+      }
+      ++kt;
+      if (end) break;
+      int t, task;
+      decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
-      const int n_tasks = ph.n_head + ph.n_gate;
-      for (int task = blockIdx.x; task < n_tasks && done; task += n_ctas) {
+      {
         const Task T = make_task<INF>(a, ph, task);
         if (t >= 1) {
           const size_t c = (size_t)T.e * g.G + T.grp;
@@ -932,6 +1002,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           }
           __syncwarp();
         }
+        if (!done) break;
       }
     }
     // The copies of the last stage of each slot land before the CTA exits
@@ -966,35 +1037,34 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const uint32_t z1_row = (uint32_t)(4 * g.Bp / 8) * grp_step;
       const uint32_t dz1 = (uint32_t)(2 * g.Bp);
       RingPos rp = {0u, 0u};
-      int k = 0;
-      bool ok = true;
-      for (int t = a.t_first; t <= a.t_last && ok; ++t) {
+      uint32_t kt = 0;
+      for (int k = 0;; ++k) {
+        const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
+                                  status);
+        if (gid < 0) break;
+        int t, task;
+        decode_task(a, gid, t, task);
         const Phase ph = make_phase(a, t);
-        const int n_tasks = ph.n_head + ph.n_gate;
-        for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
-          const Task T = make_task<INF>(a, ph, task);
-          const int buf = k & 1;
-          if (k >= 2 &&
-              !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort,
-                             status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)buf * kAccCols;
-          const int np = do_z ? T.p_valid : 0;
-          if (np == 2)
-            ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
-                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
-          else if (np == 1)
-            ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
-                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
-          else
-            ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
-                             slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
-          if (!ok) break;
-          mma_commit(&ctl->acc_full[buf]);
-        }
+        const Task T = make_task<INF>(a, ph, task);
+        const int buf = k & 1;
+        if (k >= 2 &&
+            !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
+          break;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)buf * kAccCols;
+        const int np = do_z ? T.p_valid : 0;
+        bool ok;
+        if (np == 2)
+          ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                           slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+        else if (np == 1)
+          ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                           slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+        else
+          ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+                           slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
+        if (!ok) break;
+        mma_commit(&ctl->acc_full[buf]);
       }
       // every MMA of this CTA completes before its tensor memory is freed
       mma_commit(&ctl->mma_done);
@@ -1036,12 +1106,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const int gtid = tid - kZWarp0 * 32;
       const int r = gtid & 127, pz = gtid >> 7;
       const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kZCol0 + 32u * pz;
-      uint32_t gs = 0;
+      uint32_t gs = 0, kt = 0;
       bool alive = true;
-      for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+      while (alive) {
+        const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
+                                  status);
+        if (gid < 0) break;
+        int t, task;
+        decode_task(a, gid, t, task);
         const Phase ph = make_phase(a, t);
-        const int n_tasks = ph.n_head + ph.n_gate;
-        for (int task = blockIdx.x; task < n_tasks && alive; task += n_ctas) {
+        {
           const Task T = make_task<INF>(a, ph, task);
           const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
           // uniform over the warp
@@ -1113,10 +1187,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     int k = 0;
     uint32_t red_use = 0;
     bool alive = true;
-    for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+    uint32_t kt = 0;
+    for (; alive; ++k) {
+      const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
+                                status);
+      if (gid < 0) break;
+      int t, task;
+      decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
-      const int n_tasks = ph.n_head + ph.n_gate;
-      for (int task = blockIdx.x; task < n_tasks; task += n_ctas, ++k) {
+      {
         const Task T = make_task<INF>(a, ph, task);
         const int buf = k & 1;
         const size_t c = (size_t)T.e * g.G + T.grp;
@@ -1524,8 +1603,8 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.ply = N * n * 2 * g.Bm * (size_t)g.T * sizeof(float);
   // raw words and activity words
   z.zb = 2 * N * n * (size_t)zbits_stages(g) * kZRows * sizeof(uint2);
-  // phase counters: prod and hd per (expert, group)
-  z.cnt = 2 * N * (size_t)g.G * sizeof(int);
+  // phase counters: prod and hd per (expert, group), then the task counter
+  z.cnt = (2 * N * (size_t)g.G + 1) * sizeof(int);
   return z;
 }
 
@@ -1564,11 +1643,13 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.op[1] = tb.op[1];
   a.prod = tb.cnt;
   a.hd = tb.cnt + (size_t)g.n_experts * g.G;
+  a.next_task = tb.cnt + 2 * (size_t)g.n_experts * g.G;
   a.gate_tasks = g.n_experts * g.MT * g.G;
   a.head_tasks = g.n_experts * 2 * g.G;
   a.x_tiles = g.n_experts * g.Sx * g.G;
   a.t_first = 0;
   a.t_last = s.T;
+  a.total_tasks = (a.gate_tasks + a.head_tasks) * s.T;
 
   trace_begin(SOMA_TRACE_PREP, stream);
   prep_tiles_kernel<<<dim3(g.MT * g.S + 2 * g.Sh, g.n_experts), 128, 0, stream>>>(a);
