@@ -29,6 +29,7 @@ import re
 import statistics
 import subprocess
 import sys
+import threading
 import time
 
 import numpy as np
@@ -43,11 +44,12 @@ UNIT = "perturbed tokens/s"
 # (dram__bytes_read.sum + dram__bytes_write.sum), valid only for the kernel
 # source it was taken on.
 TRAFFIC = {
-    # profiles/tc_persistent_kernel_soma_n2.md: one persistent launch, captured
-    # on the SOMA N=2 shapes at T=4 (per-launch traffic does not depend on T)
-    "soma_n2": {"bytes_per_launch": 148.339968e6 + 35.523072e6,
+    # profiles/tc_persistent_kernel_soma_n2.md: one persistent launch of the
+    # SOMA N=2 shapes at T=16 (17 phases) captured; per phase, scaled by the
+    # T + 1 phases of a launch
+    "soma_n2": {"bytes_per_phase": (2185.802e6 + 894.527488e6) / 17,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "93404859b197ada1"},
+                "source_hash": "56d8590b943a4ad9"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
     "soma_n256": {"bytes_per_launch": 39.452672e6 + 2048,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
@@ -63,7 +65,7 @@ TRAFFIC = {
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default="soma_n2")
     ap.add_argument("--seq-len", type=int, default=None,
@@ -169,7 +171,9 @@ def measured_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons every 200 ms while running."""
+    """nvidia-smi clocks and throttle reasons every 50 ms while running.  The
+    sampler is started and its first sample awaited before the timed region,
+    and only the samples taken after that count."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -178,27 +182,41 @@ class ClockSampler:
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
+        self.lines = []
+
+    def _read(self):
+        for line in self.proc.stdout:
+            if line.strip():
+                self._all.append((time.monotonic(), line))
+                self._first.set()
 
     def __enter__(self):
+        self._all = []
+        self._first = threading.Event()
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+            return self
+        self._reader = threading.Thread(target=self._read, daemon=True)
+        self._reader.start()
+        self._first.wait(timeout=5.0)
+        self._t0 = time.monotonic()
         return self
 
     def __exit__(self, *exc):
-        self.lines = []
         if self.proc is not None:
             self.proc.terminate()
             try:
-                out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
-                out, _ = self.proc.communicate()
-            self.lines = [l for l in out.splitlines() if l.strip()]
+                self.proc.wait()
+            self._reader.join(timeout=5)
+            self.lines = [l for (t, l) in self._all if t >= self._t0]
 
     def summary(self):
         sm, mx, reasons = [], [], set()
@@ -297,6 +315,18 @@ def source_hash(files):
         code = "\n".join(line.rstrip() for line in text.splitlines() if line.strip())
         h.update(code.encode())
     return h.hexdigest()[:16]
+
+
+def launch_traffic(config, T):
+    """DRAM bytes of one launch of the dominant kernel at sequence length T,
+    or None when the sources changed since the capture.  A per-phase figure
+    scales to the T + 1 phases of one persistent launch."""
+    tr = TRAFFIC.get(config)
+    if not tr or tr["source_hash"] != source_hash(tr["files"]):
+        return None
+    if "bytes_per_phase" in tr:
+        return tr["bytes_per_phase"] * (T + 1)
+    return tr["bytes_per_launch"]
 
 
 def our_arm(args):
@@ -429,9 +459,7 @@ def our_arm(args):
     one_launch = traced["prep"][1] == 0  # the resident kernel: no tile preparation
     flops_total = (gate_flops_per_timestep(c) + head_flops_per_timestep(c)) * T * K * A
     achieved = flops_total / (gate_ms / 1e3) / 1e12 if gate_n else None
-    tr = TRAFFIC.get(args.config)
-    traffic = (tr["bytes_per_launch"]
-               if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
+    traffic = launch_traffic(args.config, T)
     launches = sum(v[1] for v in traced.values())
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
@@ -449,7 +477,7 @@ def our_arm(args):
             "seq_len": T,
             "l2": "flushed between timed steps (a 256 MiB buffer is written before each "
                   "step, inside the timed region)",
-            "parallelism": f"experts batched in one launch per timestep; {world} independent "
+            "parallelism": f"experts batched in one launch per sweep; {world} independent "
                            "replica(s), no collective",
         },
         "roofline": {
@@ -746,9 +774,7 @@ def body_arm(args):
     peaks, peak_src = measured_peaks()
     clocks = clk.summary()
     peak_kind, tensor_peak = applicable_peak(peaks, clocks)
-    tr = TRAFFIC.get(args.config)
-    traffic = (tr["bytes_per_launch"]
-               if tr and tr["source_hash"] == source_hash(tr["files"]) else None)
+    traffic = launch_traffic(args.config, T)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": W, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak",

@@ -63,6 +63,7 @@ constexpr int kStages = 4;       // ring slots: shared-memory operands and TMEM 
 // another, but more loader warps measured no faster: the copies are not
 // what bounds the launch.
 constexpr int kMmaWarp = 1;
+constexpr int kRelWarp = 3;      // publishes finished tasks on the phase counters
 constexpr int kZWarp0 = 4;       // Z generators: a multiple of 4 (TMEM lane quarters)
 constexpr int kZWarps = 8;       // (probe, lane quarter)
 constexpr int kEpiWarp0 = kZWarp0 + kZWarps;
@@ -240,7 +241,8 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // phases.  Roles:
 //   warp 0        loader: lanes 0 and 1 bulk-copy the stage's A tile and
 //                 operand group tile in one instruction;
-//   warps 2, 3    the embedding part of the next timestep's operand;
+//   warp 2        idle;
+//   warp 3        releaser: publishes finished tasks on the phase counters;
 //   warp 1        MMA issuer (lane 0 alone, so no warp-wide step sits
 //                 between consecutive stages): W x operand (shared memory)
 //                 and Z_p x operand (Z_p in tensor memory) per stage into one
@@ -266,11 +268,14 @@ struct Ctl {
   uint64_t red_bar;                // the head epilogue's rendezvous
   uint64_t mma_done;
   uint64_t task_full[kTaskSlots];  // the loader published the slot's task
+  uint64_t task_ready[kTaskSlots]; // the loader acquired the task's phase counters
   uint64_t task_empty[kTaskSlots]; // every other role has read it
   int task_gid[kTaskSlots];        // global task index, -1: no more tasks
+  int epi_done;                    // epilogue warps' finished tasks (monotonic)
   uint32_t tmem_slot;
   volatile int abort;
 };
+static_assert(sizeof(Ctl) <= 1024, "the control block sits in the 1 KB before the head buffer");
 
 // A wait that times out records SOMA_ERR_TIMEOUT in the status word and sets
 // the CTA's abort flag; a wait that is still pending sees the flag within 64
@@ -335,7 +340,7 @@ struct TcArgs {
   Sweep sw;
   TcGeom g;
   int t_first, t_last;   // the phases of this launch (phase t: the gate of t, the head of t - 1)
-  int gate_tasks, head_tasks, x_tiles;  // per phase
+  int gate_tasks, head_tasks;  // per phase
   const uint8_t* w16;    // [N][MT][S] A tiles
   const uint8_t* wo16;   // [N][2][Sh] A tiles
   uint8_t* op[2];        // [N][S][G] operand group tiles; phase t reads op[t % 2] = [x_t | h_{t-1}]
@@ -353,17 +358,18 @@ struct TcArgs {
   // extents for the index checks of the checked build (bytes of w16, wo16,
   // each op buffer and the byte batch; floats of cst, pm / ps, ply, params;
   // bytes of the dynamic shared memory)
-  size_t n_w16, n_wo16, n_op, n_bytes, n_cst, n_pm, n_ply, n_params;
+  const uint8_t* xall;   // [T][N][Sx][G] embedding-part tiles of every timestep
+  size_t n_w16, n_wo16, n_op, n_xall, n_bytes, n_cst, n_pm, n_ply, n_params;
   uint32_t smem_bytes;
 };
 
 // One phase t of the sweep: the gate tasks of timestep t (t < T) and the
-// head tasks of timestep t - 1 (t >= 1), both reading op[t % 2], and the
-// embedding-part tiles of timestep t + 1 (t + 1 < T), written into
-// op[(t + 1) % 2] with the gate tasks' h part.
+// head tasks of timestep t - 1 (t >= 1), both reading the h part of op[t %
+// 2]; the gate tasks write h_t into op[(t + 1) % 2].  The embedding part of
+// every timestep's operand is written before the sweep (xall).
 struct Phase {
   int t_gate, t_head;    // timesteps, -1: none
-  int n_gate, n_head, n_x;
+  int n_gate, n_head;
   const uint8_t* op_in;
   uint8_t* op_out;
 };
@@ -375,7 +381,6 @@ __device__ __forceinline__ Phase make_phase(const TcArgs& a, int t) {
   ph.t_head = t - 1;
   ph.n_gate = t < T ? a.gate_tasks : 0;
   ph.n_head = t >= 1 ? a.head_tasks : 0;
-  ph.n_x = t + 1 < T ? a.x_tiles : 0;
   ph.op_in = a.op[t & 1];
   ph.op_out = a.op[(t + 1) & 1];
   return ph;
@@ -405,28 +410,45 @@ __device__ __forceinline__ void decode_task(const TcArgs& a, int gid, int& t, in
 // reads it and releases the slot (one arrival per warp).  Returns the global
 // task index, -1 at the end, -2 after an abort.
 __device__ __forceinline__ int next_task(uint64_t* full, uint64_t* empty, const int* gids,
-                                         uint32_t& kt, volatile int* abort, int* status) {
+                                         uint32_t& kt, volatile int* abort, int* status,
+                                         bool release = true) {
   const int sl = (int)(kt % kTaskSlots);
   if (!wait_or_abort(&full[sl], (kt / kTaskSlots) & 1u, abort, status)) return -2;
   const int gid = *reinterpret_cast<const volatile int*>(&gids[sl]);
   __syncwarp(__activemask());
-  if ((threadIdx.x & 31) == 0) mbar_arrive(&empty[sl]);
+  if (release && (threadIdx.x & 31) == 0) mbar_arrive(&empty[sl]);
   ++kt;
   return gid;
+}
+
+// Waits (bounded) until the shared counter reaches `target`; an acquire at
+// CTA scope, so the writes that the counting warps made before their
+// release-add are visible to the caller afterwards.
+__device__ __forceinline__ bool wait_smem_count(int* ctr, int target, volatile int* abort,
+                                                int* status) {
+  const uint32_t addr = smem_u32(ctr);
+  for (uint32_t n = 0; n < (1u << 22); ++n) {
+    int v;
+    asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    if (v >= target) return true;
+    if ((n & 63u) == 63u && *abort) return false;
+    __nanosleep(32);
+  }
+  *abort = 1;
+  atomicCAS(status, 0, kStatusTimeout);
+  return false;
 }
 
 // Phase counters.  A launch may run several phases; tasks of phase t + 1
 // start on the groups that phase t has finished, without a grid-wide
 // barrier.  Per (expert, group): prod counts the writes finished into the
-// group's operand (one per epilogue warp of a gate task, one per
-// embedding-part tile), hd the head tasks finished (one per epilogue warp).
+// group's operand (one per epilogue warp of a gate task), hd the head tasks
+// finished (one per epilogue warp).
 // Through phase t (inclusive):
 __device__ __forceinline__ int prod_target(const TcArgs& a, int t) {
   if (t < 0) return 0;
-  const int T = a.sw.T;
-  const int gate_phases = min(t, T - 1) + 1;
-  const int x_phases = max(0, min(t, T - 2) + 1);
-  return kEpiWarps * a.g.MT * gate_phases + a.g.Sx * x_phases;
+  const int gate_phases = min(t, a.sw.T - 1) + 1;
+  return kEpiWarps * a.g.MT * gate_phases;
 }
 __device__ __forceinline__ int hd_target(const TcArgs& a, int t) {
   return t < 1 ? 0 : kEpiWarps * 2 * t;
@@ -460,13 +482,6 @@ __device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatil
   return ok != 0;
 }
 
-// The warp's writes so far are visible before the counter moves.
-__device__ __forceinline__ void release_count(int* ctr) {
-  __threadfence();
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) atomicAdd(ctr, 1);
-}
-
 // One task: (expert, row tile, probe group).  For the gate the row tile is
 // 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
 // half.
@@ -474,7 +489,8 @@ struct Task {
   bool head;
   int e, m, grp, p_valid, nst;
   const uint8_t* a;  // A tile of stage 0
-  const uint8_t* b;  // operand group tile of stage 0
+  const uint8_t* b;  // operand group tile of stage 0 (stages < Sx of a gate task: bx)
+  const uint8_t* bx; // gate: the timestep's embedding-part tile of stage 0
 };
 
 // A phase's task list runs group by group ((expert, probe group), in
@@ -503,6 +519,8 @@ __device__ __forceinline__ Task make_task(const TcArgs& a, const Phase& ph, int 
     T.a = a.w16 + (((size_t)T.e * g.MT + T.m) * g.S) * kTileA;
     T.b = ph.op_in + (((size_t)T.e * g.S) * g.G + T.grp) * g.tileB;
   }
+  T.bx = a.xall +
+         ((((size_t)max(ph.t_gate, 0) * g.n_experts + T.e) * g.Sx) * g.G + T.grp) * g.tileB;
   return T;
 }
 
@@ -888,13 +906,9 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-template <bool INF>
-__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int first, int stride);
-
 // grid: n_ctas persistent CTAs (at most one per SM, all resident: the launch
 // is cooperative), kThreads threads.  The CTAs share the tasks of phases
-// 0 .. T through the task counter; the embedding-part tiles of phases
-// t_first .. t_last are dealt statically.
+// 0 .. T through the task counter.
 // SPARSE: sparse probes; INF: the unperturbed layout (eps = 0, one sign).
 template <bool SPARSE, bool INF>
 __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
@@ -926,10 +940,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     mbar_init(&ctl->mma_done, 1);
     for (int q = 0; q < kTaskSlots; ++q) {
       mbar_init(&ctl->task_full[q], 1);
-      // the MMA issuer, the Z warps (when probes are generated) and the
-      // epilogue warps read every task
-      mbar_init(&ctl->task_empty[q], 1 + (do_z ? kZWarps : 0) + kEpiWarps);
+      mbar_init(&ctl->task_ready[q], 1);
+      // the MMA issuer, the Z warps (when probes are generated), the
+      // epilogue warps and the releaser read every task
+      mbar_init(&ctl->task_empty[q], 2 + (do_z ? kZWarps : 0) + kEpiWarps);
     }
+    ctl->epi_done = 0;
     mbar_fence_init();
   }
   if (warp == 0) tmem_alloc(&ctl->tmem_slot, kTmemCols);
@@ -970,13 +986,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       {
         const Task T = make_task<INF>(a, ph, task);
         if (t >= 1) {
+          // the copies read what phase t - 1 wrote into the group's operand;
+          // a gate task's epilogue also overwrites what phase t - 1 read
           const size_t c = (size_t)T.e * g.G + T.grp;
           if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
-              !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status)) {
+              !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
+              (!T.head && !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status))) {
             done = false;
             break;
           }
         }
+        // the epilogue starts on the task after this arrival, which passes on
+        // the acquire of the counters (CTA scope)
+        if (lane == 0) mbar_arrive(&ctl->task_ready[sl]);
         for (int st = 0; st < T.nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
@@ -990,11 +1012,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           __syncwarp();
           if (lane < 2) {
             uint8_t* dst = lane == 0 ? slot + SL.a_off : slot + SL.b_off;
-            const uint8_t* src =
-                lane == 0 ? T.a + (size_t)st * kTileA : T.b + (size_t)st * g.G * g.tileB;
+            const bool xs = !T.head && st < g.Sx;  // an embedding-part stage
+            const uint8_t* src = lane == 0 ? T.a + (size_t)st * kTileA
+                                           : (xs ? T.bx : T.b) + (size_t)st * g.G * g.tileB;
             const uint32_t nb = lane == 0 ? kTileA : g.tileB;
-            const uint8_t* gbase = lane == 1 ? ph.op_in : (T.head ? a.wo16 : a.w16);
-            const size_t gsize = lane == 1 ? a.n_op : (T.head ? a.n_wo16 : a.n_w16);
+            const uint8_t* gbase =
+                lane == 1 ? (xs ? a.xall : ph.op_in) : (T.head ? a.wo16 : a.w16);
+            const size_t gsize =
+                lane == 1 ? (xs ? a.n_xall : a.n_op) : (T.head ? a.n_wo16 : a.n_w16);
             if (SOMA_CHECK((size_t)(dst - dyn_smem) + nb <= a.smem_bytes &&
                                src >= gbase && (size_t)(src - gbase) + nb <= gsize,
                            status))
@@ -1071,29 +1096,32 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       mbar_wait(&ctl->mma_done, 0);
     }
     __syncwarp();
-  } else if (warp == 2 || warp == 3) {
-    // ------------------------------------------------- embedding-part tiles
-    // Tile j of phase t (the x part of op[(t + 1) % 2] for one (expert,
-    // stage, group)) belongs to CTA j % n_ctas, warp 2 + (j / n_ctas) % 2.
-    // It overwrites what phase t - 1 read: it waits until that phase's gate
-    // and head tasks of the group have finished.
-    bool alive = true;
-    for (int t = a.t_first; t <= a.t_last && alive; ++t) {
+  } else if (warp == kRelWarp) {
+    // --------------------------------------------------------------- releaser
+    // Publishes each task's operand writes (gate) or finished reads (head)
+    // on the group's phase counter once the CTA's epilogue warps are done
+    // with it: one gpu-scope fence and one add per task, off the epilogue
+    // warps' path.  The epilogue warps count their finished tasks in shared
+    // memory with a CTA-scope release; this warp's acquire of that count,
+    // then its fence, order their writes before the add.
+    uint32_t kt = 0;
+    for (int k = 0;; ++k) {
+      const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
+                                status);
+      if (gid < 0) break;
+      int t, task;
+      decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
-      int i = 0;
-      for (int j = blockIdx.x; j < ph.n_x; j += n_ctas, ++i) {
-        if ((i & 1) != warp - 2) continue;
-        const int grp = j % g.G, e = j / (g.G * g.Sx);
-        const size_t c = (size_t)e * g.G + grp;
-        if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
-            !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
-            !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status)) {
-          alive = false;
-          break;
-        }
-        xpart_block<INF>(a, ph.op_out, t + 1, j, lane, 32);
-        release_count(a.prod + c);
+      const Task T = make_task<INF>(a, ph, task);
+      const size_t c = (size_t)T.e * g.G + T.grp;
+      if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
+          !wait_smem_count(&ctl->epi_done, kEpiWarps * (k + 1), abort, status))
+        break;
+      if (lane == 0) {
+        __threadfence();
+        atomicAdd(T.head ? a.hd + c : a.prod + c, kEpiWarps);
       }
+      __syncwarp();
     }
   } else if (warp >= kZWarp0 && warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
@@ -1179,9 +1207,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // --------------------------------------------------------------- epilogue
     // A gate task of phase t overwrites what phase t - 1 read (op[(t + 1) %
     // 2]) and reads the cell states that phase t - 1 wrote, possibly in
-    // another CTA (the task lists of phase 0 and the later phases differ):
-    // it waits for that phase's group before its first access.  After each
-    // task the warp publishes its writes on the group's counter.
+    // another CTA: the warp starts on it once the loader has acquired the
+    // group's counters of phase t - 1 (task_ready).  After each task it
+    // counts itself done in shared memory, and the releaser publishes the
+    // task on the group's counter.
     const int ew = warp - kEpiWarp0;
     const int q4 = warp & 3;
     int k = 0;
@@ -1189,9 +1218,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     bool alive = true;
     uint32_t kt = 0;
     for (; alive; ++k) {
+      // the slot is released after the readiness wait, so the loader cannot
+      // publish the slot's next task (and arrive on task_ready again) first
+      const int sl = (int)(kt % kTaskSlots);
+      const uint32_t tpar = (kt / kTaskSlots) & 1u;
       const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
-                                status);
+                                status, false);
       if (gid < 0) break;
+      if (!wait_or_abort(&ctl->task_ready[sl], tpar, abort, status)) break;
+      if (lane == 0) mbar_arrive(&ctl->task_empty[sl]);
       int t, task;
       decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
@@ -1200,14 +1235,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         const int buf = k & 1;
         const size_t c = (size_t)T.e * g.G + T.grp;
         GatePre G;
-        // a gate task reads cell states and overwrites operand rows that
-        // other CTAs wrote or read in phase t - 1: the warp acquires both
-        // of the group's counters itself (the loader already waited for the
-        // first, so that wait is one load)
         if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
-            !wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status) ||
-            (!T.head && (!wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
-                         !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status)))) {
+            !wait_or_abort(&ctl->acc_full[buf], (uint32_t)(k >> 1) & 1u, abort, status)) {
           alive = false;
           break;
         }
@@ -1223,8 +1252,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           gate_finish<INF>(a, ph, T, tacc, q4, G);
         }
         tc_fence_before();
-        release_count(T.head ? a.hd + c : a.prod + c);
-        if (lane == 0) mbar_arrive(&ctl->acc_empty[buf]);
+        __syncwarp();
+        if (lane == 0) {
+          asm volatile("red.release.cta.shared::cta.add.s32 [%0], 1;" ::"r"(smem_u32(&ctl->epi_done))
+                       : "memory");
+          mbar_arrive(&ctl->acc_empty[buf]);
+        }
       }
     }
   }
@@ -1235,9 +1268,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
 
 // Embedding part of the operand of timestep t: per probe p of the group the
 // rows vbar = Emb[byte_t], dhat = z_emb[byte_t] (+-1, or 0) and eps^2 dhat.
-// Block `blk` of Sx * G * N writes one (expert, stage, group) tile.
+// Block `blk` of Sx * G * N writes one (expert, stage, group) tile of xall.
 template <bool INF>
-__device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int first, int stride) {
+__device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int first,
+                            int stride) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const int st = (blk / g.G) % g.Sx, grp = blk % g.G;
@@ -1245,7 +1279,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int fi
   const Layout& L = s.lay;
   const float* th = s.params + (int64_t)e * L.P;
   const float eps2 = s.eps * s.eps;
-  uint8_t* tile = op + (((size_t)e * g.S + st) * g.G + grp) * g.tileB;
+  uint8_t* tile = xall + ((size_t)t * g.n_experts * g.Sx * g.G + blk) * g.tileB;
   const int chunks = g.rowsB * (kKt / 8);
   for (int c = first; c < chunks; c += stride) {
     const int row = c / (kKt / 8), kc = c % (kKt / 8);
@@ -1293,15 +1327,18 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* op, int t, int blk, int fi
 #pragma unroll
       for (int j = 0; j < 8; ++j) v[j] = __float2half_rn(0.f);
     }
-    if (SOMA_CHECK((size_t)(tile - op) + kmajor_offset(row, 8 * kc, kKt) + 16 <= a.n_op, a.status))
+    if (SOMA_CHECK((size_t)(tile - xall) + kmajor_offset(row, 8 * kc, kKt) + 16 <= a.n_xall,
+                   a.status))
       *reinterpret_cast<uint4*>(tile + kmajor_offset(row, 8 * kc, kKt)) =
           *reinterpret_cast<const uint4*>(v);
   }
 }
 
+// Block b: tile b % (N * Sx * G) of timestep b / (N * Sx * G).
 template <bool INF>
-__global__ void xpart_kernel(const TcArgs a, uint8_t* op, int t) {
-  xpart_block<INF>(a, op, t, blockIdx.x, threadIdx.x, blockDim.x);
+__global__ void xpart_kernel(const TcArgs a, uint8_t* xall, int tiles) {
+  xpart_block<INF>(a, xall, (int)(blockIdx.x / tiles), (int)(blockIdx.x % tiles), threadIdx.x,
+                   blockDim.x);
 }
 
 // The probe-word table of one sweep (zbits_row): block b writes the 128 rows
@@ -1605,6 +1642,7 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.zb = 2 * N * n * (size_t)zbits_stages(g) * kZRows * sizeof(uint2);
   // phase counters: prod and hd per (expert, group), then the task counter
   z.cnt = (2 * N * (size_t)g.G + 1) * sizeof(int);
+  z.xall = (size_t)g.T * N * g.Sx * g.G * g.tileB;
   return z;
 }
 
@@ -1632,6 +1670,8 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.n_w16 = z.w16;
   a.n_wo16 = z.wo16;
   a.n_op = z.op;
+  a.xall = tb.xall;
+  a.n_xall = z.xall;
   a.n_bytes = (size_t)(s.batch_per_probe ? s.n_experts * s.n_pert : s.n_experts) * s.B_mem *
               (size_t)(s.T + 1);
   a.n_cst = z.cst / sizeof(float);
@@ -1646,7 +1686,6 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.next_task = tb.cnt + 2 * (size_t)g.n_experts * g.G;
   a.gate_tasks = g.n_experts * g.MT * g.G;
   a.head_tasks = g.n_experts * 2 * g.G;
-  a.x_tiles = g.n_experts * g.Sx * g.G;
   a.t_first = 0;
   a.t_last = s.T;
   a.total_tasks = (a.gate_tasks + a.head_tasks) * s.T;
@@ -1656,11 +1695,13 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   cudaMemsetAsync(tb.op[0], 0, z.op, stream);
   cudaMemsetAsync(tb.op[1], 0, z.op, stream);
   cudaMemsetAsync(tb.cnt, 0, z.cnt, stream);
-  const int xblocks = g.n_experts * g.Sx * g.G;
+  // the embedding part of every timestep's operand, before the sweep
+  const int xtiles = g.n_experts * g.Sx * g.G;
+  const unsigned xblocks = (unsigned)((size_t)xtiles * s.T);
   if (g.inf)
-    xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
+    xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, tb.xall, xtiles);
   else
-    xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, tb.op[0], 0);
+    xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, tb.xall, xtiles);
   if (s.eps != 0.f) {
     const unsigned zblocks = (unsigned)(a.n_zrows / kZRows);
     if (s.sparse)

@@ -171,9 +171,11 @@ WsPlan plan_sweep(const soma_dims& d, int n_experts, int n_pert, int n_sign, int
     if (zl.op > w.z.op) w.z.op = zl.op;
     if (zl.cst > w.z.cst) w.z.cst = zl.cst;
     if (zl.cnt > w.z.cnt) w.z.cnt = zl.cnt;
+    if (zl.xall > w.z.xall) w.z.xall = zl.xall;
   }
   for (size_t bytes :
-       {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, w.z.cnt, coef})
+       {w.z.w16, w.z.wo16, w.z.op, w.z.op, w.z.cst, w.z.pm, w.z.pm, w.z.ply, w.z.zb, w.z.cnt,
+        w.z.xall, coef})
     w.r.add(bytes);
   w.total = w.r.total();
   return w;
@@ -192,6 +194,7 @@ TcBuffers carve_tc(const WsPlan& w, void* ws) {
   tb.ply = reinterpret_cast<float*>(p + w.r.off[7]);
   tb.zbits = reinterpret_cast<uint2*>(p + w.r.off[8]);
   tb.cnt = reinterpret_cast<int*>(p + w.r.off[9]);
+  tb.xall = p + w.r.off[10];
   return tb;
 }
 

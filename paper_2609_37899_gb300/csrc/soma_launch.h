@@ -40,7 +40,7 @@ struct TcGeom {
 constexpr int kInfGroupSeqs = 128;
 
 struct TcSizes {
-  size_t w16, wo16, op, cst, pm, ply, zb, cnt;
+  size_t w16, wo16, op, cst, pm, ply, zb, cnt, xall;
 };
 
 struct TcBuffers {
@@ -53,6 +53,7 @@ struct TcBuffers {
   float* ply;      // target logits
   uint2* zbits;    // probe-word table of the sweep
   int* cnt;        // phase counters of the persistent kernel
+  uint8_t* xall;   // embedding part of the operand of every timestep of the sweep
 };
 
 TcGeom make_tc_geom(const Layout& lay, int n_experts, int n_pert, int B, int T, int B_mem);

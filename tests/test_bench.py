@@ -61,7 +61,26 @@ def test_traffic_entries_name_existing_sources():
     for name, t in bench.TRAFFIC.items():
         for f in t["files"]:
             assert os.path.exists(os.path.join(ROOT, "paper_2609_37899_gb300", "csrc", f)), (name, f)
-        assert t["bytes_per_launch"] > 0
+        assert t.get("bytes_per_launch", t.get("bytes_per_phase", 0)) > 0
+
+
+def test_per_phase_traffic_scales_with_the_phases_of_a_launch(monkeypatch):
+    monkeypatch.setattr(bench, "TRAFFIC", {
+        "a": {"bytes_per_phase": 10.0, "files": ["forward_tc.cu"],
+              "source_hash": bench.source_hash(["forward_tc.cu"])},
+        "b": {"bytes_per_launch": 7.0, "files": ["forward_tc.cu"], "source_hash": "stale"}})
+    assert bench.launch_traffic("a", 16) == 170.0
+    assert bench.launch_traffic("b", 16) is None
+    assert bench.launch_traffic("missing", 16) is None
+
+
+def test_clock_sampler_without_nvidia_smi(monkeypatch):
+    def no_smi(*a, **k):
+        raise OSError("no nvidia-smi")
+    monkeypatch.setattr(bench.subprocess, "Popen", no_smi)
+    with bench.ClockSampler(0) as clk:
+        pass
+    assert clk.summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
 
 
 @pytest.mark.parametrize("config", ["tiny", "body_tiny"])
