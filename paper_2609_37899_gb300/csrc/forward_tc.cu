@@ -260,6 +260,17 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // accumulated), acc_empty (its epilogue has read it), mma_done (all MMAs of
 // the CTA completed).  Every wait is bounded (wait_or_abort, mbar_wait).
 // ---------------------------------------------------------------------------
+// One task: (expert, row tile, probe group).  For the gate the row tile is
+// 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
+// half.
+struct Task {
+  bool head;
+  int e, m, grp, p_valid, nst;
+  const uint8_t* a;  // A tile of stage 0
+  const uint8_t* b;  // operand group tile of stage 0 (stages < Sx of a gate task: bx)
+  const uint8_t* bx; // gate: the timestep's embedding-part tile of stage 0
+};
+
 struct Ctl {
   uint64_t full[kStages];
   uint64_t slot_free[kStages];
@@ -271,6 +282,8 @@ struct Ctl {
   uint64_t task_ready[kTaskSlots]; // the loader acquired the task's phase counters
   uint64_t task_empty[kTaskSlots]; // every other role has read it
   int task_gid[kTaskSlots];        // global task index, -1: no more tasks
+  int task_t[kTaskSlots];          // its phase
+  Task task[kTaskSlots];           // and the task, decoded once by the loader
   int epi_done;                    // epilogue warps' finished tasks (monotonic)
   uint32_t tmem_slot;
   volatile int abort;
@@ -407,16 +420,20 @@ __device__ __forceinline__ void decode_task(const TcArgs& a, int gid, int& t, in
 }
 
 // The consumer side of the task ring: waits for the next published task,
-// reads it and releases the slot (one arrival per warp).  Returns the global
-// task index, -1 at the end, -2 after an abort.
-__device__ __forceinline__ int next_task(uint64_t* full, uint64_t* empty, const int* gids,
-                                         uint32_t& kt, volatile int* abort, int* status,
-                                         bool release = true) {
+// copies it (phase t and the decoded task) and releases the slot (one
+// arrival per warp) unless `release` is false.  Returns the global task
+// index, -1 at the end, -2 after an abort.
+__device__ __forceinline__ int next_task(Ctl* ctl, uint32_t& kt, volatile int* abort, int* status,
+                                         int& t, Task& T, bool release = true) {
   const int sl = (int)(kt % kTaskSlots);
-  if (!wait_or_abort(&full[sl], (kt / kTaskSlots) & 1u, abort, status)) return -2;
-  const int gid = *reinterpret_cast<const volatile int*>(&gids[sl]);
+  if (!wait_or_abort(&ctl->task_full[sl], (kt / kTaskSlots) & 1u, abort, status)) return -2;
+  const int gid = ctl->task_gid[sl];
+  if (gid >= 0) {
+    t = ctl->task_t[sl];
+    T = ctl->task[sl];
+  }
   __syncwarp(__activemask());
-  if (release && (threadIdx.x & 31) == 0) mbar_arrive(&empty[sl]);
+  if (release && (threadIdx.x & 31) == 0) mbar_arrive(&ctl->task_empty[sl]);
   ++kt;
   return gid;
 }
@@ -481,17 +498,6 @@ __device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatil
   asm volatile("fence.proxy.async.global;" ::: "memory");
   return ok != 0;
 }
-
-// One task: (expert, row tile, probe group).  For the gate the row tile is
-// 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
-// half.
-struct Task {
-  bool head;
-  int e, m, grp, p_valid, nst;
-  const uint8_t* a;  // A tile of stage 0
-  const uint8_t* b;  // operand group tile of stage 0 (stages < Sx of a gate task: bx)
-  const uint8_t* bx; // gate: the timestep's embedding-part tile of stage 0
-};
 
 // A phase's task list runs group by group ((expert, probe group), in
 // order): the group's two head tasks, then its gate tasks (row tiles
@@ -974,17 +980,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       if (lane == 0) gid = atomicAdd(a.next_task, 1);
       gid = __shfl_sync(0xffffffffu, gid, 0);
       const bool end = gid >= a.total_tasks;
+      int t = 0, task = 0;
+      if (!end) decode_task(a, gid, t, task);
+      const Phase ph = make_phase(a, t);
+      const Task T = make_task<INF>(a, ph, task);
       if (lane == 0) {
         ctl->task_gid[sl] = end ? -1 : gid;
+        ctl->task_t[sl] = t;
+        ctl->task[sl] = T;
         mbar_arrive(&ctl->task_full[sl]);
       }
       ++kt;
       if (end) break;
-      int t, task;
-      decode_task(a, gid, t, task);
-      const Phase ph = make_phase(a, t);
       {
-        const Task T = make_task<INF>(a, ph, task);
         if (t >= 1) {
           // the copies read what phase t - 1 wrote into the group's operand;
           // a gate task's epilogue also overwrites what phase t - 1 read
@@ -1064,13 +1072,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       RingPos rp = {0u, 0u};
       uint32_t kt = 0;
       for (int k = 0;; ++k) {
-        const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
-                                  status);
-        if (gid < 0) break;
-        int t, task;
-        decode_task(a, gid, t, task);
-        const Phase ph = make_phase(a, t);
-        const Task T = make_task<INF>(a, ph, task);
+        int t;
+        Task T;
+        if (next_task(ctl, kt, abort, status, t, T) < 0) break;
         const int buf = k & 1;
         if (k >= 2 &&
             !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
@@ -1106,13 +1110,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // then its fence, order their writes before the add.
     uint32_t kt = 0;
     for (int k = 0;; ++k) {
-      const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
-                                status);
-      if (gid < 0) break;
-      int t, task;
-      decode_task(a, gid, t, task);
-      const Phase ph = make_phase(a, t);
-      const Task T = make_task<INF>(a, ph, task);
+      int t;
+      Task T;
+      if (next_task(ctl, kt, abort, status, t, T) < 0) break;
       const size_t c = (size_t)T.e * g.G + T.grp;
       if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
           !wait_smem_count(&ctl->epi_done, kEpiWarps * (k + 1), abort, status))
@@ -1137,14 +1137,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       uint32_t gs = 0, kt = 0;
       bool alive = true;
       while (alive) {
-        const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
-                                  status);
-        if (gid < 0) break;
-        int t, task;
-        decode_task(a, gid, t, task);
-        const Phase ph = make_phase(a, t);
+        int t;
+        Task T;
+        if (next_task(ctl, kt, abort, status, t, T) < 0) break;
         {
-          const Task T = make_task<INF>(a, ph, task);
           const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
           // uniform over the warp
           const bool active =
@@ -1222,16 +1218,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       // publish the slot's next task (and arrive on task_ready again) first
       const int sl = (int)(kt % kTaskSlots);
       const uint32_t tpar = (kt / kTaskSlots) & 1u;
-      const int gid = next_task(ctl->task_full, ctl->task_empty, ctl->task_gid, kt, abort,
-                                status, false);
-      if (gid < 0) break;
+      int t;
+      Task T;
+      if (next_task(ctl, kt, abort, status, t, T, false) < 0) break;
       if (!wait_or_abort(&ctl->task_ready[sl], tpar, abort, status)) break;
       if (lane == 0) mbar_arrive(&ctl->task_empty[sl]);
-      int t, task;
-      decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
       {
-        const Task T = make_task<INF>(a, ph, task);
         const int buf = k & 1;
         const size_t c = (size_t)T.e * g.G + T.grp;
         GatePre G;
