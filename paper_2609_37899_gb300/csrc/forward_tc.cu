@@ -243,8 +243,8 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 //                 operand group tile in one instruction;
 //   warp 2        idle;
 //   warp 3        releaser: publishes finished tasks on the phase counters;
-//   warp 1        MMA issuer (lane 0 alone, so no warp-wide step sits
-//                 between consecutive stages): W x operand (shared memory)
+//   warp 1        MMA issuer (the whole warp waits, one elected thread
+//                 issues): W x operand (shared memory)
 //                 and Z_p x operand (Z_p in tensor memory) per stage into one
 //                 of two TMEM accumulator buffers;
 //   warps 4..11   Z generators: thread (probe, row) expands the raw probe
@@ -330,7 +330,10 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
                                          uint32_t idesc_w, uint32_t idesc_z, uint32_t dz1,
                                          volatile int* abort, int* status) {
   for (int st = 0; st < nst; ++st) {
-    if (!wait_or_abort(&full[rp.q], rp.ph, abort, status)) return false;
+    // the whole warp waits, so the descriptor words stay warp-uniform and
+    // one elected thread issues
+    const bool ready = wait_or_abort(&full[rp.q], rp.ph, abort, status);
+    if (__any_sync(0xffffffffu, !ready)) return false;
     tc_fence_after();
     // the accumulator block, the probe tiles of the slot and the operand
     // windows (rows of 128 bytes per 8-row group step) stay inside their
@@ -341,9 +344,12 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
                     status))
       return false;
     const uint32_t so = rp.q * slot_step;
-    issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.q,
-                    idesc_w, idesc_z, dz1, st > 0 ? 1u : 0u);
-    mma_commit(&slot_free[rp.q]);
+    if (elect_one()) {
+      issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.q,
+                      idesc_w, idesc_z, dz1, st > 0 ? 1u : 0u);
+      mma_commit(&slot_free[rp.q]);
+    }
+    __syncwarp();
     rp.next();
   }
   return true;
@@ -1053,7 +1059,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp walks the tasks and stages; one elected thread issues.
+    {
       const uint32_t idesc_z = idesc_f16_f32(128, 2 * g.Bp);
       // W covers the P probes of the group (2 Bp P columns); a group with
       // one valid probe still multiplies the whole window (the rows of the
@@ -1077,7 +1084,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         if (next_task(ctl, kt, abort, status, t, T) < 0) break;
         const int buf = k & 1;
         if (k >= 2 &&
-            !wait_or_abort(&ctl->acc_empty[buf], (uint32_t)((k >> 1) - 1) & 1u, abort, status))
+            __any_sync(0xffffffffu, !wait_or_abort(&ctl->acc_empty[buf],
+                                                   (uint32_t)((k >> 1) - 1) & 1u, abort, status)))
           break;
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)buf * kAccCols;
@@ -1093,10 +1101,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
           ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
                            slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
         if (!ok) break;
-        mma_commit(&ctl->acc_full[buf]);
+        if (elect_one()) mma_commit(&ctl->acc_full[buf]);
+        __syncwarp();
       }
       // every MMA of this CTA completes before its tensor memory is freed
-      mma_commit(&ctl->mma_done);
+      if (elect_one()) mma_commit(&ctl->mma_done);
+      __syncwarp();
       mbar_wait(&ctl->mma_done, 0);
     }
     __syncwarp();

@@ -139,6 +139,15 @@ __host__ __device__ __forceinline__ uint32_t idesc_f16_f32(int M, int N) {
 // Descriptor split into its two 32-bit words: the low word holds the start
 // address (bits 0..13, in 16-byte units) and LBO; moving a descriptor by a
 // byte offset d that keeps the address below 256 KB is lo + (d >> 4).
+// One thread of the (converged) warp: true in exactly one lane.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred;
+  asm volatile(
+      "{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(pred));
+  return pred != 0;
+}
+
 __device__ __forceinline__ void mma_f16_ss_lohi(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi,
                                                 uint32_t b_lo, uint32_t b_hi, uint32_t idesc,
                                                 uint32_t accumulate) {
