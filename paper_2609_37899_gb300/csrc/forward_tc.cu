@@ -57,7 +57,8 @@ using namespace tc;
 
 namespace {
 
-constexpr int kStages = 4;       // ring slots: shared-memory operands and TMEM probe tiles
+constexpr int kStages = 5;       // ring slots of the shared-memory operands (W and operand tiles)
+constexpr int kZSlots = 4;       // ring slots of the TMEM probe tiles (TMEM holds no more)
 // Each stage's two copies (W tile, operand tile) are one 2-lane bulk-copy
 // instruction of one loader warp.  The copies of one warp complete one after
 // another, but more loader warps measured no faster: the copies are not
@@ -79,7 +80,7 @@ constexpr uint32_t kLbo = 128;              // bytes between core matrices along
 constexpr uint32_t kAccCols = 128;          // one accumulator buffer: 2 Bp P <= 128 columns
 constexpr uint32_t kZCol0 = 2 * kAccCols;   // probe tiles: slot q at kZCol0 + 64 q (+ 32 p)
 constexpr uint32_t kTmemCols = 512;
-static_assert(kZCol0 + kStages * 64 <= kTmemCols, "probe tiles fit tensor memory");
+static_assert(kZCol0 + kZSlots * 64 <= kTmemCols, "probe tiles fit tensor memory");
 
 __device__ __forceinline__ uint32_t compact16(uint32_t x) {
   x &= 0x55555555u;
@@ -256,7 +257,9 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 //                 TMEM lanes of quarter w % 4 for probe group (w - 12) / 4.
 // Barriers: full (the slot's copies landed and its Z tiles are stored: the
 // loader's arrival with the copies' bytes and one arrival per Z warp, so the
-// issuer waits once per stage), slot_free (the slot's MMAs are done), acc_full (a buffer's task is
+// issuer waits once per stage), slot_free (the slot's MMAs are done), z_free
+// (the MMAs reading a probe-tile slot are done: shared memory holds five
+// stages, tensor memory four probe tiles), acc_full (a buffer's task is
 // accumulated), acc_empty (its epilogue has read it), mma_done (all MMAs of
 // the CTA completed).  Every wait is bounded (wait_or_abort, mbar_wait).
 // ---------------------------------------------------------------------------
@@ -274,6 +277,7 @@ struct Task {
 struct Ctl {
   uint64_t full[kStages];
   uint64_t slot_free[kStages];
+  uint64_t z_free[kZSlots];        // the MMAs reading a probe-tile slot are done
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t red_bar;                // the head epilogue's rendezvous
@@ -307,14 +311,16 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
-// Ring position of the next stage: slot q and the parity of its phase.
+// Ring position of the next stage: shared-memory slot q and the parity of
+// its phase, probe-tile slot zq.
 struct RingPos {
-  uint32_t q, ph;
+  uint32_t q, ph, zq;
   __device__ __forceinline__ void next() {
     if (++q == kStages) {
       q = 0;
       ph ^= 1u;
     }
+    if (++zq == kZSlots) zq = 0;
   }
 };
 
@@ -323,7 +329,7 @@ struct RingPos {
 // with a commit.
 // The probe count NP is fixed per task, so the loop carries no dispatch.
 template <int NP>
-__device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
+__device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free, uint64_t* z_free,
                                          RingPos& rp, int nst, uint32_t d, uint32_t tmem,
                                          uint32_t a_lo0, uint32_t b_lo0, uint32_t slot_step,
                                          uint32_t hi, uint32_t w_row, uint32_t z1_row,
@@ -339,15 +345,16 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free,
     // windows (rows of 128 bytes per 8-row group step) stay inside their
     // allocations
     if (!SOMA_CHECK((d & 0xFFFFu) + dz1 + (NP >= 2 ? dz1 : 0) <= 2 * kAccCols &&
-                        kZCol0 + 64u * rp.q + 32u * (NP > 0 ? NP : 1) <= kTmemCols &&
-                        rp.q < (uint32_t)kStages,
+                        kZCol0 + 64u * rp.zq + 32u * (NP > 0 ? NP : 1) <= kTmemCols &&
+                        rp.q < (uint32_t)kStages && rp.zq < (uint32_t)kZSlots,
                     status))
       return false;
     const uint32_t so = rp.q * slot_step;
     if (elect_one()) {
-      issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.q,
+      issue_stage<NP>(d, a_lo0 + so, b_lo0 + so, hi, w_row, z1_row, tmem + kZCol0 + 64u * rp.zq,
                       idesc_w, idesc_z, dz1, st > 0 ? 1u : 0u);
       mma_commit(&slot_free[rp.q]);
+      mma_commit(&z_free[rp.zq]);
     }
     __syncwarp();
     rp.next();
@@ -944,6 +951,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       mbar_init(&ctl->full[q], do_z ? 1 + kZWarps : 1);
       mbar_init(&ctl->slot_free[q], 1);
     }
+    for (int q = 0; q < kZSlots; ++q) mbar_init(&ctl->z_free[q], 1);
     for (int q = 0; q < 2; ++q) {
       mbar_init(&ctl->acc_full[q], 1);
       mbar_init(&ctl->acc_empty[q], kEpiWarps);
@@ -1076,7 +1084,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       const uint32_t w_row = (uint32_t)(g.Bp / 8) * grp_step;  // the W window starts at row Bp
       const uint32_t z1_row = (uint32_t)(4 * g.Bp / 8) * grp_step;
       const uint32_t dz1 = (uint32_t)(2 * g.Bp);
-      RingPos rp = {0u, 0u};
+      RingPos rp = {0u, 0u, 0u};
       uint32_t kt = 0;
       for (int k = 0;; ++k) {
         int t;
@@ -1092,13 +1100,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         const int np = do_z ? T.p_valid : 0;
         bool ok;
         if (np == 2)
-          ok = mma_task<2>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+          ok = mma_task<2>(ctl->full, ctl->slot_free, ctl->z_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
                            slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
         else if (np == 1)
-          ok = mma_task<1>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+          ok = mma_task<1>(ctl->full, ctl->slot_free, ctl->z_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
                            slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
         else
-          ok = mma_task<0>(ctl->full, ctl->slot_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
+          ok = mma_task<0>(ctl->full, ctl->slot_free, ctl->z_free, rp, T.nst, d, tmem, a_lo0, b_lo0,
                            slot_step, hi, w_row, z1_row, idesc_w, idesc_z, dz1, abort, status);
         if (!ok) break;
         if (elect_one()) mma_commit(&ctl->acc_full[buf]);
@@ -1177,19 +1185,22 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
             z_run_pairs<SPARSE>(n0.y, a0.y, zw + 16);
           }
           for (int st = 0; st < T.nst; ++st, ++gs) {
+            // the stage's shared-memory slot q (its full barrier) and
+            // probe-tile slot zq
             const int q = gs % kStages;
-            const uint32_t use = gs / kStages;
+            const int zq = gs % kZSlots;
+            const uint32_t zuse = gs / kZSlots;
             // after an abort the generators stop: an arrival on a phase that
             // can no longer complete would overfill it
-            if (gs >= kStages &&
-                !wait_or_abort(&ctl->slot_free[q], (use - 1) & 1u, abort, status)) {
+            if (gs >= kZSlots &&
+                !wait_or_abort(&ctl->z_free[zq], (zuse - 1) & 1u, abort, status)) {
               alive = false;
               break;
             }
             tc_fence_after();
             if (active &&
-                SOMA_CHECK(kZCol0 + 64u * (uint32_t)q + 32u * pz + 32u <= kTmemCols, status)) {
-              tmem_st32(trow + 64u * (uint32_t)q, zw);
+                SOMA_CHECK(kZCol0 + 64u * (uint32_t)zq + 32u * pz + 32u <= kTmemCols, status)) {
+              tmem_st32(trow + 64u * (uint32_t)zq, zw);
               if (st + 1 < T.nst) {
                 z_run_pairs<SPARSE>(n1.x, a1.x, zw);
                 z_run_pairs<SPARSE>(n1.y, a1.y, zw + 16);
