@@ -64,6 +64,7 @@ constexpr int kZSlots = 4;       // ring slots of the TMEM probe tiles (TMEM hol
 // another, but more loader warps measured no faster: the copies are not
 // what bounds the launch.
 constexpr int kMmaWarp = 1;
+constexpr int kFetchWarp = 2;    // takes tasks and acquires their phase counters
 constexpr int kRelWarp = 3;      // publishes finished tasks on the phase counters
 constexpr int kZWarp0 = 4;       // Z generators: a multiple of 4 (TMEM lane quarters)
 constexpr int kZWarps = 8;       // (probe, lane quarter)
@@ -242,7 +243,8 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // phases.  Roles:
 //   warp 0        loader: lanes 0 and 1 bulk-copy the stage's A tile and
 //                 operand group tile in one instruction;
-//   warp 2        idle;
+//   warp 2        fetcher: takes the next task from the global counter,
+//                 acquires its phase counters and publishes it;
 //   warp 3        releaser: publishes finished tasks on the phase counters;
 //   warp 1        MMA issuer (the whole warp waits, one elected thread
 //                 issues): W x operand (shared memory)
@@ -283,7 +285,6 @@ struct Ctl {
   uint64_t red_bar;                // the head epilogue's rendezvous
   uint64_t mma_done;
   uint64_t task_full[kTaskSlots];  // the loader published the slot's task
-  uint64_t task_ready[kTaskSlots]; // the loader acquired the task's phase counters
   uint64_t task_empty[kTaskSlots]; // every other role has read it
   int task_gid[kTaskSlots];        // global task index, -1: no more tasks
   int task_t[kTaskSlots];          // its phase
@@ -960,10 +961,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     mbar_init(&ctl->mma_done, 1);
     for (int q = 0; q < kTaskSlots; ++q) {
       mbar_init(&ctl->task_full[q], 1);
-      mbar_init(&ctl->task_ready[q], 1);
-      // the MMA issuer, the Z warps (when probes are generated), the
-      // epilogue warps and the releaser read every task
-      mbar_init(&ctl->task_empty[q], 2 + (do_z ? kZWarps : 0) + kEpiWarps);
+      // the loader, the MMA issuer, the Z warps (when probes are
+      // generated), the epilogue warps and the releaser read every task
+      mbar_init(&ctl->task_empty[q], 3 + (do_z ? kZWarps : 0) + kEpiWarps);
     }
     ctl->epi_done = 0;
     mbar_fence_init();
@@ -974,22 +974,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   tc_fence_after();
   const uint32_t tmem = ctl->tmem_slot;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- loader
-    // the whole warp walks the stages in order and waits for their slots;
-    // lanes 0 and 1 issue the stage's two copies together.  A task of phase
-    // t >= 1 first waits until phase t - 1 has finished writing its group's
-    // operand.
-    uint32_t gs = 0, kt = 0;
-    bool done = true;
+  if (warp == kFetchWarp) {
+    // --------------------------------------------------------------- fetcher
+    // Takes the tasks in global order, decodes each, acquires the group's
+    // phase counters of phase t - 1 and only then publishes the task to the
+    // CTA's other roles, up to kTaskSlots tasks ahead of the slowest of them:
+    // the counters' round trips stay off the loader's path.  Copies read
+    // what phase t - 1 wrote into the group's operand; a gate task's
+    // epilogue also overwrites what phase t - 1 read.
+    uint32_t kt = 0;
     for (;;) {
-      // take the next task in global order and publish it to the other roles
       const int sl = (int)(kt % kTaskSlots);
       if (kt >= kTaskSlots &&
-          !wait_or_abort(&ctl->task_empty[sl], ((kt / kTaskSlots) - 1) & 1u, abort, status)) {
-        done = false;
+          !wait_or_abort(&ctl->task_empty[sl], ((kt / kTaskSlots) - 1) & 1u, abort, status))
         break;
-      }
       int gid = 0;
       if (lane == 0) gid = atomicAdd(a.next_task, 1);
       gid = __shfl_sync(0xffffffffu, gid, 0);
@@ -998,6 +996,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       if (!end) decode_task(a, gid, t, task);
       const Phase ph = make_phase(a, t);
       const Task T = make_task<INF>(a, ph, task);
+      if (!end && t >= 1) {
+        const size_t c = (size_t)T.e * g.G + T.grp;
+        if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
+            !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
+            (!T.head && !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status)))
+          break;
+      }
+      // the arrival passes the acquire of the counters on (CTA scope)
       if (lane == 0) {
         ctl->task_gid[sl] = end ? -1 : gid;
         ctl->task_t[sl] = t;
@@ -1006,21 +1012,26 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
       }
       ++kt;
       if (end) break;
+    }
+  } else if (warp == 0) {
+    // ---------------------------------------------------------------- loader
+    // the whole warp walks the stages in order and waits for their slots;
+    // lanes 0 and 1 issue the stage's two copies together.
+    uint32_t gs = 0, kt = 0;
+    bool done = true;
+    for (;;) {
+      int t;
+      Task T;
+      const int gid = next_task(ctl, kt, abort, status, t, T);
+      if (gid < 0) {
+        done = gid == -1;
+        break;
+      }
+      const Phase ph = make_phase(a, t);
+      // the operand rows other CTAs wrote (generic proxy) before the
+      // fetcher's acquire are read here by bulk copies (async proxy)
+      asm volatile("fence.proxy.async.global;" ::: "memory");
       {
-        if (t >= 1) {
-          // the copies read what phase t - 1 wrote into the group's operand;
-          // a gate task's epilogue also overwrites what phase t - 1 read
-          const size_t c = (size_t)T.e * g.G + T.grp;
-          if (!SOMA_CHECK(c < (size_t)g.n_experts * g.G, status) ||
-              !wait_counter(a.prod + c, prod_target(a, t - 1), abort, status) ||
-              (!T.head && !wait_counter(a.hd + c, hd_target(a, t - 1), abort, status))) {
-            done = false;
-            break;
-          }
-        }
-        // the epilogue starts on the task after this arrival, which passes on
-        // the acquire of the counters (CTA scope)
-        if (lane == 0) mbar_arrive(&ctl->task_ready[sl]);
         for (int st = 0; st < T.nst; ++st, ++gs) {
           const int q = gs % kStages;
           const uint32_t use = gs / kStages;
@@ -1224,8 +1235,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     // --------------------------------------------------------------- epilogue
     // A gate task of phase t overwrites what phase t - 1 read (op[(t + 1) %
     // 2]) and reads the cell states that phase t - 1 wrote, possibly in
-    // another CTA: the warp starts on it once the loader has acquired the
-    // group's counters of phase t - 1 (task_ready).  After each task it
+    // another CTA: the fetcher published the task only after acquiring the
+    // group's counters of phase t - 1.  After each task it
     // counts itself done in shared memory, and the releaser publishes the
     // task on the group's counter.
     const int ew = warp - kEpiWarp0;
@@ -1235,15 +1246,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
     bool alive = true;
     uint32_t kt = 0;
     for (; alive; ++k) {
-      // the slot is released after the readiness wait, so the loader cannot
-      // publish the slot's next task (and arrive on task_ready again) first
-      const int sl = (int)(kt % kTaskSlots);
-      const uint32_t tpar = (kt / kTaskSlots) & 1u;
       int t;
       Task T;
-      if (next_task(ctl, kt, abort, status, t, T, false) < 0) break;
-      if (!wait_or_abort(&ctl->task_ready[sl], tpar, abort, status)) break;
-      if (lane == 0) mbar_arrive(&ctl->task_empty[sl]);
+      if (next_task(ctl, kt, abort, status, t, T) < 0) break;
       const Phase ph = make_phase(a, t);
       {
         const int buf = k & 1;
