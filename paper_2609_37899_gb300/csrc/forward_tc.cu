@@ -386,7 +386,8 @@ struct TcArgs {
   // each op buffer and the byte batch; floats of cst, pm / ps, ply, params;
   // bytes of the dynamic shared memory)
   const uint8_t* xall;   // [T][N][Sx][G] embedding-part tiles of every timestep
-  size_t n_w16, n_wo16, n_op, n_xall, n_bytes, n_cst, n_pm, n_ply, n_params;
+  uint2* xbits;          // [N][n][256][Ep / 32] probe words of the embedding rows
+  size_t n_w16, n_wo16, n_op, n_xall, n_xbits, n_bytes, n_cst, n_pm, n_ply, n_params;
   uint32_t smem_bytes;
 };
 
@@ -1332,8 +1333,15 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int 
                       a.status))
         continue;
       ProbeBits bits = {0u, 0u};
-      if (!mean && s.eps != 0.f)
-        bits = probe_bits(make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i), p0, s.sparse);
+      if (!mean && s.eps != 0.f) {
+        // the row's probe words, from the table emb_bits_kernel wrote
+        const size_t wi = (((size_t)e * s.n_pert + i) * 256 + y) * (g.Ep / 32) + k0 / 32;
+        if (SOMA_CHECK(wi < a.n_xbits, a.status)) {
+          const uint2 w = a.xbits[wi];
+          bits.neg = w.x >> (k0 & 31);
+          bits.act = w.y >> (k0 & 31);
+        }
+      }
       const float mag = e2 ? eps2 : 1.f;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -1350,6 +1358,22 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int 
                    a.status))
       *reinterpret_cast<uint4*>(tile + kmajor_offset(row, 8 * kc, kKt)) =
           *reinterpret_cast<const uint4*>(v);
+  }
+}
+
+// The probe words of the embedding rows, once per sweep: block (e, i),
+// thread y, words w of row y (parameters Emb[y][32 w .. 32 w + 31], natural
+// order; bits past E belong to the next row and are never used).
+__global__ void emb_bits_kernel(const TcArgs a) {
+  const TcGeom& g = a.g;
+  const Sweep& s = a.sw;
+  const int e = blockIdx.x / s.n_pert, i = blockIdx.x % s.n_pert, y = threadIdx.x;
+  const ProbeKey k = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
+  const int words = g.Ep / 32;
+  for (int w = 0; w < words; ++w) {
+    const size_t wi = (((size_t)e * s.n_pert + i) * 256 + y) * words + w;
+    const ProbeBits b = probe_bits(k, s.lay.emb + (int64_t)y * g.E + 32 * w, s.sparse);
+    if (SOMA_CHECK(wi < a.n_xbits, a.status)) a.xbits[wi] = make_uint2(b.neg, b.act);
   }
 }
 
@@ -1648,6 +1672,12 @@ TcGeom make_tc_geom_inf(const Layout& lay, int n_experts, int B, int T) {
   return g;
 }
 
+// The embedding rows' probe words ([N][n][256][Ep / 32] uint2), rounded to 1 KB.
+size_t xbits_bytes(const TcGeom& g) {
+  const size_t b = (size_t)g.n_experts * g.n_pert * 256 * (g.Ep / 32) * sizeof(uint2);
+  return (b + 1023) & ~(size_t)1023;
+}
+
 TcSizes tc_sizes(const TcGeom& g) {
   TcSizes z;
   const size_t N = (size_t)g.n_experts, n = (size_t)g.n_pert;
@@ -1661,7 +1691,8 @@ TcSizes tc_sizes(const TcGeom& g) {
   z.zb = 2 * N * n * (size_t)zbits_stages(g) * kZRows * sizeof(uint2);
   // phase counters: prod and hd per (expert, group), then the task counter
   z.cnt = (2 * N * (size_t)g.G + 1) * sizeof(int);
-  z.xall = (size_t)g.T * N * g.Sx * g.G * g.tileB;
+  // the embedding-part tiles, after the embedding rows' probe words
+  z.xall = xbits_bytes(g) + (size_t)g.T * N * g.Sx * g.G * g.tileB;
   return z;
 }
 
@@ -1689,8 +1720,10 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.n_w16 = z.w16;
   a.n_wo16 = z.wo16;
   a.n_op = z.op;
-  a.xall = tb.xall;
-  a.n_xall = z.xall;
+  a.xbits = reinterpret_cast<uint2*>(tb.xall);
+  a.n_xbits = (size_t)g.n_experts * g.n_pert * 256 * (g.Ep / 32);
+  a.xall = tb.xall + xbits_bytes(g);
+  a.n_xall = z.xall - xbits_bytes(g);
   a.n_bytes = (size_t)(s.batch_per_probe ? s.n_experts * s.n_pert : s.n_experts) * s.B_mem *
               (size_t)(s.T + 1);
   a.n_cst = z.cst / sizeof(float);
@@ -1717,10 +1750,13 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   // the embedding part of every timestep's operand, before the sweep
   const int xtiles = g.n_experts * g.Sx * g.G;
   const unsigned xblocks = (unsigned)((size_t)xtiles * s.T);
-  if (g.inf)
-    xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, tb.xall, xtiles);
-  else
-    xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, tb.xall, xtiles);
+  uint8_t* xall = tb.xall + xbits_bytes(g);
+  if (g.inf) {
+    xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, xall, xtiles);
+  } else {
+    if (s.eps != 0.f) emb_bits_kernel<<<g.n_experts * s.n_pert, 256, 0, stream>>>(a);
+    xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, xall, xtiles);
+  }
   if (s.eps != 0.f) {
     const unsigned zblocks = (unsigned)(a.n_zrows / kZRows);
     if (s.sparse)

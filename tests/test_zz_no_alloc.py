@@ -141,7 +141,7 @@ def test_static_step_large_then_small():
     # a call that fills much of the array, then a small one on another path:
     # the small call must not see what the large one left behind
     f = _static_fn()
-    big = (2, 64, 256, 32, 200, 32, 1e-3, 1e-2)
+    big = (2, 64, 256, 32, 32, 32, 1e-3, 1e-2)
     N, E, H, B, T, n, eps, lr = big
     assert api().workspace_bytes(E, H, N, n, B, T) > 16 << 20
     theta_b = inputs.init_params(N, E, H, seed=5, std=None)
