@@ -379,7 +379,7 @@ struct TcArgs {
   float* pm;             // [N*n*2][B_mem][T][2] head max partials
   float* ps;             // sum-exp partials
   float* ply;            // [N*n*2][B_mem][T] target logits
-  const uint2* zb;       // probe-word table (zbits_kernel), n_zrows rows, then activity words
+  const uint2* zb;       // probe-word table (zbits_block), n_zrows rows, then activity words
   size_t n_zrows;
   int* status;
   // extents for the index checks of the checked build (bytes of w16, wo16,
@@ -387,6 +387,7 @@ struct TcArgs {
   // bytes of the dynamic shared memory)
   const uint8_t* xall;   // [T][N][Sx][G] embedding-part tiles of every timestep
   uint2* xbits;          // [N][n][256][Ep / 32] probe words of the embedding rows
+  uint2* zb_out;         // the probe-word table, written before the sweep (a.zb reads it)
   size_t n_w16, n_wo16, n_op, n_xall, n_xbits, n_bytes, n_cst, n_pm, n_ply, n_params;
   uint32_t smem_bytes;
 };
@@ -1156,7 +1157,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
   } else if (warp >= kZWarp0 && warp < kEpiWarp0) {
     // --------------------------------------------------------- Z generators
     // Thread (probe gtid / 128, row gtid % 128 = TMEM lane).  The raw probe
-    // words of a stage come from the table zbits_kernel wrote before the
+    // words of a stage come from the table zbits_block wrote before the
     // sweep, loaded two stages ahead.  A stage's fp16 row is expanded while
     // the previous stage's slot is still busy; once its slot is free it is
     // stored, and the next stage is expanded while that store completes.
@@ -1334,7 +1335,7 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int 
         continue;
       ProbeBits bits = {0u, 0u};
       if (!mean && s.eps != 0.f) {
-        // the row's probe words, from the table emb_bits_kernel wrote
+        // the row's probe words, from the table emb_bits_block wrote
         const size_t wi = (((size_t)e * s.n_pert + i) * 256 + y) * (g.Ep / 32) + k0 / 32;
         if (SOMA_CHECK(wi < a.n_xbits, a.status)) {
           const uint2 w = a.xbits[wi];
@@ -1361,13 +1362,15 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int 
   }
 }
 
-// The probe words of the embedding rows, once per sweep: block (e, i),
-// thread y, words w of row y (parameters Emb[y][32 w .. 32 w + 31], natural
+// The probe words of the embedding rows, once per sweep: (expert e, probe
+// i), byte value y, words w of row y (parameters Emb[y][32 w .. 32 w + 31], natural
 // order; bits past E belong to the next row and are never used).
-__global__ void emb_bits_kernel(const TcArgs a) {
+// Block b of 2 N n (128 threads): (e, i) = b / 2, byte values y of half b % 2.
+__device__ void emb_bits_block(const TcArgs& a, int b) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
-  const int e = blockIdx.x / s.n_pert, i = blockIdx.x % s.n_pert, y = threadIdx.x;
+  const int pr = b >> 1;
+  const int e = pr / s.n_pert, i = pr % s.n_pert, y = 128 * (b & 1) + (int)threadIdx.x;
   const ProbeKey k = make_probe_key(s.seed, s.step, (uint32_t)e, (uint32_t)i);
   const int words = g.Ep / 32;
   for (int w = 0; w < words; ++w) {
@@ -1387,12 +1390,12 @@ __global__ void xpart_kernel(const TcArgs a, uint8_t* xall, int tiles) {
 // The probe-word table of one sweep (zbits_row): block b writes the 128 rows
 // of (expert, probe, tile stage) b, thread r the raw words of the stage's
 // 64 parameters of tile row r (and their activity words for sparse probes).
+// Blocks of 128 threads.
 template <bool SPARSE>
-__global__ void zbits_kernel(const TcArgs a, uint2* __restrict__ out) {
+__device__ void zbits_block(const TcArgs& a, uint2* __restrict__ out, size_t b) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const int TS = zbits_stages(g);
-  const size_t b = blockIdx.x;
   const int ts = (int)(b % TS), i = (int)((b / TS) % g.n_pert), e = (int)(b / TS / g.n_pert);
   const int r = threadIdx.x;
   Task T;
@@ -1422,16 +1425,14 @@ __global__ void zbits_kernel(const TcArgs a, uint2* __restrict__ out) {
 }
 
 // fp16 A tiles of the gate weights ([x part | h part], gate-major rows) and
-// of the head weights.
-// grid (MT * S + 2 * Sh, N), 128 threads: thread r writes row r of a tile.
-__global__ void prep_tiles_kernel(const TcArgs a) {
+// of the head weights: block (tix, e) of (MT * S + 2 * Sh, N), 128 threads,
+// thread r writes row r of a tile.
+__device__ void prep_tiles_block(const TcArgs& a, int tix, int e) {
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
   const Layout& L = s.lay;
-  const int e = blockIdx.y;
   const float* th = s.params + (int64_t)e * L.P;
   const int r = threadIdx.x;
-  const int tix = blockIdx.x;
   __align__(16) __half v[kKt];
   uint8_t* tile;
   if (tix < g.MT * g.S) {
@@ -1476,6 +1477,49 @@ __global__ void prep_tiles_kernel(const TcArgs a) {
   for (int kc = 0; kc < kKt / 8; ++kc)
     *reinterpret_cast<uint4*>(tile + kmajor_offset(r, 8 * kc, kKt)) =
         *reinterpret_cast<const uint4*>(v + 8 * kc);
+}
+
+// Everything a sweep needs before its embedding part and its persistent
+// launch, in one launch of 128-thread blocks: the fp16 weight tiles
+// (n_tiles blocks), the probe-word table (n_zb), the embedding rows' probe
+// words (n_eb), then the zeroing of both operand buffers and the phase
+// counters (the remaining blocks, grid-stride).
+struct PrepJobs {
+  int n_tiles, n_zb, n_eb;
+  uint4* op0;
+  uint4* op1;
+  size_t op_vec;  // uint4 per operand buffer
+  int* cnt;
+  int n_cnt;
+};
+
+template <bool SPARSE>
+__global__ void __launch_bounds__(128) sweep_prep_kernel(const TcArgs a, const PrepJobs j) {
+  int b = (int)blockIdx.x;
+  const int per_e = a.g.MT * a.g.S + 2 * a.g.Sh;
+  if (b < j.n_tiles) {
+    prep_tiles_block(a, b % per_e, b / per_e);
+    return;
+  }
+  b -= j.n_tiles;
+  if (b < j.n_zb) {
+    zbits_block<SPARSE>(a, a.zb_out, (size_t)b);
+    return;
+  }
+  b -= j.n_zb;
+  if (b < j.n_eb) {
+    emb_bits_block(a, b);
+    return;
+  }
+  b -= j.n_eb;
+  const size_t nz = gridDim.x - (size_t)(j.n_tiles + j.n_zb + j.n_eb);
+  const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+  for (size_t v = (size_t)b * blockDim.x + threadIdx.x; v < j.op_vec; v += nz * blockDim.x) {
+    j.op0[v] = zero;
+    j.op1[v] = zero;
+  }
+  if (b == 0)
+    for (int c = (int)threadIdx.x; c < j.n_cnt; c += blockDim.x) j.cnt[c] = 0;
 }
 
 // Per (expert, probe) pair: merge the two vocabulary halves into the NLL of
@@ -1715,6 +1759,7 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.ps = tb.ps;
   a.ply = tb.ply;
   a.zb = tb.zbits;
+  a.zb_out = tb.zbits;
   a.n_zrows = (size_t)g.n_experts * g.n_pert * zbits_stages(g) * kZRows;
   a.status = status;
   a.n_w16 = z.w16;
@@ -1742,28 +1787,33 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.t_last = s.T;
   a.total_tasks = (a.gate_tasks + a.head_tasks) * s.T;
 
+  // Two launches before the sweep: the weight tiles, the probe-word tables
+  // and the zeroed operand buffers and counters; then the embedding part of
+  // every timestep's operand (it reads the embedding rows' probe words).
+  PrepJobs j;
+  j.n_tiles = (g.MT * g.S + 2 * g.Sh) * g.n_experts;
+  j.n_zb = s.eps != 0.f ? (int)(a.n_zrows / kZRows) : 0;
+  j.n_eb = s.eps != 0.f && !g.inf ? 2 * g.n_experts * s.n_pert : 0;
+  j.op0 = reinterpret_cast<uint4*>(tb.op[0]);
+  j.op1 = reinterpret_cast<uint4*>(tb.op[1]);
+  j.op_vec = z.op / sizeof(uint4);
+  j.cnt = tb.cnt;
+  j.n_cnt = (int)(z.cnt / sizeof(int));
+  const size_t zb_need = (j.op_vec + 1023) / 1024;
+  const int zero_blocks = (int)(zb_need < 1 ? 1 : zb_need < 4096 ? zb_need : 4096);
+  const unsigned pblocks = (unsigned)(j.n_tiles + j.n_zb + j.n_eb + zero_blocks);
   trace_begin(SOMA_TRACE_PREP, stream);
-  prep_tiles_kernel<<<dim3(g.MT * g.S + 2 * g.Sh, g.n_experts), 128, 0, stream>>>(a);
-  cudaMemsetAsync(tb.op[0], 0, z.op, stream);
-  cudaMemsetAsync(tb.op[1], 0, z.op, stream);
-  cudaMemsetAsync(tb.cnt, 0, z.cnt, stream);
-  // the embedding part of every timestep's operand, before the sweep
+  if (s.sparse)
+    sweep_prep_kernel<true><<<pblocks, 128, 0, stream>>>(a, j);
+  else
+    sweep_prep_kernel<false><<<pblocks, 128, 0, stream>>>(a, j);
   const int xtiles = g.n_experts * g.Sx * g.G;
   const unsigned xblocks = (unsigned)((size_t)xtiles * s.T);
   uint8_t* xall = tb.xall + xbits_bytes(g);
-  if (g.inf) {
+  if (g.inf)
     xpart_kernel<true><<<xblocks, 128, 0, stream>>>(a, xall, xtiles);
-  } else {
-    if (s.eps != 0.f) emb_bits_kernel<<<g.n_experts * s.n_pert, 256, 0, stream>>>(a);
+  else
     xpart_kernel<false><<<xblocks, 128, 0, stream>>>(a, xall, xtiles);
-  }
-  if (s.eps != 0.f) {
-    const unsigned zblocks = (unsigned)(a.n_zrows / kZRows);
-    if (s.sparse)
-      zbits_kernel<true><<<zblocks, kZRows, 0, stream>>>(a, tb.zbits);
-    else
-      zbits_kernel<false><<<zblocks, kZRows, 0, stream>>>(a, tb.zbits);
-  }
   trace_end(SOMA_TRACE_PREP, stream);
 
   // every phase of the sweep in one cooperative launch: its CTAs wait on
