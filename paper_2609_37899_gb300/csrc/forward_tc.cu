@@ -1302,8 +1302,11 @@ __device__ void xpart_block(const TcArgs& a, uint8_t* xall, int t, int blk, int 
   const float eps2 = s.eps * s.eps;
   uint8_t* tile = xall + ((size_t)t * g.n_experts * g.Sx * g.G + blk) * g.tileB;
   const int chunks = g.rowsB * (kKt / 8);
+  static_assert(kKt / 8 == 8, "a core-matrix column is 8 chunks");
   for (int c = first; c < chunks; c += stride) {
-    const int row = c / (kKt / 8), kc = c % (kKt / 8);
+    // eight consecutive chunks fill the eight rows of one core matrix (128
+    // contiguous bytes of the tile); rowsB is a multiple of 8
+    const int row = 8 * (c / 64) + (c & 7), kc = (c >> 3) & 7;
     const int blkr = row / g.Bp, b = row % g.Bp;  // row block 0..3P-1, sequence
     const int p = blkr < 3 ? 0 : 1;
     const bool mean = blkr == row_mean(p), e2 = blkr == row_e2(p);
