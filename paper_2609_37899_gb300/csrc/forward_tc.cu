@@ -1172,6 +1172,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs
         Task T;
         if (next_task(ctl, kt, abort, status, t, T) < 0) break;
         {
+          // The next task's probe words come from DRAM (the table streams
+          // through L2 once per phase): when it is already published, its
+          // rows are prefetched into L2 now, a task ahead of their loads.
+          {
+            const int sn = (int)(kt % kTaskSlots);
+            if (mbar_test_wait(&ctl->task_full[sn], (kt / kTaskSlots) & 1u) &&
+                ctl->task_gid[sn] >= 0) {
+              const Task& Tn = ctl->task[sn];
+              const size_t rn = zbits_row(g, Tn.e, Tn.grp * g.P + pz, Tn.head, Tn.m) + (size_t)r;
+              if (pz < Tn.p_valid && rn + (size_t)kZRows * (Tn.nst - 1) < a.n_zrows) {
+                for (int st = 0; st < Tn.nst; ++st) {
+                  prefetch_l2(a.zb + rn + (size_t)kZRows * st);
+                  if (SPARSE) prefetch_l2(a.zb + a.n_zrows + rn + (size_t)kZRows * st);
+                }
+              }
+            }
+          }
           const size_t row0 = zbits_row(g, T.e, T.grp * g.P + pz, T.head, T.m) + (size_t)r;
           // uniform over the warp
           const bool active =
