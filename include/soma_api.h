@@ -233,11 +233,11 @@ const char* soma_status_string(int code);
  * device time and launch counts per kernel class.  Tracing is process-wide
  * and off by default; events are created on first use and reused. */
 enum {
-  SOMA_TRACE_GATE = 0,   /* recurrent gate GEMM + fused cell update, one launch per timestep */
+  SOMA_TRACE_GATE = 0,   /* recurrent gate GEMM + fused cell update and head (one launch per sweep) */
   SOMA_TRACE_HEAD = 1,   /* output head + log-softmax + NLL */
   SOMA_TRACE_REDUCE = 2, /* loss and coefficient reduction */
   SOMA_TRACE_UPDATE = 3, /* Philox-regenerating parameter update */
-  SOMA_TRACE_PREP = 4,   /* fp16 weight tiles and embedding operands */
+  SOMA_TRACE_PREP = 4,   /* fp16 weight tiles, probe-word tables, embedding operands */
   SOMA_TRACE_KINDS = 5
 };
 typedef struct soma_kernel_times {

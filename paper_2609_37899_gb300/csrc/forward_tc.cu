@@ -28,19 +28,22 @@
 // rounding (subnormal below |eps^2 dhat| = 6e-5) costs at most 3e-8 per
 // element, below the rounding of W vbar that C already carries.
 //
-// Per timestep t, one launch of one persistent kernel with two kinds of task:
+// One cooperative launch of one persistent kernel runs the whole sweep, in
+// phases t = 0 .. T with two kinds of task:
 //   gate tasks  (expert, 32-unit row tile, group of P probes), t < T: the
-//               W tile (shared memory) and the P probe tiles Z_p (generated
-//               from Philox straight into tensor memory, the A operand of a
-//               tcgen05.mma with A in TMEM) against the operand tiles of
-//               timestep t; epilogue: gates, cell update, the h part of the
-//               operand of t + 1;
+//               W tile (shared memory) and the P probe tiles Z_p (expanded
+//               from a per-sweep table of raw Philox words straight into
+//               tensor memory, the A operand of a tcgen05.mma with A in
+//               TMEM) against the operand tiles of timestep t; epilogue:
+//               gates, cell update, the h part of the operand of t + 1;
 //   head tasks  (expert, 128-row vocabulary half, probe group) of timestep
 //               t - 1, t >= 1: the same MMAs over the h part of the same
 //               operand (h_{t-1}), then per (sequence, sign) max and sum-exp
 //               partials of the half and the target logit.
-// Extra blocks of the launch write the embedding part of the operand of
-// t + 1.  A final reduction merges the two halves into per-target NLL and
+// Per-group phase counters in global memory order the phases without a grid
+// barrier.  Before the sweep, one launch writes the weight tiles and the
+// probe-word tables, and a second the embedding part of every timestep's
+// operand.  A final reduction merges the two halves into per-target NLL and
 // the per-(expert, probe) losses and coefficients.
 #include <cuda_fp16.h>
 
@@ -73,7 +76,7 @@ constexpr int kEpiWarps = 8;     // (probe, lane quarter)
 constexpr int kEpiProbeStep = kEpiWarps / 4;  // head: warp group eg runs probes eg, eg + 2, ...
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
 static_assert(kZWarp0 % 4 == 0 && kEpiWarp0 % 4 == 0, "warp w reads TMEM lane quarter w % 4");
-constexpr int kTaskSlots = 4;               // tasks a CTA's loader publishes ahead of the others
+constexpr int kTaskSlots = 4;               // tasks a CTA's fetcher publishes ahead of the others
 constexpr int kKt = 64;                     // K per stage (fp16 elements)
 constexpr uint32_t kTileA = 128 * kKt * 2;  // one 128-row A tile per stage
 constexpr uint32_t kSbo = kKt * 16;         // bytes between 8-row groups
@@ -238,18 +241,18 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // timestep t, see make_task); one CTA per SM takes tasks in global order
 // (phase by phase, decode_task) from a counter in global memory, so the
 // tasks whose inputs are ready first run first wherever an SM is free.  Its
-// loader publishes each task to the CTA's other roles through a small ring
+// fetcher publishes each task to the CTA's other roles through a small ring
 // of slots.  Phase counters in global memory replace a barrier between
 // phases.  Roles:
 //   warp 0        loader: lanes 0 and 1 bulk-copy the stage's A tile and
 //                 operand group tile in one instruction;
-//   warp 2        fetcher: takes the next task from the global counter,
-//                 acquires its phase counters and publishes it;
-//   warp 3        releaser: publishes finished tasks on the phase counters;
 //   warp 1        MMA issuer (the whole warp waits, one elected thread
 //                 issues): W x operand (shared memory)
 //                 and Z_p x operand (Z_p in tensor memory) per stage into one
 //                 of two TMEM accumulator buffers;
+//   warp 2        fetcher: takes the next task from the global counter,
+//                 acquires its phase counters and publishes it;
+//   warp 3        releaser: publishes finished tasks on the phase counters;
 //   warps 4..11   Z generators: thread (probe, row) expands the raw probe
 //                 words of the sweep's table into the fp16 +-1 row of its
 //                 probe tile and stores it into the slot's TMEM columns
@@ -263,7 +266,8 @@ __device__ __forceinline__ void issue_stage(uint32_t d, uint32_t a_lo, uint32_t 
 // (the MMAs reading a probe-tile slot are done: shared memory holds five
 // stages, tensor memory four probe tiles), acc_full (a buffer's task is
 // accumulated), acc_empty (its epilogue has read it), mma_done (all MMAs of
-// the CTA completed).  Every wait is bounded (wait_or_abort, mbar_wait).
+// the CTA completed), task_full / task_empty (the task ring).  Every wait is
+// bounded (wait_or_abort, mbar_wait, wait_counter, wait_smem_count).
 // ---------------------------------------------------------------------------
 // One task: (expert, row tile, probe group).  For the gate the row tile is
 // 32 hidden units (128 gate rows); for the head it is a 128-row vocabulary
@@ -284,11 +288,11 @@ struct Ctl {
   uint64_t acc_empty[2];
   uint64_t red_bar;                // the head epilogue's rendezvous
   uint64_t mma_done;
-  uint64_t task_full[kTaskSlots];  // the loader published the slot's task
+  uint64_t task_full[kTaskSlots];  // the fetcher published the slot's task
   uint64_t task_empty[kTaskSlots]; // every other role has read it
   int task_gid[kTaskSlots];        // global task index, -1: no more tasks
   int task_t[kTaskSlots];          // its phase
-  Task task[kTaskSlots];           // and the task, decoded once by the loader
+  Task task[kTaskSlots];           // and the task, decoded once by the fetcher
   int epi_done;                    // epilogue warps' finished tasks (monotonic)
   uint32_t tmem_slot;
   volatile int abort;
@@ -366,7 +370,6 @@ __device__ __forceinline__ bool mma_task(uint64_t* full, uint64_t* slot_free, ui
 struct TcArgs {
   Sweep sw;
   TcGeom g;
-  int t_first, t_last;   // the phases of this launch (phase t: the gate of t, the head of t - 1)
   int gate_tasks, head_tasks;  // per phase
   const uint8_t* w16;    // [N][MT][S] A tiles
   const uint8_t* wo16;   // [N][2][Sh] A tiles
@@ -928,12 +931,12 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-// grid: n_ctas persistent CTAs (at most one per SM, all resident: the launch
-// is cooperative), kThreads threads.  The CTAs share the tasks of phases
+// grid: one persistent CTA per SM at most (all resident: the launch is
+// cooperative), kThreads threads.  The CTAs share the tasks of phases
 // 0 .. T through the task counter.
 // SPARSE: sparse probes; INF: the unperturbed layout (eps = 0, one sign).
 template <bool SPARSE, bool INF>
-__global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a, int n_ctas) {
+__global__ void __launch_bounds__(kThreads, 1) tc_persistent_kernel(const TcArgs a) {
   extern __shared__ uint8_t dyn_smem[];
   const TcGeom& g = a.g;
   const Sweep& s = a.sw;
@@ -1803,8 +1806,6 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   a.next_task = tb.cnt + 2 * (size_t)g.n_experts * g.G;
   a.gate_tasks = g.n_experts * g.MT * g.G;
   a.head_tasks = g.n_experts * 2 * g.G;
-  a.t_first = 0;
-  a.t_last = s.T;
   a.total_tasks = (a.gate_tasks + a.head_tasks) * s.T;
 
   // Two launches before the sweep: the weight tiles, the probe-word tables
@@ -1856,7 +1857,7 @@ cudaError_t launch_forward_tc(const Sweep& s, const TcGeom& g, const TcBuffers& 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   trace_begin(SOMA_TRACE_GATE, stream);
-  e = cudaLaunchKernelEx(&cfg, kernel, a, ctas);
+  e = cudaLaunchKernelEx(&cfg, kernel, a);
   trace_end(SOMA_TRACE_GATE, stream);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
