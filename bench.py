@@ -47,9 +47,9 @@ TRAFFIC = {
     # profiles/tc_persistent_kernel_soma_n2.md: one persistent launch of the
     # SOMA N=2 shapes at T=16 (17 phases) captured; per phase, scaled by the
     # T + 1 phases of a launch
-    "soma_n2": {"bytes_per_phase": (2194.849e6 + 870.107136e6) / 17,
+    "soma_n2": {"bytes_per_phase": (2194.885e6 + 869.94816e6) / 17,
                 "files": ["forward_tc.cu", "tc_primitives.cuh", "soma_device.cuh"],
-                "source_hash": "e5edca2d4dac9f67"},
+                "source_hash": "97f08f55d5cc3326"},
     # profiles/res_kernel_soma_n256.md: one full-size launch (T=512)
     "soma_n256": {"bytes_per_launch": 39.452672e6 + 2048,
                   "files": ["resident.cu", "tc_primitives.cuh", "soma_device.cuh"],
