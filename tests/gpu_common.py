@@ -61,8 +61,8 @@ def rel_l2(a, b):
 
 
 def report(kind, value):
-    """Achieved error, printed for `pytest -s` (the margins quoted in the
-    design notes come from these lines)."""
+    """Achieved error, printed for `pytest -s`: one line per parity check,
+    so the margin of every tolerance can be read off a run."""
     print(f"PARITY {kind} {value:.3e}")
 
 
